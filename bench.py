@@ -1,0 +1,546 @@
+#!/usr/bin/env python
+"""Benchmark of the GB300 shard-decode path.
+
+Metric: INT4 shard decode tokens/s at 1 GB300, with the achieved HBM
+bandwidth of the dominant kernel against the measured peak.
+
+Default workload (the Llama-3.1-8B-shaped stage 1 of 2 decode): a 16-layer
+shard (hidden 4096, 32 q / 8 kv heads, head_dim 128, FFN 14336, uint4 group
+128), token ids looked up in the shard's 128256 x 4096 embedding, one request
+with a 72-token fp16 cache decoding one token per step for 256 steps,
+identity beam_idx, all-ones attention_mask.  A run of K steps chains
+ceil(K / 256) such requests back to back (each from its own 72-token cache),
+so every step is a step of that workload.  Weights are seeded synthetic
+(no checkpoints are available); the 1.81 GB of packed weights per step are
+far larger than L2, so no L2 flush is needed between steps.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl gb300|reference]
+                  [--config 8b-decode|8b-verify|8b-microbatch|70b-decode|70b-verify|tiny]
+
+Under torchrun each rank runs an independent replica on its own GPU
+(replicas only: the path has no exchange step) and rank 0 prints one JSON
+line.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+import synth  # noqa: E402
+
+METRIC = "INT4 shard decode tokens/s at 1 GB300; achieved HBM GB/s vs ~8 TB/s peak"
+SEED = 20260802
+CONFIGS = {
+    "8b-decode": dict(shape=synth.LLAMA8B_STAGE, prefill=72, steps_per_request=256, rows=1, n=1, tokens=True,
+                      workload="llama3.1-8b-stage1of2 16L decode: 1 request, 72-token prefill, 1 token/step, "
+                               "256 steps per request, identity beam_idx, all-ones mask"),
+    "8b-verify": dict(shape=synth.LLAMA8B_STAGE, prefill=512, steps_per_request=128, rows=1, n=5, tokens=False,
+                      workload="llama3.1-8b-stage1of2 16L speculative verify: 1 request, 512-token prefill, "
+                               "1+4 rows/step, Bernoulli(0.6) prefix accept, rejected rows masked, 128 steps"),
+    "8b-microbatch": dict(shape=synth.LLAMA8B_STAGE, prefill=None, steps_per_request=64, rows=8, n=1, tokens=False,
+                          workload="llama3.1-8b-stage1of2 16L micro-batch: 8 requests, lengths U{128..2048}, "
+                                   "random beam_idx permutation per step, 1 token/request/step, 64 steps"),
+    "70b-decode": dict(shape=synth.LLAMA70B_STAGE, prefill=4096, steps_per_request=64, rows=1, n=1, tokens=False,
+                       workload="llama3.1-70b-stage1of4 20L decode: 1 request, 4096-token prefill, 1 token/step, "
+                                "64 steps"),
+    "70b-verify": dict(shape=synth.LLAMA70B_STAGE, prefill=4096, steps_per_request=64, rows=1, n=5, tokens=False,
+                       workload="llama3.1-70b-stage1of4 20L speculative verify: 4096-token prefill, 1+4 rows/step, "
+                                "Bernoulli(0.6) prefix accept, 64 steps"),
+    "tiny": dict(shape=synth.TINY, prefill=72, steps_per_request=256, rows=1, n=1, tokens=True,
+                 workload="tiny 2L h256 decode: 72-token prefill, 1 token/step"),
+}
+KINDS = ["qkv", "o", "gate_up", "down", "attention", "rmsnorm", "prologue"]
+
+
+def log(*a):
+    print(*a, file=sys.stderr, flush=True)
+
+
+# ---------------------------------------------------------------------------
+# Workload: per-step inputs (host), built from the seeded generator
+# ---------------------------------------------------------------------------
+
+class Plan:
+    """Host-side step plan of one workload: for each step, n_new per row,
+    position ids, the attention mask rows, beam_idx and token ids or hidden
+    states; per-row prefill lengths; the byte counts of the step."""
+
+    def __init__(self, cfg_name: str, K: int, seed: int, request0: int = 0):
+        c = CONFIGS[cfg_name]
+        self.name, self.c, self.shape = cfg_name, c, c["shape"]
+        s = self.shape
+        self.B = c["rows"]
+        self.n = c["n"]
+        self.M = self.B * self.n
+        self.spr = c["steps_per_request"]
+        self.K = K
+        self.R = max(1, -(-K // self.spr))  # requests (each with its own cache)
+        if c["prefill"] is None:
+            self.prefill = [synth.lengths(seed + request0 + r, self.B, 128, 2048).tolist() for r in range(self.R)]
+        else:
+            self.prefill = [[c["prefill"]] * self.B for _ in range(self.R)]
+        self.cap = max(max(p) for p in self.prefill) + self.spr * self.n + 8
+        self.stride = self.cap
+        self.steps = []
+        for r in range(self.R):
+            lens = list(self.prefill[r])     # logical (cache) length per row
+            valid = [[1] * L for L in lens]  # live entries per row
+            pos = list(lens)                 # logical positions
+            for j in range(self.spr):
+                t = r * self.spr + j
+                if t >= K:
+                    break
+                beam = None
+                if cfg_name == "8b-microbatch":
+                    beam = synth.permutation(seed, t, self.B)
+                    lens = [lens[p] for p in beam]
+                    valid = [list(valid[p]) for p in beam]
+                    pos = [pos[p] for p in beam]
+                mask = np.zeros((self.B, self.stride), np.uint8)
+                positions = []
+                for b in range(self.B):
+                    L = lens[b]
+                    mask[b, :L] = np.array(valid[b], np.uint8)
+                    mask[b, L:L + self.n] = 1
+                    positions += list(range(pos[b], pos[b] + self.n))
+                step = dict(mask=mask, pos=np.array(positions, np.int32), beam=beam)
+                if c["tokens"]:
+                    step["tokens"] = synth.token_ids(s, seed, t, self.M)
+                else:
+                    step["hidden"] = synth.hidden_in(s, seed, t, self.M)
+                kv_read = 0
+                for b in range(self.B):
+                    # K and V of the entries attention must read: the live
+                    # cache entries and the new ones, in every layer
+                    kv_read += (sum(valid[b]) + self.n) * s.kv_bytes_per_token() * s.n_layers
+                step["kv_bytes"] = kv_read
+                self.steps.append(step)
+                acc = self.n
+                if self.n > 1:
+                    acc = 1 + synth.accepted_drafts(seed, t, self.n - 1)
+                for b in range(self.B):
+                    valid[b] += [1] * acc + [0] * (self.n - acc)
+                    lens[b] += self.n
+                    pos[b] += acc
+        self.step_of = [(t // self.spr, t % self.spr) for t in range(K)]
+
+    def weight_bytes(self) -> int:
+        return self.shape.packed_bytes_per_layer() * self.shape.n_layers
+
+    def alg_bytes(self, t: int) -> int:
+        """Algorithmic HBM bytes of step t: packed weights + scales + zeros,
+        K/V of the entries attention reads, embedding rows or hidden states in,
+        hidden states out, norm weights."""
+        s = self.shape
+        io = self.M * s.hidden * 2 * 2
+        norms = s.n_layers * 2 * s.hidden * 2
+        return self.weight_bytes() + self.steps[t]["kv_bytes"] + io + norms
+
+    def kind_bytes(self, kind: str) -> int:
+        """Algorithmic bytes of one launch of a projection kind."""
+        s = self.shape
+        names = {"qkv": ("q", "k", "v"), "o": ("o",), "gate_up": ("gate", "up"), "down": ("down",)}[kind]
+        total = 0
+        for nme in names:
+            r, c = s.matrix_shape(nme)
+            G = -(-c // s.group)
+            total += r * c // 2 + r * G * 2 + r * G // 2 + self.M * c * 2 + self.M * r * 2
+        return total
+
+
+# ---------------------------------------------------------------------------
+# GPU arm
+# ---------------------------------------------------------------------------
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str):
+        self.samples = []
+        self.proc = None
+        try:
+            cmd = ["nvidia-smi", "--query-gpu=" + self.FIELDS, "--format=csv,noheader,nounits", "-lms", "100"]
+            if gpu_id:
+                cmd += ["-i", gpu_id]
+            self.proc = subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except Exception as e:  # no nvidia-smi
+            log("clock sampling unavailable:", e)
+
+    def _read(self):
+        for line in self.proc.stdout:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) >= 9:
+                self.samples.append((time.time(), parts))
+
+    def stop(self):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self, t0: float, t1: float):
+        win = [p for (ts, p) in self.samples if t0 <= ts <= t1]
+        if len(win) < 3:  # short timed region: widen to the samples next to it
+            mid = 0.5 * (t0 + t1)
+            win = [p for (ts, p) in sorted(self.samples, key=lambda x: abs(x[0] - mid))[:5]]
+        if not win:
+            return None
+
+        def num(x):
+            try:
+                return float(x)
+            except ValueError:
+                return None
+
+        sm = [num(p[1]) for p in win if num(p[1]) is not None]
+        mx = [num(p[2]) for p in win if num(p[2]) is not None]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for p in win for i in range(4) if p[5 + i].lower().startswith("active")})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(win)}
+
+
+def measured_peaks():
+    try:
+        return json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+    except Exception:
+        return {}
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    for f in ("gemv.cu", "common.cuh", "kernels.h"):
+        h.update(open(os.path.join(ROOT, "paper_2608_19147_gb300", "csrc", f), "rb").read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(kind: str, cfg: str):
+    """DRAM bytes per launch from a committed ncu summary, if it was taken on
+    the current kernel source."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        data = json.load(open(path))
+        ent = data.get("%s/%s" % (cfg, kind))
+        if ent and ent.get("kernel_hash") == kernel_source_hash():
+            return ent.get("dram_bytes_per_launch")
+    except Exception:
+        pass
+    return None
+
+
+def run_gpu(args, rank: int, world: int):
+    import torch
+
+    import paper_2608_19147_gb300 as pkg
+
+    dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", "0")))
+    torch.cuda.set_device(dev)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.init_process_group("nccl", device_id=dev)
+    c = CONFIGS[args.config]
+    shape = c["shape"]
+    K, W = args.steps, max(3, args.warmup)
+    threads = max(1, (os.cpu_count() or 1) // max(1, int(os.environ.get("LOCAL_WORLD_SIZE", world))))
+    t_gen = time.time()
+    weights = synth.make_weights(shape, SEED, threads=threads)
+    log("weights generated in %.1fs (%.2f GB packed)" % (time.time() - t_gen, weights.packed_bytes() / 1e9))
+    plan = Plan(args.config, K, SEED)
+    warm = Plan(args.config, W, SEED + 1)
+    sh = pkg.shard_create(pkg.make_config(shape), weights.layers, weights.embedding)
+    stream = torch.cuda.current_stream(dev)
+    sptr = stream.cuda_stream
+
+    def load_states(p: Plan):
+        sts = []
+        for r in range(p.R):
+            st = pkg.kv_state_alloc(sh, p.B, p.cap)
+            for b in range(p.B):
+                for layer in range(shape.n_layers):
+                    k, v = synth.kv_prefill(shape, SEED + r, b, p.prefill[r][b], layer)
+                    pkg.kv_state_load(st, b, layer, k, v)
+            sts.append(st)
+        return sts
+
+    def stage(p: Plan):
+        """Per-step inputs resident on the device before timing."""
+        to = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+        d = dict(mask=to(np.stack([s["mask"] for s in p.steps])), pos=to(np.stack([s["pos"] for s in p.steps])))
+        if c["tokens"]:
+            d["tok"] = to(np.stack([s["tokens"] for s in p.steps]))
+        else:
+            d["hid"] = to(np.stack([s["hidden"] for s in p.steps]).view(np.int16))
+        if p.steps[0]["beam"] is not None:
+            d["beam"] = to(np.stack([s["beam"] for s in p.steps]))
+        d["out"] = torch.empty((p.M, shape.hidden), dtype=torch.int16, device=dev)
+        return d
+
+    def run_steps(p: Plan, sts, d, count):
+        n_new = [p.n] * p.B
+
+        def ptrs(key):  # device address of step t's slice, precomputed
+            if key not in d:
+                return [None] * count
+            a = d[key]
+            return [a.data_ptr() + t * a.stride(0) * a.element_size() for t in range(count)]
+
+        tok, hid, beam, pos, mask = ptrs("tok"), ptrs("hid"), ptrs("beam"), ptrs("pos"), ptrs("mask")
+        out = d["out"].data_ptr()
+        state_of = [sts[p.step_of[t][0]] for t in range(count)]
+        for t in range(count):
+            pkg.shard_step(sh, state_of[t], hid[t], tok[t], n_new, pos[t], mask[t], p.stride, beam[t], out, sptr)
+
+    # warm-up (own states, so the timed requests start from their prefills)
+    wst, wd = load_states(warm), stage(warm)
+    run_steps(warm, wst, wd, W)
+    torch.cuda.synchronize()
+    pkg.shard_sync_status(sh, sptr)
+    sts, d = load_states(plan), stage(plan)
+    gpu_id = ""
+    try:
+        gpu_id = str(torch.cuda.get_device_properties(dev).uuid)
+        if gpu_id and not gpu_id.startswith("GPU-"):
+            gpu_id = "GPU-" + gpu_id
+    except Exception:
+        gpu_id = ""
+    sampler = ClockSampler(gpu_id)
+    time.sleep(0.3)
+    # ---- timed region ----
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    w0 = time.time()
+    e0.record(stream)
+    run_steps(plan, sts, d, K)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    w1 = time.time()
+    if dist:
+        dist.barrier()
+    ms = e0.elapsed_time(e1)
+    sampler.stop()
+    clocks = sampler.summary(w0, w1)
+    pkg.shard_sync_status(sh, sptr)
+    if dist:
+        tt = torch.tensor([ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms = float(tt.item())
+    for st in sts + wst:
+        pkg.kv_state_free(st)
+
+    # ---- profiled pass: events around every launch of each kernel kind ----
+    prof_K = min(K, plan.spr)
+    pplan = Plan(args.config, prof_K, SEED + 2)
+    pst, pd = load_states(pplan), stage(pplan)
+    pkg.shard_debug_profile(sh, (1 << len(KINDS)) - 1)
+    torch.cuda.synchronize()
+    run_steps(pplan, pst, pd, prof_K)
+    torch.cuda.synchronize()
+    kernels = {}
+    for i, kname in enumerate(KINDS):
+        tot, n = pkg.shard_debug_profile_read(sh, i)
+        if n:
+            kernels[kname] = {"launches": n, "avg_us": 1000.0 * tot / n, "total_ms": tot}
+    pkg.shard_debug_profile(sh, 0)
+    for st in pst:
+        pkg.kv_state_free(st)
+    tot_all = sum(v["total_ms"] for v in kernels.values())
+    for kname, v in kernels.items():
+        v["share"] = v["total_ms"] / tot_all if tot_all else None
+        if kname in ("qkv", "o", "gate_up", "down"):
+            v["alg_bytes_per_launch"] = pplan.kind_bytes(kname)
+            v["achieved_gbs"] = v["alg_bytes_per_launch"] / (v["avg_us"] * 1e3)
+
+    # ---- end to end through the host-buffer entry point ----
+    eplan = Plan(args.config, K, SEED + 3)
+    est = load_states(eplan)
+    out = np.empty((eplan.M, shape.hidden), np.uint16)
+    h2d = d2h = 0
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    t0 = time.perf_counter()
+    for t in range(K):
+        r, _ = eplan.step_of[t]
+        s = eplan.steps[t]
+        pkg.shard_step_host(sh, est[r], s.get("hidden"), s.get("tokens"), [eplan.n] * eplan.B, s["pos"], s["mask"],
+                            s["beam"], out, sptr)
+    t1 = time.perf_counter()
+    s0 = eplan.steps[0]
+    h2d = (s0["mask"].nbytes + s0["pos"].nbytes + (s0["tokens"].nbytes if "tokens" in s0 else s0["hidden"].nbytes)
+           + (s0["beam"].nbytes if s0["beam"] is not None else 0))
+    d2h = out.nbytes
+    e2e_s = t1 - t0
+    if dist:
+        tt = torch.tensor([e2e_s], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        e2e_s = float(tt.item())
+    for st in est:
+        pkg.kv_state_free(st)
+    pkg.shard_destroy(sh)
+
+    if rank != 0:
+        if dist:
+            dist.destroy_process_group()
+        return
+    peaks = measured_peaks()
+    peak = peaks.get("hbm_gbs")
+    peak_note = "of measured" if peak else "of fallback"
+    if not peak:
+        peak = 6800.0
+    dominant = max((k for k in kernels if k in ("qkv", "o", "gate_up", "down")), key=lambda k: kernels[k]["total_ms"])
+    dk = kernels[dominant]
+    rows_per_step = plan.M
+    value = world * K * rows_per_step / (ms / 1e3)
+    step_bytes = sum(plan.alg_bytes(t) for t in range(K)) / K
+    launches_per_step = 1 + 7 * shape.n_layers
+    result = {
+        "metric": METRIC,
+        "value": value,
+        "unit": "tokens/s",
+        "n_gpus": world,
+        "steps": K,
+        "warmup": W,
+        "ms_per_step": ms / K,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "w4a16 (uint4 weights, fp16 activations, fp32 accumulate)",
+        "data": "synthetic (seeded Gaussian weights quantised to uint4; no checkpoints available)",
+        "config": {
+            "workload": c["workload"],
+            "shard": "%s: %d layers, hidden %d, %dq/%dkv heads, head_dim %d, ffn %d, group %d" % (
+                shape.name, shape.n_layers, shape.hidden, shape.n_heads, shape.n_kv_heads, shape.head_dim, shape.ffn,
+                shape.group),
+            "rows_per_step": rows_per_step,
+            "requests_chained": plan.R,
+            "l2": "no flush: each step streams %.2f GB of packed weights, far larger than the 129 MB L2" % (
+                plan.weight_bytes() / 1e9),
+            "parallelism": "replicas" if world > 1 else "single GPU",
+            "seed": SEED,
+        },
+        "step_alg_bytes": step_bytes,
+        "step_achieved_gbs": step_bytes / (ms / K * 1e6),
+        "roofline": {
+            "kernel": "gemv_%s" % dominant,
+            "bound": "hbm",
+            "achieved": dk["achieved_gbs"],
+            "peak": peak,
+            "unit": "GB/s",
+            "frac": dk["achieved_gbs"] / peak,
+            "peak_note": "%s (%s copy bandwidth); per-launch duration from CUDA events around each launch in a "
+                         "profiled pass of the same workload" % (peak_note, "MEASURED_PEAKS.json hbm_gbs"),
+            "traffic": profiled_traffic(dominant, args.config),
+        },
+        "kernels": kernels,
+        "e2e": {"value": world * K * rows_per_step / e2e_s, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h},
+        "gpu_launches": K * launches_per_step,
+        "clocks": clocks,
+    }
+    if world == 1 and not args.no_cpu_baseline:
+        result["cpu_baseline"] = cpu_baseline(args.config, weights, budget_s=args.cpu_budget)
+    print(json.dumps(result), flush=True)
+    if dist:
+        dist.destroy_process_group()
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle arm
+# ---------------------------------------------------------------------------
+
+def cpu_baseline(cfg_name: str, weights, budget_s: float = 20.0, max_steps: int = 256):
+    """The fp64 CPU oracle, as it stands, on a bounded sample of the workload:
+    the first steps of one request, until about budget_s seconds of work."""
+    import oracle
+
+    threads = os.cpu_count() or 1
+    oracle.set_threads(threads)
+    plan = Plan(cfg_name, max_steps, SEED)
+    shape = plan.shape
+    ref = oracle.OracleShard(shape, weights)
+    st = ref.state(plan.B, plan.cap)
+    for b in range(plan.B):
+        for layer in range(shape.n_layers):
+            k, v = synth.kv_prefill(shape, SEED + 0, b, plan.prefill[0][b], layer)
+            st.load(b, layer, k, v)
+    n = 0
+    t0 = time.perf_counter()
+    while n < min(max_steps, plan.spr):
+        s = plan.steps[n]
+        rc, _, _ = st.step([plan.n] * plan.B, s["pos"], s["mask"], hidden_in=s.get("hidden"),
+                           token_ids=s.get("tokens"), beam_idx=s["beam"])
+        assert rc == 0, rc
+        n += 1
+        if time.perf_counter() - t0 > budget_s:
+            break
+    el = time.perf_counter() - t0
+    return {"value": n * plan.M / el, "unit": "tokens/s", "cores": threads, "kind": "oracle",
+            "sample": "first %d steps of one request of the %s workload (%d rows/step), fp64 oracle, "
+                      "OpenMP over output rows with %d threads, %.1f s" % (n, cfg_name, plan.M, threads, el)}
+
+
+def run_reference(args, rank: int, world: int):
+    if rank != 0:
+        return
+    c = CONFIGS[args.config]
+    shape = c["shape"]
+    weights = synth.make_weights(shape, SEED)
+    budget = float(os.environ.get("REFERENCE_BUDGET_S", "120"))
+    cb = cpu_baseline(args.config, weights, budget_s=budget, max_steps=args.steps)
+    result = {
+        "metric": METRIC, "value": cb["value"], "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": 1000.0 * CONFIGS[args.config]["rows"] * c["n"] / cb["value"],
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f64", "data": "synthetic (seeded Gaussian weights quantised to uint4)",
+        "config": {"workload": c["workload"], "rows_per_step": c["rows"] * c["n"]},
+        "impl": "reference",
+        "cpu_baseline": cb,
+        "e2e": {"value": cb["value"], "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(result), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2048)
+    ap.add_argument("--warmup", type=int, default=16)
+    ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    ap.add_argument("--config", default="8b-decode", choices=list(CONFIGS))
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-budget", type=float, default=20.0)
+    args = ap.parse_args()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+    else:
+        run_gpu(args, rank, world)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,220 @@
+// Internal interface between the host side of libshard and its kernels.
+#pragma once
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+namespace shard {
+
+constexpr int kMaxTokens = 16;    // SHARD_MAX_TOKENS
+constexpr int kMaxRequests = 16;  // SHARD_MAX_REQUESTS
+
+// ---------------------------------------------------------------------------
+// Private INT4 weight layout ("unit stream").
+//
+// A fused projection with N output rows and K inputs is cut into row-blocks
+// of 64 rows and units of 128 inputs.  Unit (rb, ku) is one contiguous run of
+// unit_bytes(group) bytes at offset (rb * upr + ku) * unit_bytes, with
+// upr = ceil(K / 128) units per row-block, so the whole matrix is one linear
+// stream that bulk copies read front to back.
+//
+// Unit contents:
+//  [0, 4096)   codes: 8 fragment tiles of 512 bytes, tile ft = kc * 4 + rt for
+//              the 64-input half kc and the 16-row tile rt.  Lane l of a warp
+//              reads 16 bytes at ft * 512 + 16 * l: four 32-bit words, word j
+//              holding the 8 nibbles of that lane's m16n8k16 A fragment for
+//              virtual k-block j.  With gid = l / 4, tig = l % 4, h = j / 2,
+//              jj = j % 2 and k0 = 128 * ku + 64 * kc + 32 * h + 8 * tig + 4 * jj:
+//                bits  0..3 / 16..19 : row gid,     inputs k0,   k0+1   (a0)
+//                bits  4..7 / 20..23 : row gid + 8, inputs k0,   k0+1   (a1)
+//                bits  8..11/ 24..27 : row gid,     inputs k0+2, k0+3   (a2)
+//                bits 12..15/ 28..31 : row gid + 8, inputs k0+2, k0+3   (a3)
+//              (rows relative to the tile).  The matching B fragment of
+//              token n is then four consecutive activations x[n][k0..k0+3],
+//              so a lane's activations for a (kc, h) pair are 8 contiguous
+//              fp16 values: activations stay in natural [token][input] order.
+//  [4096, ..)  per group of the unit (128 / group groups, group in 32/64/128):
+//              64 fp16 scales then 64 uint8 zero points, each ordered
+//              [gid 0..7][rt 0..3][lo, hi] so one lane reads its 8 scales with
+//              one 16-byte load and its 8 zero points with one 8-byte load.
+// Rows past the real ones and inputs past K carry code 0 / zero point 0 /
+// scale 0, or (inputs of a real group past K) the group's zero point, so they
+// contribute exactly 0.
+// ---------------------------------------------------------------------------
+constexpr int kRowsPerBlock = 64;
+constexpr int kUnitK = 128;
+constexpr int kCodeBytes = 4096;
+constexpr int kMetaBytesPerGroup = 192;
+inline int unit_bytes_for_group(int group) { return kCodeBytes + (kUnitK / group) * kMetaBytesPerGroup; }
+
+enum OpKind { OP_QKV = 0, OP_O = 1, OP_GU = 2, OP_DOWN = 3, N_OPS = 4 };
+
+// Row order inside the fused projections:
+//  OP_QKV: q heads, then k heads, then v heads (d rows each).  Within a q or k
+//          head, 16-row tile jt holds rotary pairs: rows 0..7 are dims
+//          8*jt .. 8*jt+7 and rows 8..15 are dims d/2 + 8*jt .. +7.  v rows
+//          are in natural order.
+//  OP_GU:  16-row tile t holds gate rows 8t..8t+7 (rows 0..7) and up rows
+//          8t..8t+7 (rows 8..15).
+//  OP_O, OP_DOWN: natural order.
+struct OpDims {
+  int kind, Hq, Hkv, d, F, H;
+};
+
+// Natural output index of GPU row R of an op (q, k, v concatenated for QKV;
+// gate then up for GU), or -1 for a padding row.
+__host__ __device__ inline int natural_row(const OpDims& o, int R) {
+  int T = R >> 4, r = R & 15;
+  if (o.kind == OP_QKV) {
+    int tph = o.d >> 4, nq = o.Hq * tph, nk = o.Hkv * tph;
+    if (T < nq + nk) {
+      int base = T < nq ? 0 : o.Hq * o.d;
+      int t = T < nq ? T : T - nq;
+      int head = t / tph, jt = t % tph;
+      int dim = r < 8 ? 8 * jt + r : (o.d >> 1) + 8 * jt + (r - 8);
+      return base + head * o.d + dim;
+    }
+    int Rv = R - (o.Hq + o.Hkv) * o.d;
+    return Rv < o.Hkv * o.d ? (o.Hq + o.Hkv) * o.d + Rv : -1;
+  }
+  if (o.kind == OP_GU) {
+    int j = 8 * T + (r & 7);
+    if (j >= o.F) return -1;
+    return r < 8 ? j : o.F + j;
+  }
+  return R < o.H ? R : -1;
+}
+
+struct PackedOp {
+  uint8_t* units = nullptr;  // device
+  int n_rb = 0, upr = 0, unit_bytes = 0, group = 0, K = 0, Kp = 0, rows = 0;
+  size_t bytes = 0;
+  OpDims dims{};
+};
+
+// Step parameters, written on the device by the step prologue and read by
+// every later kernel of the step.
+struct StepParams {
+  int M, B, abort_step, pad0;
+  int tok_req[kMaxTokens];
+  int tok_idx[kMaxTokens];
+  int tok_pos[kMaxTokens];
+  int tok_slot[kMaxTokens];   // physical slot: phys_row * capacity + position in row
+  int req_tok0[kMaxRequests + 1];
+  int req_P[kMaxRequests];    // row length after the gather, before the append
+  int req_len[kMaxRequests];  // row length after the append
+  const uint8_t* mask;
+  int mask_stride, pad1;
+  uint16_t* hidden_out;
+  const int* bt;     // current beam table [n_rows][capacity]
+};
+
+enum EpiKind { EPI_STORE = 0, EPI_QKV = 1, EPI_RESID = 2, EPI_SWIGLU = 3 };
+
+struct EpiArgs {
+  int kind;
+  OpDims dims;
+  float* y;  // EPI_STORE: y[m][natural row], row stride y_ld
+  int y_ld;
+  float* q;                   // EPI_QKV: q fp32 [M][Hq*d]
+  uint16_t* kpool;            // EPI_QKV: this layer's K pool [n_rows][Hkv][cap][d]
+  uint16_t* vpool;
+  int cap;
+  const float2* rope;         // [max_position][d/2] (cos, sin)
+  float* x;                   // EPI_RESID: residual [M][H]
+  int write_out;              // EPI_RESID: also write fp16(x) to sp->hidden_out
+  uint16_t* h;                // EPI_SWIGLU: fp16 [M][h_ld]
+  int h_ld;
+};
+
+struct GemvArgs {
+  const uint8_t* units;
+  int n_rb, upr;
+  const uint16_t* act;  // fp16 activations [M][act_ld]
+  int act_ld;
+  int M;                // tokens when sp == nullptr
+  const StepParams* sp; // step parameters (nullptr on the standalone path)
+  float* partials;      // [grid][2][64][16] fp32 scratch
+  int* counters;        // [n_rb] zero-initialised, self-resetting
+  int* status;
+  EpiArgs ep;
+};
+
+// Launch geometry of the GEMV for a given token bucket (nt = 1: M <= 8,
+// nt = 2: M <= 16).
+int gemv_grid(int nt, int num_sms);
+size_t gemv_partials_floats(int grid);
+cudaError_t launch_gemv(const GemvArgs& a, int nt, int group, int grid, cudaStream_t s, bool pdl);
+// One-time per-device kernel attribute setup (dynamic shared memory limits).
+cudaError_t gemv_setup();
+
+struct NormArgs {
+  const float* x; int H;
+  const uint16_t* w;
+  float eps;
+  uint16_t* out; int out_ld;
+  int M;                 // when sp == nullptr
+  const StepParams* sp;
+};
+cudaError_t launch_rmsnorm(const NormArgs& a, cudaStream_t s, bool pdl);
+
+struct AttnArgs {
+  const float* q;        // [M][Hq*d]
+  const uint16_t* kpool; // layer's pools [n_rows][Hkv][cap][d]
+  const uint16_t* vpool;
+  int cap, Hq, Hkv, d, chunk, n_chunks;
+  float* part;           // scratch [B][Hkv][n_chunks][G*16][d+2]
+  int* counters;         // [B*Hkv]
+  uint16_t* out;         // fp16 [M][out_ld]
+  int out_ld;
+  const StepParams* sp;
+};
+cudaError_t launch_attention(const AttnArgs& a, int B, cudaStream_t s, bool pdl);
+size_t attention_part_floats(int B, int Hkv, int n_chunks, int G, int d);
+size_t attention_smem_bytes(int G, int chunk, int d);
+cudaError_t attention_setup(size_t max_smem);
+
+struct PrologueArgs {
+  int B, M;
+  int n_new[kMaxRequests];
+  int cursor[kMaxRequests];  // physical append position of each row
+  const int* beam_idx;   // dev or nullptr
+  const uint16_t* hidden_in;
+  const int* token_ids;
+  const int* position_ids;
+  const uint8_t* mask;
+  int mask_stride;
+  uint16_t* hidden_out;
+  const int* bt_src;
+  int* bt_dst;
+  int* lens;             // [n_rows] row lengths (updated)
+  int cap, max_position, vocab, H;
+  const uint16_t* embedding;
+  float* x;              // residual [M][H]
+  int* status;
+  StepParams* sp;
+};
+cudaError_t launch_prologue(const PrologueArgs& a, cudaStream_t s, bool pdl);
+
+// Weight repacking (one fused op; all source pointers device).
+// Source matrices of a fused op (q, k, v for OP_QKV; gate, up for OP_GU; one
+// matrix otherwise), in the boundary's packed format, on the device.
+struct RepackSrc {
+  const uint8_t* codes[3];
+  const uint16_t* scales[3];
+  const uint8_t* zeros[3];
+  int rows[3];
+};
+// rowmap: dev int [n_rb * 64]; entry = (source << 24) | source row, or -1.
+cudaError_t launch_repack(const PackedOp& op, const int* rowmap, const RepackSrc& src, cudaStream_t s);
+// Debug: dequantise an op back to natural order y[natural row][k] (fp32).
+cudaError_t launch_unpack(const PackedOp& op, float* out, int ld, cudaStream_t s);
+
+// KV utilities
+cudaError_t launch_kv_gather(const uint16_t* pool, int n_layers, size_t layer_stride, int Hkv, int cap, int d,
+                             const int* slots, int n, uint16_t* out /* [n_layers][n][Hkv][d] */, cudaStream_t s);
+cudaError_t launch_kv_scatter(uint16_t* pool, int n_layers, size_t layer_stride, int Hkv, int cap, int d, int row,
+                              const uint16_t* in /* [n_layers][n][Hkv][d] */, int n, cudaStream_t s);
+cudaError_t launch_fill_identity(int* bt, int n_rows, int cap, int row /* -1 = all */, cudaStream_t s);
+
+}  // namespace shard

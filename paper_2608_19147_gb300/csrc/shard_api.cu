@@ -1,0 +1,1046 @@
+// Host side of libshard: the C ABI declared in include/shard.h and
+// include/shard_debug.h.
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <map>
+#include <memory>
+#include <string>
+#include <vector>
+
+#include "../../include/shard.h"
+#include "../../include/shard_debug.h"
+#include "common.cuh"
+
+using namespace shard;
+
+namespace {
+
+thread_local std::string g_error;
+
+int fail(int code, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_error = buf;
+  return code;
+}
+
+#define CUDA_TRY(expr)                                                                        \
+  do {                                                                                        \
+    cudaError_t _e = (expr);                                                                  \
+    if (_e != cudaSuccess)                                                                    \
+      return fail(_e == cudaErrorMemoryAllocation ? SHARD_ENOMEM : SHARD_ECUDA, "%s: %s (%s:%d)", #expr, \
+                  cudaGetErrorString(_e), __FILE__, __LINE__);                                \
+  } while (0)
+
+template <class T>
+struct DevBuf {
+  T* p = nullptr;
+  size_t n = 0;
+  ~DevBuf() {
+    if (p) cudaFree(p);
+  }
+  cudaError_t alloc(size_t count) {
+    n = count;
+    return cudaMalloc(reinterpret_cast<void**>(&p), sizeof(T) * (count ? count : 1));
+  }
+};
+
+std::string status_message(int bits) {
+  std::string s;
+  if (bits & ST_BEAM_IDX) s += "beam_idx entry outside [0, B); ";
+  if (bits & ST_CAPACITY) s += "append would exceed the KV capacity; ";
+  if (bits & ST_MASK_NEW) s += "attention_mask is 0 at a new entry; ";
+  if (bits & ST_MASK_STRIDE) s += "mask_stride smaller than a row's length after the step; ";
+  if (bits & ST_POSITION) s += "position id outside [0, max_position); ";
+  if (bits & ST_TOKEN) s += "token id outside [0, vocab); ";
+  if (bits & ST_WAIT_TIMEOUT) s += "pipeline wait timed out; ";
+  return s;
+}
+
+}  // namespace
+
+struct GraphEntry {
+  cudaGraph_t graph = nullptr;      // kept alive: node handles refer to it
+  cudaGraphExec_t exec = nullptr;
+  cudaGraphNode_t prologue = nullptr;
+  cudaKernelNodeParams prologue_params{};  // as captured; kernelParams swapped per step
+};
+
+struct shard_s {
+  int device = 0;
+  shard_config cfg{};
+  int num_sms = 0;
+  int H = 0, Hq = 0, Hkv = 0, d = 0, F = 0, L = 0, dq = 0, dkv = 0;
+  int Kp_H = 0, Kp_dq = 0, Kp_F = 0;
+  std::vector<PackedOp> ops;      // [L][N_OPS]
+  uint8_t* weight_pool = nullptr;  // all units of all layers
+  size_t weight_bytes = 0;
+  uint16_t* norms = nullptr;       // [L][2][H]
+  uint16_t* embedding = nullptr;   // [V][H]
+  float2* rope = nullptr;          // [max_position][d/2]
+  // per-step work buffers (one set per shard)
+  float* x = nullptr;              // [16][H]
+  uint16_t* act_h = nullptr;       // [16][Kp_H]
+  uint16_t* act_attn = nullptr;    // [16][Kp_dq]
+  uint16_t* act_f = nullptr;       // [16][Kp_F]
+  float* q = nullptr;              // [16][dq]
+  float* partials = nullptr;
+  int* counters = nullptr;
+  int max_rb = 0;
+  int* status = nullptr;           // device status word
+  int* status_host = nullptr;      // pinned mirror (copied after each step)
+  StepParams* sp = nullptr;
+  int grid[3] = {0, 0, 0};         // GEMV grid per token bucket
+  bool use_graph = true, use_pdl = true;
+  cudaStream_t capture_stream = nullptr;
+  // staging for shard_step_host
+  void* pin = nullptr;
+  size_t pin_bytes = 0;
+  void* dstage = nullptr;
+  size_t dstage_bytes = 0;
+  std::vector<kvstate_s*> states;
+  // launch profiling (debug): CUDA events around launches of selected kinds
+  unsigned profile_mask = 0;
+  std::vector<cudaEvent_t> ev_pool;
+  std::vector<std::pair<int, std::pair<cudaEvent_t, cudaEvent_t>>> ev_used;
+};
+
+struct kvstate_s {
+  shard_s* sh = nullptr;
+  int n_rows = 0, cap = 0;
+  uint16_t* k = nullptr;  // [L][n_rows][Hkv][cap][d]
+  uint16_t* v = nullptr;
+  size_t layer_stride = 0;
+  int* bt[2] = {nullptr, nullptr};
+  int bt_cur = 0;
+  int* lens = nullptr;    // device [n_rows]
+  std::vector<int> cursor, len_host;
+  bool shared = false;    // rows may share entries (a beam gather ran)
+  bool poisoned = false;  // a step aborted on the device
+  int chunk = 64, n_chunks = 0;
+  float* attn_part = nullptr;
+  int* attn_counters = nullptr;
+  std::map<int, GraphEntry> graphs;
+};
+
+namespace {
+
+void free_state(kvstate_s* st) {
+  if (!st) return;
+  for (auto& kv : st->graphs) {
+    if (kv.second.exec) cudaGraphExecDestroy(kv.second.exec);
+    if (kv.second.graph) cudaGraphDestroy(kv.second.graph);
+  }
+  cudaFree(st->k);
+  cudaFree(st->v);
+  cudaFree(st->bt[0]);
+  cudaFree(st->bt[1]);
+  cudaFree(st->lens);
+  cudaFree(st->attn_part);
+  cudaFree(st->attn_counters);
+  delete st;
+}
+
+int round_up(int v, int m) { return (v + m - 1) / m * m; }
+
+// Row maps of the fused projections (see kernels.h): entry = (source << 24) | row.
+std::vector<int> build_rowmap(int kind, const shard_s& s, int n_rb) {
+  std::vector<int> rm((size_t)n_rb * kRowsPerBlock, -1);
+  if (kind == OP_QKV) {
+    const int tph = s.d / 16, half = s.d / 2;
+    int R = 0;
+    for (int src = 0; src < 2; ++src) {
+      const int heads = src == 0 ? s.Hq : s.Hkv;
+      for (int h = 0; h < heads; ++h)
+        for (int jt = 0; jt < tph; ++jt)
+          for (int r = 0; r < 16; ++r, ++R) {
+            const int dim = r < 8 ? 8 * jt + r : half + 8 * jt + (r - 8);
+            rm[R] = (src << 24) | (h * s.d + dim);
+          }
+    }
+    for (int e = 0; e < s.Hkv * s.d; ++e, ++R) rm[R] = (2 << 24) | e;
+  } else if (kind == OP_GU) {
+    const int tiles = (s.F + 7) / 8;
+    for (int t = 0; t < tiles; ++t)
+      for (int r = 0; r < 16; ++r) {
+        const int j = 8 * t + (r & 7);
+        if (j < s.F) rm[(size_t)t * 16 + r] = ((r < 8 ? 0 : 1) << 24) | j;
+      }
+  } else {
+    for (int R = 0; R < s.H; ++R) rm[R] = R;
+  }
+  return rm;
+}
+
+int op_rows(int kind, const shard_s& s) {
+  switch (kind) {
+    case OP_QKV: return (s.Hq + 2 * s.Hkv) * s.d;
+    case OP_GU: return ((s.F + 7) / 8) * 16;
+    default: return s.H;
+  }
+}
+int op_K(int kind, const shard_s& s) {
+  switch (kind) {
+    case OP_O: return s.dq;
+    case OP_DOWN: return s.F;
+    default: return s.H;
+  }
+}
+
+int nt_for(int M) { return M <= 8 ? 1 : 2; }
+
+// Profiled kinds: the four projections (OpKind), then these.
+enum { PK_ATTENTION = 4, PK_NORM = 5, PK_PROLOGUE = 6, PK_N = 7 };
+
+cudaEvent_t pool_event(shard_s* sh) {
+  if (sh->ev_pool.empty()) {
+    cudaEvent_t e = nullptr;
+    if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+    return e;
+  }
+  cudaEvent_t e = sh->ev_pool.back();
+  sh->ev_pool.pop_back();
+  return e;
+}
+
+// Brackets one launch with events when its kind is being profiled.
+struct ProfScope {
+  shard_s* sh;
+  int kind;
+  cudaStream_t s;
+  cudaEvent_t a = nullptr;
+  ProfScope(shard_s* sh_, int kind_, cudaStream_t s_) : sh(sh_), kind(kind_), s(s_) {
+    if (sh->profile_mask & (1u << kind)) {
+      a = pool_event(sh);
+      if (a) cudaEventRecord(a, s);
+    }
+  }
+  ~ProfScope() {
+    if (!a) return;
+    cudaEvent_t b = pool_event(sh);
+    if (!b) return;
+    cudaEventRecord(b, s);
+    sh->ev_used.push_back({kind, {a, b}});
+  }
+};
+
+// Enqueues the whole step after the prologue.
+int enqueue_layers(shard_s* sh, kvstate_s* st, int nt, cudaStream_t s, bool pdl) {
+  const int B = st->n_rows;
+  for (int l = 0; l < sh->L; ++l) {
+    PackedOp* ops = &sh->ops[(size_t)l * N_OPS];
+    const uint16_t* nrm = sh->norms + (size_t)l * 2 * sh->H;
+    NormArgs na{sh->x, sh->H, nrm, static_cast<float>(sh->cfg.rms_eps), sh->act_h, sh->Kp_H, 0, sh->sp};
+    {
+      ProfScope ps(sh, PK_NORM, s);
+      CUDA_TRY(launch_rmsnorm(na, s, pdl));
+    }
+    GemvArgs g{};
+    g.sp = sh->sp;
+    g.partials = sh->partials;
+    g.counters = sh->counters;
+    g.status = sh->status;
+    // q, k, v with RoPE and K/V append
+    g.units = ops[OP_QKV].units;
+    g.n_rb = ops[OP_QKV].n_rb;
+    g.upr = ops[OP_QKV].upr;
+    g.act = sh->act_h;
+    g.act_ld = sh->Kp_H;
+    g.ep = EpiArgs{};
+    g.ep.kind = EPI_QKV;
+    g.ep.dims = ops[OP_QKV].dims;
+    g.ep.q = sh->q;
+    g.ep.kpool = st->k + (size_t)l * st->layer_stride;
+    g.ep.vpool = st->v + (size_t)l * st->layer_stride;
+    g.ep.cap = st->cap;
+    g.ep.rope = sh->rope;
+    {
+      ProfScope ps(sh, OP_QKV, s);
+      CUDA_TRY(launch_gemv(g, nt, sh->cfg.group, std::min<long long>(sh->grid[nt], (long long)g.n_rb * g.upr), s, pdl));
+    }
+    // attention
+    AttnArgs aa{};
+    aa.q = sh->q;
+    aa.kpool = g.ep.kpool;
+    aa.vpool = g.ep.vpool;
+    aa.cap = st->cap;
+    aa.Hq = sh->Hq;
+    aa.Hkv = sh->Hkv;
+    aa.d = sh->d;
+    aa.chunk = st->chunk;
+    aa.n_chunks = st->n_chunks;
+    aa.part = st->attn_part;
+    aa.counters = st->attn_counters;
+    aa.out = sh->act_attn;
+    aa.out_ld = sh->Kp_dq;
+    aa.sp = sh->sp;
+    {
+      ProfScope ps(sh, PK_ATTENTION, s);
+      CUDA_TRY(launch_attention(aa, B, s, pdl));
+    }
+    // o projection + residual
+    g.units = ops[OP_O].units;
+    g.n_rb = ops[OP_O].n_rb;
+    g.upr = ops[OP_O].upr;
+    g.act = sh->act_attn;
+    g.act_ld = sh->Kp_dq;
+    g.ep = EpiArgs{};
+    g.ep.kind = EPI_RESID;
+    g.ep.dims = ops[OP_O].dims;
+    g.ep.x = sh->x;
+    {
+      ProfScope ps(sh, OP_O, s);
+      CUDA_TRY(launch_gemv(g, nt, sh->cfg.group, std::min<long long>(sh->grid[nt], (long long)g.n_rb * g.upr), s, pdl));
+    }
+    // MLP
+    na.w = nrm + sh->H;
+    {
+      ProfScope ps(sh, PK_NORM, s);
+      CUDA_TRY(launch_rmsnorm(na, s, pdl));
+    }
+    g.units = ops[OP_GU].units;
+    g.n_rb = ops[OP_GU].n_rb;
+    g.upr = ops[OP_GU].upr;
+    g.act = sh->act_h;
+    g.act_ld = sh->Kp_H;
+    g.ep = EpiArgs{};
+    g.ep.kind = EPI_SWIGLU;
+    g.ep.dims = ops[OP_GU].dims;
+    g.ep.h = sh->act_f;
+    g.ep.h_ld = sh->Kp_F;
+    {
+      ProfScope ps(sh, OP_GU, s);
+      CUDA_TRY(launch_gemv(g, nt, sh->cfg.group, std::min<long long>(sh->grid[nt], (long long)g.n_rb * g.upr), s, pdl));
+    }
+    g.units = ops[OP_DOWN].units;
+    g.n_rb = ops[OP_DOWN].n_rb;
+    g.upr = ops[OP_DOWN].upr;
+    g.act = sh->act_f;
+    g.act_ld = sh->Kp_F;
+    g.ep = EpiArgs{};
+    g.ep.kind = EPI_RESID;
+    g.ep.dims = ops[OP_DOWN].dims;
+    g.ep.x = sh->x;
+    g.ep.write_out = (l == sh->L - 1) ? 1 : 0;
+    {
+      ProfScope ps(sh, OP_DOWN, s);
+      CUDA_TRY(launch_gemv(g, nt, sh->cfg.group, std::min<long long>(sh->grid[nt], (long long)g.n_rb * g.upr), s, pdl));
+    }
+  }
+  return SHARD_OK;
+}
+
+int get_graph(shard_s* sh, kvstate_s* st, int nt, const PrologueArgs& pa, GraphEntry** out) {
+  auto it = st->graphs.find(nt);
+  if (it != st->graphs.end()) {
+    *out = &it->second;
+    return SHARD_OK;
+  }
+  cudaStream_t cs = sh->capture_stream;
+  CUDA_TRY(cudaStreamBeginCapture(cs, cudaStreamCaptureModeThreadLocal));
+  int rc = SHARD_OK;
+  cudaError_t e = launch_prologue(pa, cs, false);
+  if (e != cudaSuccess) rc = fail(SHARD_ECUDA, "prologue launch during capture: %s", cudaGetErrorString(e));
+  if (rc == SHARD_OK) rc = enqueue_layers(sh, st, nt, cs, sh->use_pdl);
+  cudaGraph_t graph = nullptr;
+  cudaError_t e2 = cudaStreamEndCapture(cs, &graph);
+  if (rc != SHARD_OK) {
+    if (graph) cudaGraphDestroy(graph);
+    return rc;
+  }
+  if (e2 != cudaSuccess) return fail(SHARD_ECUDA, "graph capture: %s", cudaGetErrorString(e2));
+  size_t n_roots = 0;
+  CUDA_TRY(cudaGraphGetRootNodes(graph, nullptr, &n_roots));
+  if (n_roots != 1) {
+    cudaGraphDestroy(graph);
+    return fail(SHARD_ECUDA, "captured step graph has %zu root nodes (expected 1)", n_roots);
+  }
+  GraphEntry ge;
+  ge.graph = graph;
+  e = cudaGraphGetRootNodes(graph, &ge.prologue, &n_roots);
+  if (e == cudaSuccess) e = cudaGraphKernelNodeGetParams(ge.prologue, &ge.prologue_params);
+  if (e == cudaSuccess) e = cudaGraphInstantiate(&ge.exec, graph, 0);
+  if (e != cudaSuccess) {
+    cudaGraphDestroy(graph);
+    return fail(SHARD_ECUDA, "graph instantiate: %s", cudaGetErrorString(e));
+  }
+  auto res = st->graphs.emplace(nt, ge);
+  *out = &res.first->second;
+  return SHARD_OK;
+}
+
+int check_pending_status(shard_s* sh) {
+  const int bits = *reinterpret_cast<volatile int*>(sh->status_host);
+  if (bits) {
+    *reinterpret_cast<volatile int*>(sh->status_host) = 0;
+    for (auto* st : sh->states) st->poisoned = true;
+    return fail(SHARD_EINVAL, "an earlier step was rejected on the device: %s", status_message(bits).c_str());
+  }
+  return SHARD_OK;
+}
+
+}  // namespace
+
+// ===========================================================================
+// C ABI
+// ===========================================================================
+
+extern "C" {
+
+const char* shard_last_error(void) { return g_error.c_str(); }
+
+int shard_create(const shard_config* cfg, const shard_weights_host* w, shard_t* out) {
+  if (!cfg || !w || !out || !w->layers) return fail(SHARD_EINVAL, "shard_create: null argument");
+  *out = nullptr;
+  const shard_config& c = *cfg;
+  if (c.n_layers < 1 || c.hidden < 16 || c.n_heads < 1 || c.n_kv_heads < 1 || c.head_dim < 16 || c.ffn < 1 ||
+      c.max_position < 1 || c.vocab < 0 || !(c.rms_eps >= 0) || !(c.rope_theta > 0))
+    return fail(SHARD_EINVAL, "shard_create: invalid dimensions");
+  if (c.n_heads % c.n_kv_heads) return fail(SHARD_EINVAL, "n_heads must be a multiple of n_kv_heads");
+  if (c.head_dim % 16) return fail(SHARD_EUNSUPPORTED, "head_dim must be a multiple of 16");
+  if (c.group != 32 && c.group != 64 && c.group != 128) return fail(SHARD_EUNSUPPORTED, "group must be 32, 64 or 128");
+  if (c.hidden % 8 || (c.n_heads * c.head_dim) % 8) return fail(SHARD_EUNSUPPORTED, "hidden must be a multiple of 8");
+  if (c.n_heads / c.n_kv_heads * kMaxTokens > 256) return fail(SHARD_EUNSUPPORTED, "n_heads / n_kv_heads must be <= 16");
+  if (c.vocab > 0 && !w->embedding) return fail(SHARD_EINVAL, "vocab > 0 needs an embedding");
+
+  auto sh = std::unique_ptr<shard_s>(new shard_s());
+  CUDA_TRY(cudaGetDevice(&sh->device));
+  CUDA_TRY(cudaDeviceGetAttribute(&sh->num_sms, cudaDevAttrMultiProcessorCount, sh->device));
+  CUDA_TRY(gemv_setup());
+  CUDA_TRY(attention_setup(attention_smem_bytes(c.n_heads / c.n_kv_heads, 64, c.head_dim)));
+  sh->cfg = c;
+  sh->H = c.hidden;
+  sh->Hq = c.n_heads;
+  sh->Hkv = c.n_kv_heads;
+  sh->d = c.head_dim;
+  sh->F = c.ffn;
+  sh->L = c.n_layers;
+  sh->dq = sh->Hq * sh->d;
+  sh->dkv = sh->Hkv * sh->d;
+  sh->Kp_H = round_up(sh->H, kUnitK);
+  sh->Kp_dq = round_up(sh->dq, kUnitK);
+  sh->Kp_F = round_up(sh->F, kUnitK);
+  const int ub = unit_bytes_for_group(c.group);
+
+  // Geometry of each op and the pool size.
+  sh->ops.resize((size_t)sh->L * N_OPS);
+  size_t total = 0;
+  for (int l = 0; l < sh->L; ++l)
+    for (int k = 0; k < N_OPS; ++k) {
+      PackedOp& op = sh->ops[(size_t)l * N_OPS + k];
+      op.rows = op_rows(k, *sh);
+      op.K = op_K(k, *sh);
+      op.Kp = round_up(op.K, kUnitK);
+      op.n_rb = (op.rows + kRowsPerBlock - 1) / kRowsPerBlock;
+      op.upr = op.Kp / kUnitK;
+      op.unit_bytes = ub;
+      op.group = c.group;
+      op.bytes = (size_t)op.n_rb * op.upr * ub;
+      op.dims = OpDims{k, sh->Hq, sh->Hkv, sh->d, sh->F, sh->H};
+      total += op.bytes;
+      sh->max_rb = std::max(sh->max_rb, op.n_rb);
+    }
+  sh->weight_bytes = total;
+  CUDA_TRY(cudaMalloc(&sh->weight_pool, total));
+  {
+    size_t off = 0;
+    for (auto& op : sh->ops) {
+      op.units = sh->weight_pool + off;
+      off += op.bytes;
+    }
+  }
+
+  // Upload and repack, op by op.
+  {
+    cudaStream_t s = nullptr;
+    size_t max_src = 0;
+    for (int k = 0; k < N_OPS; ++k) {
+      const PackedOp& op = sh->ops[k];
+      const int G = (op.K + c.group - 1) / c.group;
+      const size_t per_row = (size_t)(op.K + 1) / 2 + (size_t)G * 2 + (size_t)(G + 1) / 2;
+      max_src = std::max(max_src, per_row * (size_t)op.rows);
+    }
+    DevBuf<uint8_t> src;
+    DevBuf<int> rowmap;
+    CUDA_TRY(src.alloc(max_src + 3 * 256));
+    CUDA_TRY(rowmap.alloc((size_t)sh->max_rb * kRowsPerBlock));
+    for (int l = 0; l < sh->L; ++l) {
+      const shard_layer_host& lw = w->layers[l];
+      for (int k = 0; k < N_OPS; ++k) {
+        PackedOp& op = sh->ops[(size_t)l * N_OPS + k];
+        int mats[3] = {-1, -1, -1}, nm = 0;
+        int rows[3] = {0, 0, 0};
+        if (k == OP_QKV) {
+          mats[0] = SHARD_Q; mats[1] = SHARD_K; mats[2] = SHARD_V; nm = 3;
+          rows[0] = sh->dq; rows[1] = sh->dkv; rows[2] = sh->dkv;
+        } else if (k == OP_GU) {
+          mats[0] = SHARD_GATE; mats[1] = SHARD_UP; nm = 2;
+          rows[0] = rows[1] = sh->F;
+        } else {
+          mats[0] = (k == OP_O) ? SHARD_O : SHARD_DOWN; nm = 1;
+          rows[0] = sh->H;
+        }
+        const int G = (op.K + c.group - 1) / c.group;
+        const size_t cb = (size_t)(op.K + 1) / 2, sb = (size_t)G * 2, zb = (size_t)(G + 1) / 2;
+        RepackSrc rs{};
+        size_t off = 0;
+        for (int i = 0; i < nm; ++i) {
+          const shard_matrix_host& m = lw.w[mats[i]];
+          if (!m.codes || !m.scales || !m.zeros) return fail(SHARD_EINVAL, "layer %d matrix %d: null pointer", l, mats[i]);
+          auto put = [&](const void* hp, size_t bytes) -> uint8_t* {
+            off = (off + 255) / 256 * 256;
+            uint8_t* dp = src.p + off;
+            off += bytes;
+            return cudaMemcpy(dp, hp, bytes, cudaMemcpyHostToDevice) == cudaSuccess ? dp : nullptr;
+          };
+          rs.codes[i] = put(m.codes, cb * rows[i]);
+          rs.scales[i] = reinterpret_cast<const uint16_t*>(put(m.scales, sb * rows[i]));
+          rs.zeros[i] = put(m.zeros, zb * rows[i]);
+          rs.rows[i] = rows[i];
+          if (!rs.codes[i] || !rs.scales[i] || !rs.zeros[i]) return fail(SHARD_ECUDA, "weight upload failed");
+        }
+        std::vector<int> rm = build_rowmap(k, *sh, op.n_rb);
+        CUDA_TRY(cudaMemcpy(rowmap.p, rm.data(), rm.size() * sizeof(int), cudaMemcpyHostToDevice));
+        CUDA_TRY(launch_repack(op, rowmap.p, rs, s));
+        CUDA_TRY(cudaDeviceSynchronize());
+      }
+    }
+  }
+
+  // Norm weights, embedding, rotary table.
+  CUDA_TRY(cudaMalloc(&sh->norms, sizeof(uint16_t) * (size_t)sh->L * 2 * sh->H));
+  for (int l = 0; l < sh->L; ++l) {
+    if (!w->layers[l].attn_norm || !w->layers[l].ffn_norm) return fail(SHARD_EINVAL, "layer %d: null norm", l);
+    CUDA_TRY(cudaMemcpy(sh->norms + (size_t)l * 2 * sh->H, w->layers[l].attn_norm, sizeof(uint16_t) * sh->H,
+                        cudaMemcpyHostToDevice));
+    CUDA_TRY(cudaMemcpy(sh->norms + (size_t)l * 2 * sh->H + sh->H, w->layers[l].ffn_norm, sizeof(uint16_t) * sh->H,
+                        cudaMemcpyHostToDevice));
+  }
+  if (c.vocab > 0) {
+    CUDA_TRY(cudaMalloc(&sh->embedding, sizeof(uint16_t) * (size_t)c.vocab * sh->H));
+    CUDA_TRY(cudaMemcpy(sh->embedding, w->embedding, sizeof(uint16_t) * (size_t)c.vocab * sh->H,
+                        cudaMemcpyHostToDevice));
+  }
+  {
+    // cos/sin of pos * theta^(-2i/d), computed in double, stored as fp32.
+    const int half = sh->d / 2;
+    std::vector<float2> tab((size_t)c.max_position * half);
+    for (int p = 0; p < c.max_position; ++p)
+      for (int i = 0; i < half; ++i) {
+        const double ang = (double)p * std::pow(c.rope_theta, -2.0 * i / sh->d);
+        tab[(size_t)p * half + i] = make_float2((float)std::cos(ang), (float)std::sin(ang));
+      }
+    CUDA_TRY(cudaMalloc(&sh->rope, sizeof(float2) * tab.size()));
+    CUDA_TRY(cudaMemcpy(sh->rope, tab.data(), sizeof(float2) * tab.size(), cudaMemcpyHostToDevice));
+  }
+
+  // Work buffers.
+  CUDA_TRY(cudaMalloc(&sh->x, sizeof(float) * kMaxTokens * sh->H));
+  CUDA_TRY(cudaMalloc(&sh->act_h, sizeof(uint16_t) * kMaxTokens * sh->Kp_H));
+  CUDA_TRY(cudaMalloc(&sh->act_attn, sizeof(uint16_t) * kMaxTokens * sh->Kp_dq));
+  CUDA_TRY(cudaMalloc(&sh->act_f, sizeof(uint16_t) * kMaxTokens * sh->Kp_F));
+  CUDA_TRY(cudaMemset(sh->act_h, 0, sizeof(uint16_t) * kMaxTokens * sh->Kp_H));
+  CUDA_TRY(cudaMemset(sh->act_attn, 0, sizeof(uint16_t) * kMaxTokens * sh->Kp_dq));
+  CUDA_TRY(cudaMemset(sh->act_f, 0, sizeof(uint16_t) * kMaxTokens * sh->Kp_F));
+  CUDA_TRY(cudaMalloc(&sh->q, sizeof(float) * kMaxTokens * sh->dq));
+  for (int nt = 1; nt <= 2; ++nt) sh->grid[nt] = gemv_grid(nt, sh->num_sms);
+  CUDA_TRY(cudaMalloc(&sh->partials, sizeof(float) * gemv_partials_floats(std::max(sh->grid[1], sh->grid[2]))));
+  CUDA_TRY(cudaMalloc(&sh->counters, sizeof(int) * sh->max_rb));
+  CUDA_TRY(cudaMemset(sh->counters, 0, sizeof(int) * sh->max_rb));
+  CUDA_TRY(cudaMalloc(&sh->status, sizeof(int)));
+  CUDA_TRY(cudaMemset(sh->status, 0, sizeof(int)));
+  CUDA_TRY(cudaHostAlloc(&sh->status_host, sizeof(int), cudaHostAllocDefault));
+  *sh->status_host = 0;
+  CUDA_TRY(cudaMalloc(&sh->sp, sizeof(StepParams)));
+  CUDA_TRY(cudaMemset(sh->sp, 0, sizeof(StepParams)));
+  CUDA_TRY(cudaStreamCreateWithFlags(&sh->capture_stream, cudaStreamNonBlocking));
+  CUDA_TRY(cudaDeviceSynchronize());
+  *out = sh.release();
+  return SHARD_OK;
+}
+
+int shard_destroy(shard_t sh) {
+  if (!sh) return fail(SHARD_EINVAL, "shard_destroy: null shard");
+  cudaSetDevice(sh->device);
+  cudaDeviceSynchronize();
+  for (auto* st : sh->states) free_state(st);
+  cudaFree(sh->weight_pool);
+  cudaFree(sh->norms);
+  cudaFree(sh->embedding);
+  cudaFree(sh->rope);
+  cudaFree(sh->x);
+  cudaFree(sh->act_h);
+  cudaFree(sh->act_attn);
+  cudaFree(sh->act_f);
+  cudaFree(sh->q);
+  cudaFree(sh->partials);
+  cudaFree(sh->counters);
+  cudaFree(sh->status);
+  cudaFree(sh->sp);
+  cudaFree(sh->dstage);
+  if (sh->pin) cudaFreeHost(sh->pin);
+  if (sh->status_host) cudaFreeHost(sh->status_host);
+  if (sh->capture_stream) cudaStreamDestroy(sh->capture_stream);
+  for (auto e : sh->ev_pool) cudaEventDestroy(e);
+  for (auto& u : sh->ev_used) {
+    cudaEventDestroy(u.second.first);
+    cudaEventDestroy(u.second.second);
+  }
+  delete sh;
+  return SHARD_OK;
+}
+
+int shard_set_option(shard_t sh, int option, int value) {
+  if (!sh) return fail(SHARD_EINVAL, "null shard");
+  if (option == SHARD_OPT_GRAPH) {
+    sh->use_graph = value != 0;
+  } else if (option == SHARD_OPT_PDL) {
+    sh->use_pdl = value != 0;
+    for (auto* st : sh->states) {
+      for (auto& kv : st->graphs) {
+        cudaGraphExecDestroy(kv.second.exec);
+        cudaGraphDestroy(kv.second.graph);
+      }
+      st->graphs.clear();
+    }
+  } else {
+    return fail(SHARD_EINVAL, "unknown option %d", option);
+  }
+  return SHARD_OK;
+}
+
+int kv_state_alloc(shard_t sh, int n_rows, int capacity, kvstate_t* out) {
+  if (!sh || !out) return fail(SHARD_EINVAL, "kv_state_alloc: null argument");
+  if (n_rows < 1 || n_rows > SHARD_MAX_REQUESTS) return fail(SHARD_EINVAL, "n_rows must be in [1, %d]", SHARD_MAX_REQUESTS);
+  if (capacity < 1 || (long long)n_rows * capacity >= (1LL << 31)) return fail(SHARD_EINVAL, "invalid capacity");
+  CUDA_TRY(cudaSetDevice(sh->device));
+  auto st = new kvstate_s();
+  st->sh = sh;
+  st->n_rows = n_rows;
+  st->cap = capacity;
+  st->layer_stride = (size_t)n_rows * sh->Hkv * capacity * sh->d;
+  const size_t pool = st->layer_stride * sh->L;
+  st->cursor.assign(n_rows, 0);
+  st->len_host.assign(n_rows, 0);
+  st->chunk = 64;
+  st->n_chunks = (capacity + st->chunk - 1) / st->chunk;
+  int rc = SHARD_OK;
+  auto chk = [&](cudaError_t e) {
+    if (e != cudaSuccess && rc == SHARD_OK)
+      rc = fail(e == cudaErrorMemoryAllocation ? SHARD_ENOMEM : SHARD_ECUDA, "kv_state_alloc: %s", cudaGetErrorString(e));
+  };
+  chk(cudaMalloc(&st->k, sizeof(uint16_t) * pool));
+  chk(cudaMalloc(&st->v, sizeof(uint16_t) * pool));
+  chk(cudaMalloc(&st->bt[0], sizeof(int) * (size_t)n_rows * capacity));
+  chk(cudaMalloc(&st->bt[1], sizeof(int) * (size_t)n_rows * capacity));
+  chk(cudaMalloc(&st->lens, sizeof(int) * n_rows));
+  const int G = sh->Hq / sh->Hkv;
+  chk(cudaMalloc(&st->attn_part, sizeof(float) * attention_part_floats(n_rows, sh->Hkv, st->n_chunks, G, sh->d)));
+  chk(cudaMalloc(&st->attn_counters, sizeof(int) * n_rows * sh->Hkv));
+  if (rc == SHARD_OK) {
+    chk(cudaMemset(st->lens, 0, sizeof(int) * n_rows));
+    chk(cudaMemset(st->attn_counters, 0, sizeof(int) * n_rows * sh->Hkv));
+    chk(cudaMemset(st->k, 0, sizeof(uint16_t) * pool));
+    chk(cudaMemset(st->v, 0, sizeof(uint16_t) * pool));
+    chk(launch_fill_identity(st->bt[0], n_rows, capacity, -1, nullptr));
+    chk(launch_fill_identity(st->bt[1], n_rows, capacity, -1, nullptr));
+    chk(cudaDeviceSynchronize());
+  }
+  if (rc != SHARD_OK) {
+    free_state(st);
+    return rc;
+  }
+  sh->states.push_back(st);
+  *out = st;
+  return SHARD_OK;
+}
+
+int kv_state_free(kvstate_t st) {
+  if (!st) return fail(SHARD_EINVAL, "null state");
+  shard_s* sh = st->sh;
+  cudaSetDevice(sh->device);
+  cudaDeviceSynchronize();
+  for (size_t i = 0; i < sh->states.size(); ++i)
+    if (sh->states[i] == st) {
+      sh->states.erase(sh->states.begin() + i);
+      break;
+    }
+  free_state(st);
+  return SHARD_OK;
+}
+
+int kv_state_reset(kvstate_t st, int row) {
+  if (!st) return fail(SHARD_EINVAL, "null state");
+  if (row < -1 || row >= st->n_rows) return fail(SHARD_EINVAL, "row %d out of range", row);
+  CUDA_TRY(cudaSetDevice(st->sh->device));
+  CUDA_TRY(cudaDeviceSynchronize());
+  if (row == -1) {
+    CUDA_TRY(cudaMemset(st->lens, 0, sizeof(int) * st->n_rows));
+    CUDA_TRY(launch_fill_identity(st->bt[0], st->n_rows, st->cap, -1, nullptr));
+    CUDA_TRY(launch_fill_identity(st->bt[1], st->n_rows, st->cap, -1, nullptr));
+    st->cursor.assign(st->n_rows, 0);
+    st->len_host.assign(st->n_rows, 0);
+    st->bt_cur = 0;
+    st->shared = false;
+    st->poisoned = false;
+  } else {
+    if (st->shared) return fail(SHARD_EUNSUPPORTED, "rows share entries after a beam gather; reset all rows (-1)");
+    CUDA_TRY(cudaMemset(st->lens + row, 0, sizeof(int)));
+    CUDA_TRY(launch_fill_identity(st->bt[st->bt_cur], st->n_rows, st->cap, row, nullptr));
+    st->cursor[row] = 0;
+    st->len_host[row] = 0;
+  }
+  CUDA_TRY(cudaDeviceSynchronize());
+  return SHARD_OK;
+}
+
+int kv_state_load(kvstate_t st, int row, int layer, const uint16_t* k, const uint16_t* v, int len) {
+  if (!st || !k || !v) return fail(SHARD_EINVAL, "kv_state_load: null argument");
+  shard_s* sh = st->sh;
+  if (row < 0 || row >= st->n_rows || layer < 0 || layer >= sh->L || len < 0)
+    return fail(SHARD_EINVAL, "kv_state_load: row/layer/len out of range");
+  if (len > st->cap) return fail(SHARD_ECAPACITY, "kv_state_load: len %d > capacity %d", len, st->cap);
+  if (st->shared) return fail(SHARD_EUNSUPPORTED, "rows share entries after a beam gather; reset all rows (-1) first");
+  CUDA_TRY(cudaSetDevice(sh->device));
+  CUDA_TRY(cudaDeviceSynchronize());
+  const size_t d2 = sizeof(uint16_t) * sh->d;
+  for (int h = 0; h < sh->Hkv; ++h) {
+    const size_t off = (size_t)layer * st->layer_stride + (((size_t)row * sh->Hkv + h) * st->cap) * sh->d;
+    if (len > 0) {
+      CUDA_TRY(cudaMemcpy2D(st->k + off, d2, k + (size_t)h * sh->d, d2 * sh->Hkv, d2, len, cudaMemcpyHostToDevice));
+      CUDA_TRY(cudaMemcpy2D(st->v + off, d2, v + (size_t)h * sh->d, d2 * sh->Hkv, d2, len, cudaMemcpyHostToDevice));
+    }
+  }
+  CUDA_TRY(launch_fill_identity(st->bt[st->bt_cur], st->n_rows, st->cap, row, nullptr));
+  CUDA_TRY(cudaMemcpy(st->lens + row, &len, sizeof(int), cudaMemcpyHostToDevice));
+  st->cursor[row] = len;
+  st->len_host[row] = len;
+  CUDA_TRY(cudaDeviceSynchronize());
+  return SHARD_OK;
+}
+
+int kv_state_length(kvstate_t st, int row, int* len) {
+  if (!st || !len || row < 0 || row >= st->n_rows) return fail(SHARD_EINVAL, "kv_state_length: bad argument");
+  CUDA_TRY(cudaSetDevice(st->sh->device));
+  CUDA_TRY(cudaDeviceSynchronize());
+  CUDA_TRY(cudaMemcpy(len, st->lens + row, sizeof(int), cudaMemcpyDeviceToHost));
+  return SHARD_OK;
+}
+
+int kv_state_read(kvstate_t st, int row, int layer, int start, int len, uint16_t* k, uint16_t* v) {
+  if (!st || !k || !v) return fail(SHARD_EINVAL, "kv_state_read: null argument");
+  shard_s* sh = st->sh;
+  if (row < 0 || row >= st->n_rows || layer < 0 || layer >= sh->L || start < 0 || len < 0)
+    return fail(SHARD_EINVAL, "kv_state_read: row/layer/start/len out of range");
+  int cur = 0;
+  int rc = kv_state_length(st, row, &cur);
+  if (rc) return rc;
+  if (start + len > cur) return fail(SHARD_EINVAL, "kv_state_read: [%d, %d) beyond row length %d", start, start + len, cur);
+  if (len == 0) return SHARD_OK;
+  DevBuf<uint16_t> tmp;
+  CUDA_TRY(tmp.alloc((size_t)len * sh->Hkv * sh->d));
+  const int* slots = st->bt[st->bt_cur] + (size_t)row * st->cap + start;
+  for (int which = 0; which < 2; ++which) {
+    const uint16_t* pool = (which == 0 ? st->k : st->v) + (size_t)layer * st->layer_stride;
+    CUDA_TRY(launch_kv_gather(pool, 1, st->layer_stride, sh->Hkv, st->cap, sh->d, slots, len, tmp.p, nullptr));
+    CUDA_TRY(cudaMemcpy(which == 0 ? k : v, tmp.p, sizeof(uint16_t) * tmp.n, cudaMemcpyDeviceToHost));
+  }
+  return SHARD_OK;
+}
+
+int kv_trim(kvstate_t st, int row, const uint8_t* keep, int len) {
+  if (!st || !keep) return fail(SHARD_EINVAL, "kv_trim: null argument");
+  shard_s* sh = st->sh;
+  if (row < 0 || row >= st->n_rows) return fail(SHARD_EINVAL, "kv_trim: row out of range");
+  if (st->shared) return fail(SHARD_EUNSUPPORTED, "kv_trim: rows share entries after a beam gather");
+  int cur = 0;
+  int rc = kv_state_length(st, row, &cur);
+  if (rc) return rc;
+  if (len != cur) return fail(SHARD_EINVAL, "kv_trim: len %d != row length %d", len, cur);
+  std::vector<int> slots;
+  for (int j = 0; j < len; ++j)
+    if (keep[j]) slots.push_back(row * st->cap + j);  // unshared rows map entry j to slot (row, j)
+  const int n = static_cast<int>(slots.size());
+  if (n > 0) {
+    DevBuf<int> dslots;
+    DevBuf<uint16_t> tmp;
+    CUDA_TRY(dslots.alloc(n));
+    CUDA_TRY(cudaMemcpy(dslots.p, slots.data(), sizeof(int) * n, cudaMemcpyHostToDevice));
+    CUDA_TRY(tmp.alloc((size_t)sh->L * n * sh->Hkv * sh->d));
+    for (int which = 0; which < 2; ++which) {
+      uint16_t* pool = which == 0 ? st->k : st->v;
+      CUDA_TRY(launch_kv_gather(pool, sh->L, st->layer_stride, sh->Hkv, st->cap, sh->d, dslots.p, n, tmp.p, nullptr));
+      CUDA_TRY(launch_kv_scatter(pool, sh->L, st->layer_stride, sh->Hkv, st->cap, sh->d, row, tmp.p, n, nullptr));
+    }
+    CUDA_TRY(cudaDeviceSynchronize());
+  }
+  CUDA_TRY(launch_fill_identity(st->bt[st->bt_cur], st->n_rows, st->cap, row, nullptr));
+  CUDA_TRY(cudaMemcpy(st->lens + row, &n, sizeof(int), cudaMemcpyHostToDevice));
+  st->cursor[row] = n;
+  st->len_host[row] = n;
+  CUDA_TRY(cudaDeviceSynchronize());
+  return SHARD_OK;
+}
+
+int shard_step(shard_t sh, kvstate_t st, const uint16_t* hidden_in, const int32_t* token_ids, const int32_t* n_new,
+               int B, const int32_t* position_ids, const uint8_t* attention_mask, int mask_stride,
+               const int32_t* beam_idx, uint16_t* hidden_out, void* cuda_stream) {
+  if (!sh || !st || st->sh != sh) return fail(SHARD_EINVAL, "shard_step: shard/state mismatch");
+  if (!n_new || !position_ids || !attention_mask || !hidden_out) return fail(SHARD_EINVAL, "shard_step: null argument");
+  if ((hidden_in == nullptr) == (token_ids == nullptr))
+    return fail(SHARD_EINVAL, "shard_step: pass exactly one of hidden_in and token_ids");
+  if (token_ids && sh->cfg.vocab <= 0) return fail(SHARD_EUNSUPPORTED, "shard_step: this shard has no embedding");
+  if (B != st->n_rows) return fail(SHARD_EINVAL, "shard_step: B (%d) must equal the state's n_rows (%d)", B, st->n_rows);
+  if (mask_stride < 1) return fail(SHARD_EINVAL, "shard_step: mask_stride must be >= 1");
+  int M = 0, maxn = 0;
+  for (int b = 0; b < B; ++b) {
+    if (n_new[b] < 1) return fail(SHARD_EINVAL, "shard_step: n_new[%d] = %d < 1", b, n_new[b]);
+    M += n_new[b];
+    maxn = std::max(maxn, n_new[b]);
+  }
+  if (M > SHARD_MAX_TOKENS) return fail(SHARD_EINVAL, "shard_step: %d new tokens > %d", M, SHARD_MAX_TOKENS);
+  if (st->poisoned) return fail(SHARD_EINVAL, "shard_step: the KV state was left inconsistent by a rejected step; reset it");
+  int rc = check_pending_status(sh);
+  if (rc) return rc;
+  for (int b = 0; b < B; ++b) {
+    if (st->cursor[b] + n_new[b] > st->cap)
+      return fail(SHARD_ECAPACITY, "shard_step: row %d would hold %d entries > capacity %d", b, st->cursor[b] + n_new[b],
+                  st->cap);
+    if (!st->shared && !beam_idx) {
+      if (st->len_host[b] + n_new[b] > mask_stride)
+        return fail(SHARD_EINVAL, "shard_step: mask_stride %d < row %d length after the step %d", mask_stride, b,
+                    st->len_host[b] + n_new[b]);
+    }
+  }
+  CUDA_TRY(cudaSetDevice(sh->device));
+  cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+
+  PrologueArgs pa{};
+  pa.B = B;
+  pa.M = M;
+  for (int b = 0; b < B; ++b) {
+    pa.n_new[b] = n_new[b];
+    pa.cursor[b] = st->cursor[b];
+  }
+  pa.beam_idx = beam_idx;
+  pa.hidden_in = hidden_in;
+  pa.token_ids = token_ids;
+  pa.position_ids = position_ids;
+  pa.mask = attention_mask;
+  pa.mask_stride = mask_stride;
+  pa.hidden_out = hidden_out;
+  pa.bt_src = st->bt[st->bt_cur];
+  pa.bt_dst = st->bt[beam_idx ? st->bt_cur ^ 1 : st->bt_cur];
+  pa.lens = st->lens;
+  pa.cap = st->cap;
+  pa.max_position = sh->cfg.max_position;
+  pa.vocab = sh->cfg.vocab;
+  pa.H = sh->H;
+  pa.embedding = sh->embedding;
+  pa.x = sh->x;
+  pa.status = sh->status;
+  pa.sp = sh->sp;
+  const int nt = nt_for(M);
+
+  if (sh->use_graph && sh->profile_mask == 0) {
+    GraphEntry* ge = nullptr;
+    rc = get_graph(sh, st, nt, pa, &ge);
+    if (rc) return rc;
+    cudaKernelNodeParams kp = ge->prologue_params;
+    void* args[1] = {&pa};
+    kp.kernelParams = args;
+    kp.extra = nullptr;
+    CUDA_TRY(cudaGraphExecKernelNodeSetParams(ge->exec, ge->prologue, &kp));
+    CUDA_TRY(cudaGraphLaunch(ge->exec, s));
+  } else {
+    {
+      ProfScope ps(sh, PK_PROLOGUE, s);
+      CUDA_TRY(launch_prologue(pa, s, false));
+    }
+    rc = enqueue_layers(sh, st, nt, s, sh->use_pdl);
+    if (rc) return rc;
+  }
+  CUDA_TRY(cudaMemcpyAsync(sh->status_host, sh->status, sizeof(int), cudaMemcpyDeviceToHost, s));
+
+  for (int b = 0; b < B; ++b) st->cursor[b] += n_new[b];
+  if (beam_idx) {
+    st->bt_cur ^= 1;
+    st->shared = true;
+    int mx = 0;
+    for (int b = 0; b < B; ++b) mx = std::max(mx, st->len_host[b]);
+    for (int b = 0; b < B; ++b) st->len_host[b] = mx + n_new[b];  // upper bound
+  } else {
+    for (int b = 0; b < B; ++b) st->len_host[b] += n_new[b];
+  }
+  return SHARD_OK;
+}
+
+int shard_step_host(shard_t sh, kvstate_t st, const uint16_t* hidden_in, const int32_t* token_ids,
+                    const int32_t* n_new, int B, const int32_t* position_ids, const uint8_t* attention_mask,
+                    int mask_stride, const int32_t* beam_idx, uint16_t* hidden_out, void* cuda_stream) {
+  if (!sh || !st || !n_new || !position_ids || !attention_mask || !hidden_out)
+    return fail(SHARD_EINVAL, "shard_step_host: null argument");
+  if (B < 1 || B > SHARD_MAX_REQUESTS || mask_stride < 1) return fail(SHARD_EINVAL, "shard_step_host: bad B or mask_stride");
+  int M = 0;
+  for (int b = 0; b < B; ++b) M += n_new[b] > 0 ? n_new[b] : 0;
+  if (M < 1 || M > SHARD_MAX_TOKENS) return fail(SHARD_EINVAL, "shard_step_host: bad token count");
+  CUDA_TRY(cudaSetDevice(sh->device));
+  const size_t b_hid = hidden_in ? sizeof(uint16_t) * M * sh->H : 0;
+  const size_t b_tok = token_ids ? sizeof(int32_t) * M : 0;
+  const size_t b_pos = sizeof(int32_t) * M;
+  const size_t b_mask = (size_t)B * mask_stride;
+  const size_t b_beam = beam_idx ? sizeof(int32_t) * B : 0;
+  const size_t b_out = sizeof(uint16_t) * M * sh->H;
+  auto al = [](size_t v) { return (v + 255) / 256 * 256; };
+  const size_t in_bytes = al(b_hid) + al(b_tok) + al(b_pos) + al(b_mask) + al(b_beam);
+  const size_t need = in_bytes + al(b_out);
+  if (sh->pin_bytes < need) {
+    if (sh->pin) cudaFreeHost(sh->pin);
+    sh->pin = nullptr;
+    CUDA_TRY(cudaHostAlloc(&sh->pin, need, cudaHostAllocDefault));
+    sh->pin_bytes = need;
+  }
+  if (sh->dstage_bytes < need) {
+    cudaFree(sh->dstage);
+    sh->dstage = nullptr;
+    CUDA_TRY(cudaMalloc(&sh->dstage, need));
+    sh->dstage_bytes = need;
+  }
+  uint8_t* hp = static_cast<uint8_t*>(sh->pin);
+  uint8_t* dp = static_cast<uint8_t*>(sh->dstage);
+  size_t off = 0;
+  auto stage = [&](const void* src, size_t bytes) -> uint8_t* {
+    if (!src || !bytes) return nullptr;
+    memcpy(hp + off, src, bytes);
+    uint8_t* d = dp + off;
+    off += al(bytes);
+    return d;
+  };
+  const uint16_t* d_hid = reinterpret_cast<const uint16_t*>(stage(hidden_in, b_hid));
+  const int32_t* d_tok = reinterpret_cast<const int32_t*>(stage(token_ids, b_tok));
+  const int32_t* d_pos = reinterpret_cast<const int32_t*>(stage(position_ids, b_pos));
+  const uint8_t* d_mask = stage(attention_mask, b_mask);
+  const int32_t* d_beam = reinterpret_cast<const int32_t*>(stage(beam_idx, b_beam));
+  uint16_t* d_out = reinterpret_cast<uint16_t*>(dp + in_bytes);
+  cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+  CUDA_TRY(cudaMemcpyAsync(dp, hp, off, cudaMemcpyHostToDevice, s));
+  int rc = shard_step(sh, st, d_hid, d_tok, n_new, B, d_pos, d_mask, mask_stride, d_beam, d_out, cuda_stream);
+  if (rc) {
+    cudaStreamSynchronize(s);
+    return rc;
+  }
+  CUDA_TRY(cudaMemcpyAsync(hp + in_bytes, d_out, b_out, cudaMemcpyDeviceToHost, s));
+  CUDA_TRY(cudaStreamSynchronize(s));
+  memcpy(hidden_out, hp + in_bytes, b_out);
+  return SHARD_OK;
+}
+
+int shard_sync_status(shard_t sh, void* cuda_stream) {
+  if (!sh) return fail(SHARD_EINVAL, "null shard");
+  CUDA_TRY(cudaSetDevice(sh->device));
+  CUDA_TRY(cudaStreamSynchronize(static_cast<cudaStream_t>(cuda_stream)));
+  int bits = 0;
+  CUDA_TRY(cudaMemcpy(&bits, sh->status, sizeof(int), cudaMemcpyDeviceToHost));
+  CUDA_TRY(cudaMemset(sh->status, 0, sizeof(int)));
+  *reinterpret_cast<volatile int*>(sh->status_host) = 0;
+  if (bits) {
+    for (auto* st : sh->states) st->poisoned = true;
+    return fail(SHARD_EINVAL, "device guard: %s", status_message(bits).c_str());
+  }
+  return SHARD_OK;
+}
+
+// ---------------------------------------------------------------------------
+// Debug / test entry points (include/shard_debug.h)
+// ---------------------------------------------------------------------------
+
+int shard_debug_op_info(shard_t sh, int layer, int op, int* rows, int* K, long long* bytes) {
+  if (!sh || layer < 0 || layer >= sh->L || op < 0 || op >= N_OPS) return fail(SHARD_EINVAL, "bad op");
+  const PackedOp& p = sh->ops[(size_t)layer * N_OPS + op];
+  const int nat[N_OPS] = {sh->dq + 2 * sh->dkv, sh->H, 2 * sh->F, sh->H};
+  if (rows) *rows = nat[op];
+  if (K) *K = p.K;
+  if (bytes) *bytes = (long long)p.bytes;
+  return SHARD_OK;
+}
+
+int shard_debug_unpack(shard_t sh, int layer, int op, float* out, int ld) {
+  if (!sh || !out || layer < 0 || layer >= sh->L || op < 0 || op >= N_OPS) return fail(SHARD_EINVAL, "bad argument");
+  const PackedOp& p = sh->ops[(size_t)layer * N_OPS + op];
+  if (ld < p.K) return fail(SHARD_EINVAL, "ld < K");
+  CUDA_TRY(cudaSetDevice(sh->device));
+  CUDA_TRY(launch_unpack(p, out, ld, nullptr));
+  CUDA_TRY(cudaDeviceSynchronize());
+  return SHARD_OK;
+}
+
+int shard_debug_gemv(shard_t sh, int layer, int op, const uint16_t* x, int M, float* y, int y_ld, void* cuda_stream) {
+  if (!sh || !x || !y || layer < 0 || layer >= sh->L || op < 0 || op >= N_OPS) return fail(SHARD_EINVAL, "bad argument");
+  if (M < 1 || M > SHARD_MAX_TOKENS) return fail(SHARD_EINVAL, "M out of range");
+  const PackedOp& p = sh->ops[(size_t)layer * N_OPS + op];
+  CUDA_TRY(cudaSetDevice(sh->device));
+  cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+  // x [M][K] -> zero-padded [M][Kp] in the shard's activation buffer
+  uint16_t* act = (op == OP_O) ? sh->act_attn : (op == OP_DOWN) ? sh->act_f : sh->act_h;
+  const int ld = (op == OP_O) ? sh->Kp_dq : (op == OP_DOWN) ? sh->Kp_F : sh->Kp_H;
+  CUDA_TRY(cudaMemsetAsync(act, 0, sizeof(uint16_t) * ld * M, s));
+  CUDA_TRY(cudaMemcpy2DAsync(act, sizeof(uint16_t) * ld, x, sizeof(uint16_t) * p.K, sizeof(uint16_t) * p.K, M,
+                             cudaMemcpyDeviceToDevice, s));
+  GemvArgs g{};
+  g.units = p.units;
+  g.n_rb = p.n_rb;
+  g.upr = p.upr;
+  g.act = act;
+  g.act_ld = ld;
+  g.M = M;
+  g.sp = nullptr;
+  g.partials = sh->partials;
+  g.counters = sh->counters;
+  g.status = sh->status;
+  g.ep.kind = EPI_STORE;
+  g.ep.dims = p.dims;
+  g.ep.y = y;
+  g.ep.y_ld = y_ld;
+  const int nt = nt_for(M);
+  CUDA_TRY(launch_gemv(g, nt, sh->cfg.group, std::min<long long>(sh->grid[nt], (long long)p.n_rb * p.upr), s, false));
+  return SHARD_OK;
+}
+
+int shard_debug_profile(shard_t sh, unsigned kinds) {
+  if (!sh) return fail(SHARD_EINVAL, "null shard");
+  if (kinds >> PK_N) return fail(SHARD_EINVAL, "unknown kind bits");
+  sh->profile_mask = kinds;
+  return SHARD_OK;
+}
+
+int shard_debug_profile_read(shard_t sh, int kind, double* total_ms, int* launches) {
+  if (!sh || !total_ms || !launches || kind < 0 || kind >= PK_N) return fail(SHARD_EINVAL, "bad argument");
+  CUDA_TRY(cudaSetDevice(sh->device));
+  double t = 0.0;
+  int n = 0;
+  std::vector<std::pair<int, std::pair<cudaEvent_t, cudaEvent_t>>> keep;
+  for (auto& u : sh->ev_used) {
+    if (u.first != kind) {
+      keep.push_back(u);
+      continue;
+    }
+    CUDA_TRY(cudaEventSynchronize(u.second.second));
+    float ms = 0.f;
+    CUDA_TRY(cudaEventElapsedTime(&ms, u.second.first, u.second.second));
+    t += ms;
+    ++n;
+    sh->ev_pool.push_back(u.second.first);
+    sh->ev_pool.push_back(u.second.second);
+  }
+  sh->ev_used.swap(keep);
+  *total_ms = t;
+  *launches = n;
+  return SHARD_OK;
+}
+
+}  // extern "C"
