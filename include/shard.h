@@ -184,6 +184,32 @@ int shard_step_host(shard_t shard, kvstate_t state, const uint16_t* hidden_in, c
  * violated condition).  Clears the status. */
 int shard_sync_status(shard_t shard, void* cuda_stream);
 
+/* One projection of the shard, y[m][r] = sum_k W[r][k] * x[m][k], without
+ * any device allocation: for callers that must not allocate device memory
+ * while they run (a runtime that has pre-reserved all of HBM in its own pool
+ * and forbids outside cudaMalloc, a thread that may not take the allocator's
+ * lock, or a loop where an allocation's implicit synchronisation is not
+ * allowed).  It runs the same kernel as the step's projections; the kernel's
+ * scratch (cross-CTA partial sums, arrival counters, a zero-padded copy of x)
+ * lives in one fixed 4 MiB device array inside the library, which every GPU
+ * that loads the library holds until the process exits.  The paper has no
+ * counterpart; this is a deployment convenience.
+ *   op      0 = q|k|v, 1 = o, 2 = gate|up, 3 = down (row order as in
+ *           shard_debug.h); layer in [0, n_layers)
+ *   x       dev fp16 [M][K], K the op's input width, 1 <= M <= 16
+ *   y       dev fp32 [M][y_ld], y_ld >= the op's natural row count
+ * Calls larger than the fixed array (scratch for M tokens of K inputs and
+ * the op's row-blocks) fail with ECAPACITY and a message giving the sizes.
+ * The first call on each device resolves the array's device address (with
+ * that device made current); make that first call before any stream capture.
+ * Every call on a device shares the one array and it keeps the last call's
+ * contents (the call zeroes what must start at zero): calls whose work
+ * overlaps on the GPU -- different streams, or different host threads --
+ * race and corrupt each other's results.  Asynchronous on cuda_stream; it
+ * does not synchronise. */
+int shard_gemv_noalloc(shard_t shard, int layer, int op, const uint16_t* x, int M, float* y, int y_ld,
+                       void* cuda_stream);
+
 /* Options.  SHARD_OPT_GRAPH: replay each step from a captured CUDA graph
  * (default 1).  SHARD_OPT_PDL: launch kernels with programmatic dependent
  * launch so each one's weight prefetch overlaps its predecessor (default 1). */

@@ -28,7 +28,7 @@ OP_QKV, OP_O, OP_GU, OP_DOWN = 0, 1, 2, 3
 EXPORTS = ("shard_create", "shard_destroy", "kv_state_alloc", "kv_state_free", "kv_state_reset", "kv_state_load",
            "kv_state_read", "kv_state_length", "kv_trim", "shard_step", "shard_step_host", "shard_sync_status",
            "shard_set_option", "shard_last_error", "shard_debug_op_info", "shard_debug_unpack", "shard_debug_gemv",
-           "shard_debug_profile", "shard_debug_profile_read")
+           "shard_debug_profile", "shard_debug_profile_read", "shard_gemv_noalloc")
 KIND_QKV, KIND_O, KIND_GU, KIND_DOWN, KIND_ATTENTION, KIND_NORM, KIND_PROLOGUE = range(7)
 
 
@@ -90,6 +90,7 @@ def load_library(path: str = LIB_PATH):
         "shard_debug_unpack": ([vp, ip, ip, vp, ip], ip),
         "shard_debug_gemv": ([vp, ip, ip, vp, ip, vp, ip, vp], ip),
         "shard_debug_profile": ([vp, ctypes.c_uint], ip),
+        "shard_gemv_noalloc": ([vp, ip, ip, vp, ip, vp, ip, vp], ip),
         "shard_debug_profile_read": ([vp, ip, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_int)], ip),
     }
     for name, (args, res) in sig.items():
@@ -240,3 +241,10 @@ def shard_debug_profile_read(shard: int, kind: int):
     t, n = ctypes.c_double(), ctypes.c_int()
     _check(load_library().shard_debug_profile_read(shard, kind, ctypes.byref(t), ctypes.byref(n)))
     return t.value, n.value
+
+
+def shard_gemv_noalloc(shard: int, layer: int, op: int, x: int, M: int, y: int, y_ld: int, stream: int = 0,
+                       check: bool = True) -> int:
+    """One projection with the library's fixed scratch array (no device allocation)."""
+    rc = load_library().shard_gemv_noalloc(shard, layer, op, x, M, y, y_ld, stream or None)
+    return _check(rc) if check else rc

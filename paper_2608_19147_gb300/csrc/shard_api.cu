@@ -1044,3 +1044,32 @@ int shard_debug_profile_read(shard_t sh, int kind, double* total_ms, int* launch
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Support for shard_gemv_noalloc (noalloc.cu)
+// ---------------------------------------------------------------------------
+namespace shard {
+
+struct NoAllocView {
+  const PackedOp* op;
+  int group, grid_nt1, grid_nt2, device, rows;
+};
+
+int shard_noalloc_fail(int code, const char* msg) { return fail(code, "%s", msg); }
+
+int shard_noalloc_view(shard_t sh, int layer, int op, NoAllocView* v) {
+  if (!sh || !v) return fail(SHARD_EINVAL, "shard_gemv_noalloc: null shard");
+  if (layer < 0 || layer >= sh->L || op < 0 || op >= N_OPS)
+    return fail(SHARD_EINVAL, "shard_gemv_noalloc: layer %d / op %d out of range", layer, op);
+  v->op = &sh->ops[(size_t)layer * N_OPS + op];
+  v->group = sh->cfg.group;
+  v->grid_nt1 = sh->grid[1];
+  v->grid_nt2 = sh->grid[2];
+  v->device = sh->device;
+  const int nat[N_OPS] = {sh->dq + 2 * sh->dkv, sh->H, 2 * sh->F, sh->H};
+  v->rows = nat[op];
+  return SHARD_OK;
+}
+
+}  // namespace shard
+
