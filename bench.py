@@ -2,7 +2,8 @@
 """Benchmark of the GB300 shard-decode path.
 
 Metric: INT4 shard decode tokens/s at 1 GB300, with the achieved HBM
-bandwidth of the dominant kernel against the measured peak.
+bandwidth of the step kernel (the whole decode step is one launch) against
+the measured peak.
 
 Default workload (the Llama-3.1-8B-shaped stage 1 of 2 decode): a 16-layer
 shard (hidden 4096, 32 q / 8 kv heads, head_dim 128, FFN 14336, uint4 group
@@ -62,7 +63,7 @@ CONFIGS = {
     "tiny": dict(shape=synth.TINY, prefill=72, steps_per_request=256, rows=1, n=1, tokens=True,
                  workload="tiny 2L h256 decode: 72-token prefill, 1 token/step"),
 }
-KINDS = ["qkv", "o", "gate_up", "down", "attention", "rmsnorm", "prologue"]
+PHASES = ["norm1", "qkv", "attention", "attention_merge", "o", "norm2", "gate_up", "down"]
 
 
 def log(*a):
@@ -228,7 +229,7 @@ def measured_peaks():
 
 def kernel_source_hash() -> str:
     h = hashlib.sha256()
-    for f in ("gemv.cu", "common.cuh", "kernels.h"):
+    for f in ("gemv_core.cuh", "step_kernel.cu", "common.cuh", "kernels.h"):
         h.update(open(os.path.join(ROOT, "paper_2608_19147_gb300", "csrc", f), "rb").read())
     return h.hexdigest()[:16]
 
@@ -311,6 +312,12 @@ def run_gpu(args, rank: int, world: int):
         for t in range(count):
             pkg.shard_step(sh, state_of[t], hid[t], tok[t], n_new, pos[t], mask[t], p.stride, beam[t], out, sptr)
 
+    def run_steps_one(p: Plan, sts, d, t):
+        r, _ = p.step_of[t]
+        g = lambda key: (d[key][t].data_ptr() if key in d else None)
+        pkg.shard_step(sh, sts[r], g("hid"), g("tok"), [p.n] * p.B, d["pos"][t].data_ptr(), d["mask"][t].data_ptr(),
+                       p.stride, g("beam"), d["out"].data_ptr(), sptr)
+
     # warm-up (own states, so the timed requests start from their prefills)
     wst, wd = load_states(warm), stage(warm)
     run_steps(warm, wst, wd, W)
@@ -351,28 +358,30 @@ def run_gpu(args, rank: int, world: int):
     for st in sts + wst:
         pkg.kv_state_free(st)
 
-    # ---- profiled pass: events around every launch of each kernel kind ----
-    prof_K = min(K, plan.spr)
+    # ---- per-phase times: the step kernel's barrier timestamps, averaged
+    # over a pass of the same workload (one step, then read, per step) ----
+    prof_K = min(K, 64)
     pplan = Plan(args.config, prof_K, SEED + 2)
     pst, pd = load_states(pplan), stage(pplan)
-    pkg.shard_debug_profile(sh, (1 << len(KINDS)) - 1)
-    torch.cuda.synchronize()
-    run_steps(pplan, pst, pd, prof_K)
-    torch.cuda.synchronize()
-    kernels = {}
-    for i, kname in enumerate(KINDS):
-        tot, n = pkg.shard_debug_profile_read(sh, i)
-        if n:
-            kernels[kname] = {"launches": n, "avg_us": 1000.0 * tot / n, "total_ms": tot}
-    pkg.shard_debug_profile(sh, 0)
+    n_ph = 8 * shape.n_layers
+    acc = np.zeros(n_ph)
+    for t in range(prof_K):
+        run_steps_one(pplan, pst, pd, t)
+        acc += np.array(pkg.shard_debug_phase_times(sh, shape.n_layers))
+    acc /= prof_K
+    # times[0] is the prologue, then the eight phases of every layer (the
+    # last layer's down phase ends with the kernel, not at a barrier)
+    phases = {"prologue": {"total_us_per_step": float(acc[0])}}
+    lay = acc[1:].tolist() + [0.0]
+    for i, name in enumerate(PHASES):
+        v = np.array(lay[i::8])
+        phases[name] = {"avg_us_per_layer": float(v.mean()), "total_us_per_step": float(v.sum())}
+    for name, kind in (("qkv", "qkv"), ("o", "o"), ("gate_up", "gate_up"), ("down", "down")):
+        t_us = phases[name]["avg_us_per_layer"]
+        if t_us > 0:
+            phases[name]["achieved_gbs"] = pplan.kind_bytes(kind) / (t_us * 1e3)
     for st in pst:
         pkg.kv_state_free(st)
-    tot_all = sum(v["total_ms"] for v in kernels.values())
-    for kname, v in kernels.items():
-        v["share"] = v["total_ms"] / tot_all if tot_all else None
-        if kname in ("qkv", "o", "gate_up", "down"):
-            v["alg_bytes_per_launch"] = pplan.kind_bytes(kname)
-            v["achieved_gbs"] = v["alg_bytes_per_launch"] / (v["avg_us"] * 1e3)
 
     # ---- end to end through the host-buffer entry point ----
     eplan = Plan(args.config, K, SEED + 3)
@@ -411,12 +420,10 @@ def run_gpu(args, rank: int, world: int):
     peak_note = "of measured" if peak else "of fallback"
     if not peak:
         peak = 6800.0
-    dominant = max((k for k in kernels if k in ("qkv", "o", "gate_up", "down")), key=lambda k: kernels[k]["total_ms"])
-    dk = kernels[dominant]
     rows_per_step = plan.M
     value = world * K * rows_per_step / (ms / 1e3)
     step_bytes = sum(plan.alg_bytes(t) for t in range(K)) / K
-    launches_per_step = 1 + 7 * shape.n_layers
+    launches_per_step = 1  # the whole step is one kernel
     result = {
         "metric": METRIC,
         "value": value,
@@ -443,19 +450,19 @@ def run_gpu(args, rank: int, world: int):
             "seed": SEED,
         },
         "step_alg_bytes": step_bytes,
-        "step_achieved_gbs": step_bytes / (ms / K * 1e6),
         "roofline": {
-            "kernel": "gemv_%s" % dominant,
+            "kernel": "step_kernel (the whole decode step: %d layers in one launch)" % shape.n_layers,
             "bound": "hbm",
-            "achieved": dk["achieved_gbs"],
+            "achieved": step_bytes / (ms / K * 1e6),
             "peak": peak,
             "unit": "GB/s",
-            "frac": dk["achieved_gbs"] / peak,
-            "peak_note": "%s (%s copy bandwidth); per-launch duration from CUDA events around each launch in a "
-                         "profiled pass of the same workload" % (peak_note, "MEASURED_PEAKS.json hbm_gbs"),
-            "traffic": profiled_traffic(dominant, args.config),
+            "frac": step_bytes / (ms / K * 1e6) / peak,
+            "peak_note": "%s: MEASURED_PEAKS.json hbm_gbs (a copy bandwidth); achieved = algorithmic bytes per "
+                         "launch / CUDA-event time of the timed launches" % peak_note,
+            "traffic": profiled_traffic("step", args.config),
+            "frac_of_8tbs_nominal": step_bytes / (ms / K * 1e6) / 8000.0,
         },
-        "kernels": kernels,
+        "phases": phases,
         "e2e": {"value": world * K * rows_per_step / e2e_s, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
         "gpu_launches": K * launches_per_step,

@@ -210,12 +210,6 @@ int shard_sync_status(shard_t shard, void* cuda_stream);
 int shard_gemv_noalloc(shard_t shard, int layer, int op, const uint16_t* x, int M, float* y, int y_ld,
                        void* cuda_stream);
 
-/* Options.  SHARD_OPT_GRAPH: replay each step from a captured CUDA graph
- * (default 1).  SHARD_OPT_PDL: launch kernels with programmatic dependent
- * launch so each one's weight prefetch overlaps its predecessor (default 1). */
-enum { SHARD_OPT_GRAPH = 1, SHARD_OPT_PDL = 2 };
-int shard_set_option(shard_t shard, int option, int value);
-
 /* Message of the calling thread's last failed call ("" if none). */
 const char* shard_last_error(void);
 

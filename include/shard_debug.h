@@ -38,17 +38,13 @@ int shard_debug_unpack(shard_t shard, int layer, int op, float* out, int ld);
 int shard_debug_gemv(shard_t shard, int layer, int op, const uint16_t* x, int M, float* y, int y_ld,
                      void* cuda_stream);
 
-/* Launch profiling.  `kinds` is a bit set over
- *   0 q|k|v projection, 1 o projection, 2 gate|up projection, 3 down
- *   projection, 4 attention, 5 RMSNorm, 6 step prologue;
- * while it is non-zero, shard_step launches kernels directly (no graph
- * replay) and brackets every launch of a selected kind with CUDA events on
- * the launching stream.  0 turns profiling off. */
-int shard_debug_profile(shard_t shard, unsigned kinds);
-
-/* Waits for the recorded launches of one kind, returns their summed duration
- * in milliseconds and their count, and forgets them. */
-int shard_debug_profile_read(shard_t shard, int kind, double* total_ms, int* launches);
+/* Phase durations of the last completed shard_step, from the GPU's global
+ * timer read by one thread at each grid barrier of the step kernel: us[i] is
+ * the time between barrier i and barrier i+1 (barrier 0 = kernel start;
+ * order: prologue, then per layer: RMSNorm, q|k|v, attention partials,
+ * attention merge, o, RMSNorm, gate|up, down).  Returns the number of values
+ * written (at most n), or a negative error.  Synchronises the device. */
+int shard_debug_phase_times(shard_t shard, double* us, int n);
 
 #ifdef __cplusplus
 }

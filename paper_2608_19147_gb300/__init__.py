@@ -21,15 +21,14 @@ LIB_PATH = os.path.join(_HERE, "libshard.so")
 SHARD_OK, SHARD_EINVAL, SHARD_ECAPACITY, SHARD_ENOMEM, SHARD_ECUDA, SHARD_EUNSUPPORTED = 0, -1, -2, -3, -4, -5
 SHARD_MAX_TOKENS = 16
 SHARD_MAX_REQUESTS = 16
-SHARD_OPT_GRAPH, SHARD_OPT_PDL = 1, 2
 OP_QKV, OP_O, OP_GU, OP_DOWN = 0, 1, 2, 3
 
 # Every symbol include/shard.h and include/shard_debug.h declare.
 EXPORTS = ("shard_create", "shard_destroy", "kv_state_alloc", "kv_state_free", "kv_state_reset", "kv_state_load",
            "kv_state_read", "kv_state_length", "kv_trim", "shard_step", "shard_step_host", "shard_sync_status",
-           "shard_set_option", "shard_last_error", "shard_debug_op_info", "shard_debug_unpack", "shard_debug_gemv",
-           "shard_debug_profile", "shard_debug_profile_read", "shard_gemv_noalloc")
-KIND_QKV, KIND_O, KIND_GU, KIND_DOWN, KIND_ATTENTION, KIND_NORM, KIND_PROLOGUE = range(7)
+           "shard_last_error", "shard_debug_op_info", "shard_debug_unpack", "shard_debug_gemv",
+           "shard_debug_phase_times", "shard_gemv_noalloc")
+PHASES = ("norm1", "qkv", "attention", "attention_merge", "o", "norm2", "gate_up", "down")
 
 
 class ShardError(RuntimeError):
@@ -83,15 +82,13 @@ def load_library(path: str = LIB_PATH):
         "shard_step": ([vp, vp, vp, vp, i32p, ip, vp, vp, ip, vp, vp, vp], ip),
         "shard_step_host": ([vp, vp, vp, vp, i32p, ip, vp, vp, ip, vp, vp, vp], ip),
         "shard_sync_status": ([vp, vp], ip),
-        "shard_set_option": ([vp, ip, ip], ip),
         "shard_last_error": ([], ctypes.c_char_p),
         "shard_debug_op_info": ([vp, ip, ip, ctypes.POINTER(ctypes.c_int), ctypes.POINTER(ctypes.c_int),
                                  ctypes.POINTER(ctypes.c_longlong)], ip),
         "shard_debug_unpack": ([vp, ip, ip, vp, ip], ip),
         "shard_debug_gemv": ([vp, ip, ip, vp, ip, vp, ip, vp], ip),
-        "shard_debug_profile": ([vp, ctypes.c_uint], ip),
         "shard_gemv_noalloc": ([vp, ip, ip, vp, ip, vp, ip, vp], ip),
-        "shard_debug_profile_read": ([vp, ip, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_int)], ip),
+        "shard_debug_phase_times": ([vp, ctypes.POINTER(ctypes.c_double), ip], ip),
     }
     for name, (args, res) in sig.items():
         f = getattr(lib, name)
@@ -144,10 +141,6 @@ def shard_create(cfg: shard_config, layers: Sequence, embedding: Optional[np.nda
 
 def shard_destroy(shard: int) -> None:
     _check(load_library().shard_destroy(shard))
-
-
-def shard_set_option(shard: int, option: int, value: int) -> None:
-    _check(load_library().shard_set_option(shard, option, value))
 
 
 def kv_state_alloc(shard: int, n_rows: int, capacity: int) -> int:
@@ -232,15 +225,15 @@ def shard_debug_gemv(shard: int, layer: int, op: int, x: int, M: int, y: int, y_
     _check(load_library().shard_debug_gemv(shard, layer, op, x, M, y, y_ld, stream or None))
 
 
-def shard_debug_profile(shard: int, kinds: int) -> None:
-    _check(load_library().shard_debug_profile(shard, kinds))
-
-
-def shard_debug_profile_read(shard: int, kind: int):
-    """(total milliseconds, launches) of the recorded launches of one kind."""
-    t, n = ctypes.c_double(), ctypes.c_int()
-    _check(load_library().shard_debug_profile_read(shard, kind, ctypes.byref(t), ctypes.byref(n)))
-    return t.value, n.value
+def shard_debug_phase_times(shard: int, n_layers: int):
+    """Durations (microseconds) of the last step's phases: the prologue, then
+    per layer the eight phases named in PHASES."""
+    n = 8 * n_layers
+    buf = (ctypes.c_double * n)()
+    k = load_library().shard_debug_phase_times(shard, buf, n)
+    if k < 0:
+        _check(k)
+    return list(buf)[:k]
 
 
 def shard_gemv_noalloc(shard: int, layer: int, op: int, x: int, M: int, y: int, y_ld: int, stream: int = 0,

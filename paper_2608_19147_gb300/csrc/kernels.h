@@ -147,32 +147,7 @@ size_t gemv_partials_floats(int grid);
 cudaError_t launch_gemv(const GemvArgs& a, int nt, int group, int grid, cudaStream_t s, bool pdl);
 // One-time per-device kernel attribute setup (dynamic shared memory limits).
 cudaError_t gemv_setup();
-
-struct NormArgs {
-  const float* x; int H;
-  const uint16_t* w;
-  float eps;
-  uint16_t* out; int out_ld;
-  int M;                 // when sp == nullptr
-  const StepParams* sp;
-};
-cudaError_t launch_rmsnorm(const NormArgs& a, cudaStream_t s, bool pdl);
-
-struct AttnArgs {
-  const float* q;        // [M][Hq*d]
-  const uint16_t* kpool; // layer's pools [n_rows][Hkv][cap][d]
-  const uint16_t* vpool;
-  int cap, Hq, Hkv, d, chunk, n_chunks;
-  float* part;           // scratch [B][Hkv][n_chunks][G*16][d+2]
-  int* counters;         // [B*Hkv]
-  uint16_t* out;         // fp16 [M][out_ld]
-  int out_ld;
-  const StepParams* sp;
-};
-cudaError_t launch_attention(const AttnArgs& a, int B, cudaStream_t s, bool pdl);
-size_t attention_part_floats(int B, int Hkv, int n_chunks, int G, int d);
-size_t attention_smem_bytes(int G, int chunk, int d);
-cudaError_t attention_setup(size_t max_smem);
+int gemv_warps_per_cta();
 
 struct PrologueArgs {
   int B, M;
@@ -194,7 +169,46 @@ struct PrologueArgs {
   int* status;
   StepParams* sp;
 };
-cudaError_t launch_prologue(const PrologueArgs& a, cudaStream_t s, bool pdl);
+
+// A projection's unit stream as the device code walks it.
+struct OpDesc {
+  const uint8_t* units;
+  int n_rb, upr;
+};
+
+// Arguments of the whole-step kernel (step_kernel.cu).
+struct StepKernelArgs {
+  PrologueArgs pro;          // per-step values
+  const OpDesc* ops;         // [4 * L]: q|k|v, o, gate|up, down of each layer
+  int L, H, Hq, Hkv, d, F, Kp_H, Kp_dq, Kp_F;
+  float eps;
+  const uint16_t* norms;     // [L][2][H]
+  const float2* rope;        // [max_position][d/2]
+  float* x;                  // residual [16][H]
+  uint16_t* act_h;           // [16][Kp_H]
+  uint16_t* act_attn;        // [16][Kp_dq]
+  uint16_t* act_f;           // [16][Kp_F]
+  float* q;                  // [16][Hq*d]
+  float* partials;           // projection pieces [grid][2][64][16]
+  int* counters;             // [max row-blocks]
+  uint16_t* kpool;           // [L][n_rows][Hkv][cap][d]
+  uint16_t* vpool;
+  size_t layer_stride;
+  int cap, n_chunks;         // attention items are 32 entries
+  float* attn_part;          // [B][Hkv][n_chunks][16*G][d+2]
+  int* status;
+  unsigned long long* barrier;         // grid-barrier counter (monotonic)
+  unsigned long long barrier_base;     // its value when this launch starts
+  unsigned long long* phase_clock;     // [8L + 1] globaltimer at each barrier
+};
+// One-time attribute setup of the step kernel variants for a group size and
+// head dim; number of grid barriers per step; launch (cooperative, one CTA
+// per SM).
+cudaError_t step_setup(int group, int head_dim);
+int step_barriers(int n_layers);
+cudaError_t launch_step(const StepKernelArgs& a, int nt, int group, int grid, cudaStream_t s);
+size_t step_attention_part_floats(int B, int Hkv, int n_chunks, int G, int d);
+constexpr int kAttnChunk = 32;
 
 // Weight repacking (one fused op; all source pointers device).
 // Source matrices of a fused op (q, k, v for OP_QKV; gate, up for OP_GU; one

@@ -1,158 +1,8 @@
-// Step prologue, RMSNorm, weight repacking and KV-pool utilities.
+// Weight repacking and KV-pool utilities.
 #include "common.cuh"
 
 namespace shard {
 namespace {
-
-// ---------------------------------------------------------------------------
-// Step prologue (one CTA).  Applies the beam_idx gather to the per-row entry
-// tables (Section 4: row b continues the entries of row beam_idx[b]; the K/V
-// data stay where they are), appends the new tokens' entries at their
-// physical slots, checks every device-resident input, loads the residual
-// stream from hidden_in or the embedding, and publishes the step parameters.
-// On any violation it sets status bits and marks the step aborted without
-// touching the state.
-// ---------------------------------------------------------------------------
-constexpr int kPrologueThreads = 1024;
-
-__global__ void __launch_bounds__(kPrologueThreads) prologue_kernel(const PrologueArgs a) {
-  __shared__ int s_src[kMaxRequests], s_P[kMaxRequests], s_len[kMaxRequests], s_tok0[kMaxRequests + 1];
-  __shared__ int s_req[kMaxTokens], s_idx[kMaxTokens];
-  __shared__ int s_err;
-  pdl_launch_dependents();
-  pdl_wait();
-  const int tid = threadIdx.x, nth = blockDim.x;
-  if (tid == 0) {
-    // A step rejected earlier freezes the state until the host resets it.
-    s_err = __ldcg(a.status) != 0 ? ST_STICKY : 0;
-    int t = 0;
-    for (int b = 0; b < a.B; ++b) {
-      s_tok0[b] = t;
-      for (int i = 0; i < a.n_new[b]; ++i, ++t) {
-        s_req[t] = b;
-        s_idx[t] = i;
-      }
-    }
-    s_tok0[a.B] = t;
-  }
-  if (tid < a.B) {
-    int src = a.beam_idx ? __ldcg(a.beam_idx + tid) : tid;
-    if (src < 0 || src >= a.B) {
-      atomicOr(&s_err, ST_BEAM_IDX);
-      src = tid;
-    }
-    s_src[tid] = src;
-    s_P[tid] = __ldcg(a.lens + src);
-  }
-  __syncthreads();
-  if (tid < a.B) {
-    const int L = s_P[tid] + a.n_new[tid];
-    if (L > a.cap || a.cursor[tid] + a.n_new[tid] > a.cap) atomicOr(&s_err, ST_CAPACITY);
-    if (L > a.mask_stride) atomicOr(&s_err, ST_MASK_STRIDE);
-    s_len[tid] = L;
-  }
-  __syncthreads();
-  for (int m = tid; m < a.M; m += nth) {
-    const int b = s_req[m], j = s_P[b] + s_idx[m];
-    if (j < a.mask_stride && __ldcg(a.mask + (size_t)b * a.mask_stride + j) == 0) atomicOr(&s_err, ST_MASK_NEW);
-    const int pos = __ldcg(a.position_ids + m);
-    if (pos < 0 || pos >= a.max_position) atomicOr(&s_err, ST_POSITION);
-    if (a.token_ids) {
-      const int tok = __ldcg(a.token_ids + m);
-      if (tok < 0 || tok >= a.vocab) atomicOr(&s_err, ST_TOKEN);
-    }
-  }
-  __syncthreads();
-  if (s_err) {
-    if (tid == 0) {
-      atomicOr(a.status, s_err & ~ST_STICKY);
-      a.sp->abort_step = 1;
-    }
-    return;
-  }
-  // Entry tables: gather (beam) then append.
-  if (a.beam_idx) {
-    for (int b = 0; b < a.B; ++b) {
-      const int* src = a.bt_src + (size_t)s_src[b] * a.cap;
-      int* dst = a.bt_dst + (size_t)b * a.cap;
-      for (int j = tid; j < s_P[b]; j += nth) dst[j] = __ldcg(src + j);
-    }
-  }
-  for (int m = tid; m < a.M; m += nth) {
-    const int b = s_req[m], i = s_idx[m];
-    a.bt_dst[(size_t)b * a.cap + s_P[b] + i] = b * a.cap + a.cursor[b] + i;
-  }
-  if (tid < a.B) a.lens[tid] = s_len[tid];
-  // Residual stream.
-  const size_t n = (size_t)a.M * a.H;
-  for (size_t e = tid; e < n; e += nth) {
-    const int m = static_cast<int>(e / a.H);
-    const size_t k = e % a.H;
-    uint16_t h;
-    if (a.hidden_in)
-      h = __ldcg(a.hidden_in + e);
-    else
-      h = a.embedding[(size_t)__ldcg(a.token_ids + m) * a.H + k];
-    a.x[e] = h2f(h);
-  }
-  if (tid == 0) {
-    StepParams* sp = a.sp;
-    sp->M = a.M;
-    sp->B = a.B;
-    sp->abort_step = 0;
-    for (int m = 0; m < a.M; ++m) {
-      const int b = s_req[m];
-      sp->tok_req[m] = b;
-      sp->tok_idx[m] = s_idx[m];
-      sp->tok_pos[m] = __ldcg(a.position_ids + m);
-      sp->tok_slot[m] = b * a.cap + a.cursor[b] + s_idx[m];
-    }
-    for (int b = 0; b <= a.B; ++b) sp->req_tok0[b] = s_tok0[b];
-    for (int b = 0; b < a.B; ++b) {
-      sp->req_P[b] = s_P[b];
-      sp->req_len[b] = s_len[b];
-    }
-    sp->mask = a.mask;
-    sp->mask_stride = a.mask_stride;
-    sp->hidden_out = a.hidden_out;
-    sp->bt = a.bt_dst;
-  }
-}
-
-// ---------------------------------------------------------------------------
-// RMSNorm: out[m][k] = fp16(x[m][k] / sqrt(mean_k x^2 + eps) * w[k]).  One CTA
-// per token; the sum of squares is reduced in a fixed order.
-// ---------------------------------------------------------------------------
-constexpr int kNormThreads = 256;
-
-__global__ void __launch_bounds__(kNormThreads) rmsnorm_kernel(const NormArgs a) {
-  __shared__ float s_part[kNormThreads / 32];
-  __shared__ float s_rstd;
-  pdl_launch_dependents();
-  pdl_wait();
-  const int M = a.sp ? a.sp->M : a.M;
-  if ((a.sp && a.sp->abort_step) || (int)blockIdx.x >= M) return;
-  const int m = blockIdx.x;
-  const float* x = a.x + (size_t)m * a.H;
-  float ss = 0.f;
-  for (int k = threadIdx.x; k < a.H; k += kNormThreads) {
-    const float v = __ldcg(x + k);
-    ss = fmaf(v, v, ss);
-  }
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
-  if ((threadIdx.x & 31) == 0) s_part[threadIdx.x >> 5] = ss;
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    float t = 0.f;
-    for (int w = 0; w < kNormThreads / 32; ++w) t += s_part[w];
-    s_rstd = rsqrtf(t / a.H + a.eps);
-  }
-  __syncthreads();
-  const float r = s_rstd;
-  uint16_t* out = a.out + (size_t)m * a.out_ld;
-  for (int k = threadIdx.x; k < a.H; k += kNormThreads) out[k] = f2h(__ldcg(x + k) * r * h2f(a.w[k]));
-}
 
 // ---------------------------------------------------------------------------
 // Repacking into the unit stream (see kernels.h for the layout).
@@ -289,32 +139,7 @@ int grid_for(size_t n, int threads) {
   return g < 1 ? 1 : static_cast<int>(g);
 }
 
-cudaLaunchConfig_t make_cfg(dim3 grid, dim3 block, size_t smem, cudaStream_t s, bool pdl, cudaLaunchAttribute* attr) {
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = grid;
-  cfg.blockDim = block;
-  cfg.dynamicSmemBytes = smem;
-  cfg.stream = s;
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = pdl ? 1 : 0;
-  return cfg;
-}
-
 }  // namespace
-
-cudaError_t launch_prologue(const PrologueArgs& a, cudaStream_t s, bool pdl) {
-  cudaLaunchAttribute attr[1];
-  cudaLaunchConfig_t cfg = make_cfg(dim3(1), dim3(kPrologueThreads), 0, s, pdl, attr);
-  return cudaLaunchKernelEx(&cfg, prologue_kernel, a);
-}
-
-cudaError_t launch_rmsnorm(const NormArgs& a, cudaStream_t s, bool pdl) {
-  cudaLaunchAttribute attr[1];
-  cudaLaunchConfig_t cfg = make_cfg(dim3(a.sp ? kMaxTokens : a.M), dim3(kNormThreads), 0, s, pdl, attr);
-  return cudaLaunchKernelEx(&cfg, rmsnorm_kernel, a);
-}
 
 cudaError_t launch_repack(const PackedOp& op, const int* rowmap, const RepackSrc& src, cudaStream_t s) {
   SrcView v{src, op.K, op.group, (op.K + op.group - 1) / op.group};

@@ -20,9 +20,9 @@
 namespace shard {
 namespace {
 
-// 4 MiB: partials for up to 2 CTAs per SM on 152 SMs (2.4 MiB), counters for
-// 1024 row-blocks (4 KiB), and 16 padded activation rows of up to 28672
-// inputs (896 KiB).
+// 4 MiB: the padded activations (16 rows of up to 28672 inputs: 896 KiB), the
+// row-block counters (4 KiB for 1024 row-blocks) and the cross-CTA partial
+// sums of as many CTAs as fit in the rest (8 KiB per CTA).
 constexpr size_t kNoAllocScratchBytes = 4u << 20;
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 
@@ -62,15 +62,21 @@ int shard_gemv_noalloc(shard_t sh, int layer, int op, const uint16_t* x, int M, 
   }
   const PackedOp& p = *v.op;
   const int nt = M <= 8 ? 1 : 2;
-  const int grid = static_cast<int>(std::min<long long>(nt == 1 ? v.grid_nt1 : v.grid_nt2, (long long)p.n_rb * p.upr));
-  // Scratch layout: [partials | counters | activations], 256-byte aligned parts.
-  const size_t part_bytes = (gemv_partials_floats(grid) * sizeof(float) + 255) / 256 * 256;
+  // Scratch layout: [partials | counters | activations], 256-byte aligned
+  // parts.  The grid shrinks until its partials fit next to the rest.
   const size_t cnt_bytes = ((size_t)(p.n_rb + 1) * sizeof(int) + 255) / 256 * 256;  // counters + status word
   const size_t act_bytes = (size_t)M * p.Kp * sizeof(uint16_t);
-  if (part_bytes + cnt_bytes + act_bytes > kNoAllocScratchBytes) {
+  const size_t per_cta = gemv_partials_floats(1) * sizeof(float);
+  long long fit = 0;
+  if (cnt_bytes + act_bytes < kNoAllocScratchBytes) fit = (long long)((kNoAllocScratchBytes - cnt_bytes - act_bytes) / per_cta);
+  const int grid = static_cast<int>(std::min<long long>(std::min<long long>(nt == 1 ? v.grid_nt1 : v.grid_nt2, fit),
+                                                        (long long)p.n_rb * p.upr));
+  const size_t part_bytes = (gemv_partials_floats(grid > 0 ? grid : 0) * sizeof(float) + 255) / 256 * 256;
+  if (grid < 1 || part_bytes + cnt_bytes + act_bytes > kNoAllocScratchBytes) {
     snprintf(g_msg, sizeof(g_msg),
-             "shard_gemv_noalloc: needs %zu bytes of scratch (M=%d, K=%d, %d row-blocks, grid %d) > the fixed %zu",
-             part_bytes + cnt_bytes + act_bytes, M, p.K, p.n_rb, grid, kNoAllocScratchBytes);
+             "shard_gemv_noalloc: needs %zu bytes of scratch for M=%d, K=%d and %d row-blocks plus %zu per CTA; "
+             "the fixed array has %zu",
+             cnt_bytes + act_bytes, M, p.K, p.n_rb, per_cta, kNoAllocScratchBytes);
     return shard_noalloc_fail(SHARD_ECAPACITY, g_msg);
   }
   if (y_ld < v.rows) {

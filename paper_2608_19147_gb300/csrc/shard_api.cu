@@ -64,13 +64,6 @@ std::string status_message(int bits) {
 
 }  // namespace
 
-struct GraphEntry {
-  cudaGraph_t graph = nullptr;      // kept alive: node handles refer to it
-  cudaGraphExec_t exec = nullptr;
-  cudaGraphNode_t prologue = nullptr;
-  cudaKernelNodeParams prologue_params{};  // as captured; kernelParams swapped per step
-};
-
 struct shard_s {
   int device = 0;
   shard_config cfg{};
@@ -95,19 +88,18 @@ struct shard_s {
   int* status = nullptr;           // device status word
   int* status_host = nullptr;      // pinned mirror (copied after each step)
   StepParams* sp = nullptr;
-  int grid[3] = {0, 0, 0};         // GEMV grid per token bucket
-  bool use_graph = true, use_pdl = true;
-  cudaStream_t capture_stream = nullptr;
+  int grid[3] = {0, 0, 0};         // standalone GEMV grid per token bucket
+  OpDesc* ops_dev = nullptr;       // [4L] op descriptors for the step kernel
+  unsigned long long* barrier = nullptr;  // grid-barrier counter
+  unsigned long long barrier_base = 0;    // its value at the next launch
+  unsigned long long* phase_clock = nullptr;  // [8L + 1]
+  int n_barriers = 0;
   // staging for shard_step_host
   void* pin = nullptr;
   size_t pin_bytes = 0;
   void* dstage = nullptr;
   size_t dstage_bytes = 0;
   std::vector<kvstate_s*> states;
-  // launch profiling (debug): CUDA events around launches of selected kinds
-  unsigned profile_mask = 0;
-  std::vector<cudaEvent_t> ev_pool;
-  std::vector<std::pair<int, std::pair<cudaEvent_t, cudaEvent_t>>> ev_used;
 };
 
 struct kvstate_s {
@@ -122,27 +114,20 @@ struct kvstate_s {
   std::vector<int> cursor, len_host;
   bool shared = false;    // rows may share entries (a beam gather ran)
   bool poisoned = false;  // a step aborted on the device
-  int chunk = 64, n_chunks = 0;
+  int n_chunks = 0;       // attention items per row (32 entries each)
   float* attn_part = nullptr;
-  int* attn_counters = nullptr;
-  std::map<int, GraphEntry> graphs;
 };
 
 namespace {
 
 void free_state(kvstate_s* st) {
   if (!st) return;
-  for (auto& kv : st->graphs) {
-    if (kv.second.exec) cudaGraphExecDestroy(kv.second.exec);
-    if (kv.second.graph) cudaGraphDestroy(kv.second.graph);
-  }
   cudaFree(st->k);
   cudaFree(st->v);
   cudaFree(st->bt[0]);
   cudaFree(st->bt[1]);
   cudaFree(st->lens);
   cudaFree(st->attn_part);
-  cudaFree(st->attn_counters);
   delete st;
 }
 
@@ -194,186 +179,6 @@ int op_K(int kind, const shard_s& s) {
 
 int nt_for(int M) { return M <= 8 ? 1 : 2; }
 
-// Profiled kinds: the four projections (OpKind), then these.
-enum { PK_ATTENTION = 4, PK_NORM = 5, PK_PROLOGUE = 6, PK_N = 7 };
-
-cudaEvent_t pool_event(shard_s* sh) {
-  if (sh->ev_pool.empty()) {
-    cudaEvent_t e = nullptr;
-    if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
-    return e;
-  }
-  cudaEvent_t e = sh->ev_pool.back();
-  sh->ev_pool.pop_back();
-  return e;
-}
-
-// Brackets one launch with events when its kind is being profiled.
-struct ProfScope {
-  shard_s* sh;
-  int kind;
-  cudaStream_t s;
-  cudaEvent_t a = nullptr;
-  ProfScope(shard_s* sh_, int kind_, cudaStream_t s_) : sh(sh_), kind(kind_), s(s_) {
-    if (sh->profile_mask & (1u << kind)) {
-      a = pool_event(sh);
-      if (a) cudaEventRecord(a, s);
-    }
-  }
-  ~ProfScope() {
-    if (!a) return;
-    cudaEvent_t b = pool_event(sh);
-    if (!b) return;
-    cudaEventRecord(b, s);
-    sh->ev_used.push_back({kind, {a, b}});
-  }
-};
-
-// Enqueues the whole step after the prologue.
-int enqueue_layers(shard_s* sh, kvstate_s* st, int nt, cudaStream_t s, bool pdl) {
-  const int B = st->n_rows;
-  for (int l = 0; l < sh->L; ++l) {
-    PackedOp* ops = &sh->ops[(size_t)l * N_OPS];
-    const uint16_t* nrm = sh->norms + (size_t)l * 2 * sh->H;
-    NormArgs na{sh->x, sh->H, nrm, static_cast<float>(sh->cfg.rms_eps), sh->act_h, sh->Kp_H, 0, sh->sp};
-    {
-      ProfScope ps(sh, PK_NORM, s);
-      CUDA_TRY(launch_rmsnorm(na, s, pdl));
-    }
-    GemvArgs g{};
-    g.sp = sh->sp;
-    g.partials = sh->partials;
-    g.counters = sh->counters;
-    g.status = sh->status;
-    // q, k, v with RoPE and K/V append
-    g.units = ops[OP_QKV].units;
-    g.n_rb = ops[OP_QKV].n_rb;
-    g.upr = ops[OP_QKV].upr;
-    g.act = sh->act_h;
-    g.act_ld = sh->Kp_H;
-    g.ep = EpiArgs{};
-    g.ep.kind = EPI_QKV;
-    g.ep.dims = ops[OP_QKV].dims;
-    g.ep.q = sh->q;
-    g.ep.kpool = st->k + (size_t)l * st->layer_stride;
-    g.ep.vpool = st->v + (size_t)l * st->layer_stride;
-    g.ep.cap = st->cap;
-    g.ep.rope = sh->rope;
-    {
-      ProfScope ps(sh, OP_QKV, s);
-      CUDA_TRY(launch_gemv(g, nt, sh->cfg.group, std::min<long long>(sh->grid[nt], (long long)g.n_rb * g.upr), s, pdl));
-    }
-    // attention
-    AttnArgs aa{};
-    aa.q = sh->q;
-    aa.kpool = g.ep.kpool;
-    aa.vpool = g.ep.vpool;
-    aa.cap = st->cap;
-    aa.Hq = sh->Hq;
-    aa.Hkv = sh->Hkv;
-    aa.d = sh->d;
-    aa.chunk = st->chunk;
-    aa.n_chunks = st->n_chunks;
-    aa.part = st->attn_part;
-    aa.counters = st->attn_counters;
-    aa.out = sh->act_attn;
-    aa.out_ld = sh->Kp_dq;
-    aa.sp = sh->sp;
-    {
-      ProfScope ps(sh, PK_ATTENTION, s);
-      CUDA_TRY(launch_attention(aa, B, s, pdl));
-    }
-    // o projection + residual
-    g.units = ops[OP_O].units;
-    g.n_rb = ops[OP_O].n_rb;
-    g.upr = ops[OP_O].upr;
-    g.act = sh->act_attn;
-    g.act_ld = sh->Kp_dq;
-    g.ep = EpiArgs{};
-    g.ep.kind = EPI_RESID;
-    g.ep.dims = ops[OP_O].dims;
-    g.ep.x = sh->x;
-    {
-      ProfScope ps(sh, OP_O, s);
-      CUDA_TRY(launch_gemv(g, nt, sh->cfg.group, std::min<long long>(sh->grid[nt], (long long)g.n_rb * g.upr), s, pdl));
-    }
-    // MLP
-    na.w = nrm + sh->H;
-    {
-      ProfScope ps(sh, PK_NORM, s);
-      CUDA_TRY(launch_rmsnorm(na, s, pdl));
-    }
-    g.units = ops[OP_GU].units;
-    g.n_rb = ops[OP_GU].n_rb;
-    g.upr = ops[OP_GU].upr;
-    g.act = sh->act_h;
-    g.act_ld = sh->Kp_H;
-    g.ep = EpiArgs{};
-    g.ep.kind = EPI_SWIGLU;
-    g.ep.dims = ops[OP_GU].dims;
-    g.ep.h = sh->act_f;
-    g.ep.h_ld = sh->Kp_F;
-    {
-      ProfScope ps(sh, OP_GU, s);
-      CUDA_TRY(launch_gemv(g, nt, sh->cfg.group, std::min<long long>(sh->grid[nt], (long long)g.n_rb * g.upr), s, pdl));
-    }
-    g.units = ops[OP_DOWN].units;
-    g.n_rb = ops[OP_DOWN].n_rb;
-    g.upr = ops[OP_DOWN].upr;
-    g.act = sh->act_f;
-    g.act_ld = sh->Kp_F;
-    g.ep = EpiArgs{};
-    g.ep.kind = EPI_RESID;
-    g.ep.dims = ops[OP_DOWN].dims;
-    g.ep.x = sh->x;
-    g.ep.write_out = (l == sh->L - 1) ? 1 : 0;
-    {
-      ProfScope ps(sh, OP_DOWN, s);
-      CUDA_TRY(launch_gemv(g, nt, sh->cfg.group, std::min<long long>(sh->grid[nt], (long long)g.n_rb * g.upr), s, pdl));
-    }
-  }
-  return SHARD_OK;
-}
-
-int get_graph(shard_s* sh, kvstate_s* st, int nt, const PrologueArgs& pa, GraphEntry** out) {
-  auto it = st->graphs.find(nt);
-  if (it != st->graphs.end()) {
-    *out = &it->second;
-    return SHARD_OK;
-  }
-  cudaStream_t cs = sh->capture_stream;
-  CUDA_TRY(cudaStreamBeginCapture(cs, cudaStreamCaptureModeThreadLocal));
-  int rc = SHARD_OK;
-  cudaError_t e = launch_prologue(pa, cs, false);
-  if (e != cudaSuccess) rc = fail(SHARD_ECUDA, "prologue launch during capture: %s", cudaGetErrorString(e));
-  if (rc == SHARD_OK) rc = enqueue_layers(sh, st, nt, cs, sh->use_pdl);
-  cudaGraph_t graph = nullptr;
-  cudaError_t e2 = cudaStreamEndCapture(cs, &graph);
-  if (rc != SHARD_OK) {
-    if (graph) cudaGraphDestroy(graph);
-    return rc;
-  }
-  if (e2 != cudaSuccess) return fail(SHARD_ECUDA, "graph capture: %s", cudaGetErrorString(e2));
-  size_t n_roots = 0;
-  CUDA_TRY(cudaGraphGetRootNodes(graph, nullptr, &n_roots));
-  if (n_roots != 1) {
-    cudaGraphDestroy(graph);
-    return fail(SHARD_ECUDA, "captured step graph has %zu root nodes (expected 1)", n_roots);
-  }
-  GraphEntry ge;
-  ge.graph = graph;
-  e = cudaGraphGetRootNodes(graph, &ge.prologue, &n_roots);
-  if (e == cudaSuccess) e = cudaGraphKernelNodeGetParams(ge.prologue, &ge.prologue_params);
-  if (e == cudaSuccess) e = cudaGraphInstantiate(&ge.exec, graph, 0);
-  if (e != cudaSuccess) {
-    cudaGraphDestroy(graph);
-    return fail(SHARD_ECUDA, "graph instantiate: %s", cudaGetErrorString(e));
-  }
-  auto res = st->graphs.emplace(nt, ge);
-  *out = &res.first->second;
-  return SHARD_OK;
-}
-
 int check_pending_status(shard_s* sh) {
   const int bits = *reinterpret_cast<volatile int*>(sh->status_host);
   if (bits) {
@@ -411,8 +216,9 @@ int shard_create(const shard_config* cfg, const shard_weights_host* w, shard_t* 
   auto sh = std::unique_ptr<shard_s>(new shard_s());
   CUDA_TRY(cudaGetDevice(&sh->device));
   CUDA_TRY(cudaDeviceGetAttribute(&sh->num_sms, cudaDevAttrMultiProcessorCount, sh->device));
+  if (c.head_dim != 64 && c.head_dim != 128) return fail(SHARD_EUNSUPPORTED, "head_dim must be 64 or 128");
   CUDA_TRY(gemv_setup());
-  CUDA_TRY(attention_setup(attention_smem_bytes(c.n_heads / c.n_kv_heads, 64, c.head_dim)));
+  CUDA_TRY(step_setup(c.group, c.head_dim));
   sh->cfg = c;
   sh->H = c.hidden;
   sh->Hq = c.n_heads;
@@ -549,7 +355,11 @@ int shard_create(const shard_config* cfg, const shard_weights_host* w, shard_t* 
   CUDA_TRY(cudaMemset(sh->act_f, 0, sizeof(uint16_t) * kMaxTokens * sh->Kp_F));
   CUDA_TRY(cudaMalloc(&sh->q, sizeof(float) * kMaxTokens * sh->dq));
   for (int nt = 1; nt <= 2; ++nt) sh->grid[nt] = gemv_grid(nt, sh->num_sms);
-  CUDA_TRY(cudaMalloc(&sh->partials, sizeof(float) * gemv_partials_floats(std::max(sh->grid[1], sh->grid[2]))));
+  {
+    const size_t step_pieces = (size_t)sh->num_sms * 2 * 1024;
+    const size_t n = std::max(gemv_partials_floats(std::max(sh->grid[1], sh->grid[2])), step_pieces);
+    CUDA_TRY(cudaMalloc(&sh->partials, sizeof(float) * n));
+  }
   CUDA_TRY(cudaMalloc(&sh->counters, sizeof(int) * sh->max_rb));
   CUDA_TRY(cudaMemset(sh->counters, 0, sizeof(int) * sh->max_rb));
   CUDA_TRY(cudaMalloc(&sh->status, sizeof(int)));
@@ -558,7 +368,17 @@ int shard_create(const shard_config* cfg, const shard_weights_host* w, shard_t* 
   *sh->status_host = 0;
   CUDA_TRY(cudaMalloc(&sh->sp, sizeof(StepParams)));
   CUDA_TRY(cudaMemset(sh->sp, 0, sizeof(StepParams)));
-  CUDA_TRY(cudaStreamCreateWithFlags(&sh->capture_stream, cudaStreamNonBlocking));
+  {
+    std::vector<OpDesc> od(sh->ops.size());
+    for (size_t i = 0; i < od.size(); ++i) od[i] = OpDesc{sh->ops[i].units, sh->ops[i].n_rb, sh->ops[i].upr};
+    CUDA_TRY(cudaMalloc(&sh->ops_dev, sizeof(OpDesc) * od.size()));
+    CUDA_TRY(cudaMemcpy(sh->ops_dev, od.data(), sizeof(OpDesc) * od.size(), cudaMemcpyHostToDevice));
+  }
+  sh->n_barriers = step_barriers(sh->L);
+  CUDA_TRY(cudaMalloc(&sh->barrier, sizeof(unsigned long long)));
+  CUDA_TRY(cudaMemset(sh->barrier, 0, sizeof(unsigned long long)));
+  CUDA_TRY(cudaMalloc(&sh->phase_clock, sizeof(unsigned long long) * (sh->n_barriers + 1)));
+  CUDA_TRY(cudaMemset(sh->phase_clock, 0, sizeof(unsigned long long) * (sh->n_barriers + 1)));
   CUDA_TRY(cudaDeviceSynchronize());
   *out = sh.release();
   return SHARD_OK;
@@ -585,32 +405,10 @@ int shard_destroy(shard_t sh) {
   cudaFree(sh->dstage);
   if (sh->pin) cudaFreeHost(sh->pin);
   if (sh->status_host) cudaFreeHost(sh->status_host);
-  if (sh->capture_stream) cudaStreamDestroy(sh->capture_stream);
-  for (auto e : sh->ev_pool) cudaEventDestroy(e);
-  for (auto& u : sh->ev_used) {
-    cudaEventDestroy(u.second.first);
-    cudaEventDestroy(u.second.second);
-  }
+  cudaFree(sh->ops_dev);
+  cudaFree(sh->barrier);
+  cudaFree(sh->phase_clock);
   delete sh;
-  return SHARD_OK;
-}
-
-int shard_set_option(shard_t sh, int option, int value) {
-  if (!sh) return fail(SHARD_EINVAL, "null shard");
-  if (option == SHARD_OPT_GRAPH) {
-    sh->use_graph = value != 0;
-  } else if (option == SHARD_OPT_PDL) {
-    sh->use_pdl = value != 0;
-    for (auto* st : sh->states) {
-      for (auto& kv : st->graphs) {
-        cudaGraphExecDestroy(kv.second.exec);
-        cudaGraphDestroy(kv.second.graph);
-      }
-      st->graphs.clear();
-    }
-  } else {
-    return fail(SHARD_EINVAL, "unknown option %d", option);
-  }
   return SHARD_OK;
 }
 
@@ -627,8 +425,7 @@ int kv_state_alloc(shard_t sh, int n_rows, int capacity, kvstate_t* out) {
   const size_t pool = st->layer_stride * sh->L;
   st->cursor.assign(n_rows, 0);
   st->len_host.assign(n_rows, 0);
-  st->chunk = 64;
-  st->n_chunks = (capacity + st->chunk - 1) / st->chunk;
+  st->n_chunks = (capacity + kAttnChunk - 1) / kAttnChunk;
   int rc = SHARD_OK;
   auto chk = [&](cudaError_t e) {
     if (e != cudaSuccess && rc == SHARD_OK)
@@ -640,11 +437,9 @@ int kv_state_alloc(shard_t sh, int n_rows, int capacity, kvstate_t* out) {
   chk(cudaMalloc(&st->bt[1], sizeof(int) * (size_t)n_rows * capacity));
   chk(cudaMalloc(&st->lens, sizeof(int) * n_rows));
   const int G = sh->Hq / sh->Hkv;
-  chk(cudaMalloc(&st->attn_part, sizeof(float) * attention_part_floats(n_rows, sh->Hkv, st->n_chunks, G, sh->d)));
-  chk(cudaMalloc(&st->attn_counters, sizeof(int) * n_rows * sh->Hkv));
+  chk(cudaMalloc(&st->attn_part, sizeof(float) * step_attention_part_floats(n_rows, sh->Hkv, st->n_chunks, G, sh->d)));
   if (rc == SHARD_OK) {
     chk(cudaMemset(st->lens, 0, sizeof(int) * n_rows));
-    chk(cudaMemset(st->attn_counters, 0, sizeof(int) * n_rows * sh->Hkv));
     chk(cudaMemset(st->k, 0, sizeof(uint16_t) * pool));
     chk(cudaMemset(st->v, 0, sizeof(uint16_t) * pool));
     chk(launch_fill_identity(st->bt[0], n_rows, capacity, -1, nullptr));
@@ -845,26 +640,41 @@ int shard_step(shard_t sh, kvstate_t st, const uint16_t* hidden_in, const int32_
   pa.x = sh->x;
   pa.status = sh->status;
   pa.sp = sh->sp;
-  const int nt = nt_for(M);
-
-  if (sh->use_graph && sh->profile_mask == 0) {
-    GraphEntry* ge = nullptr;
-    rc = get_graph(sh, st, nt, pa, &ge);
-    if (rc) return rc;
-    cudaKernelNodeParams kp = ge->prologue_params;
-    void* args[1] = {&pa};
-    kp.kernelParams = args;
-    kp.extra = nullptr;
-    CUDA_TRY(cudaGraphExecKernelNodeSetParams(ge->exec, ge->prologue, &kp));
-    CUDA_TRY(cudaGraphLaunch(ge->exec, s));
-  } else {
-    {
-      ProfScope ps(sh, PK_PROLOGUE, s);
-      CUDA_TRY(launch_prologue(pa, s, false));
-    }
-    rc = enqueue_layers(sh, st, nt, s, sh->use_pdl);
-    if (rc) return rc;
-  }
+  StepKernelArgs ka{};
+  ka.pro = pa;
+  ka.ops = sh->ops_dev;
+  ka.L = sh->L;
+  ka.H = sh->H;
+  ka.Hq = sh->Hq;
+  ka.Hkv = sh->Hkv;
+  ka.d = sh->d;
+  ka.F = sh->F;
+  ka.Kp_H = sh->Kp_H;
+  ka.Kp_dq = sh->Kp_dq;
+  ka.Kp_F = sh->Kp_F;
+  ka.eps = static_cast<float>(sh->cfg.rms_eps);
+  ka.norms = sh->norms;
+  ka.rope = sh->rope;
+  ka.x = sh->x;
+  ka.act_h = sh->act_h;
+  ka.act_attn = sh->act_attn;
+  ka.act_f = sh->act_f;
+  ka.q = sh->q;
+  ka.partials = sh->partials;
+  ka.counters = sh->counters;
+  ka.kpool = st->k;
+  ka.vpool = st->v;
+  ka.layer_stride = st->layer_stride;
+  ka.cap = st->cap;
+  ka.n_chunks = st->n_chunks;
+  ka.attn_part = st->attn_part;
+  ka.status = sh->status;
+  ka.barrier = sh->barrier;
+  ka.barrier_base = sh->barrier_base;
+  ka.phase_clock = sh->phase_clock;
+  const int grid = sh->num_sms;
+  CUDA_TRY(launch_step(ka, M <= 8 ? 1 : 2, sh->cfg.group, grid, s));
+  sh->barrier_base += (unsigned long long)sh->n_barriers * grid;
   CUDA_TRY(cudaMemcpyAsync(sh->status_host, sh->status, sizeof(int), cudaMemcpyDeviceToHost, s));
 
   for (int b = 0; b < B; ++b) st->cursor[b] += n_new[b];
@@ -1011,36 +821,15 @@ int shard_debug_gemv(shard_t sh, int layer, int op, const uint16_t* x, int M, fl
   return SHARD_OK;
 }
 
-int shard_debug_profile(shard_t sh, unsigned kinds) {
-  if (!sh) return fail(SHARD_EINVAL, "null shard");
-  if (kinds >> PK_N) return fail(SHARD_EINVAL, "unknown kind bits");
-  sh->profile_mask = kinds;
-  return SHARD_OK;
-}
-
-int shard_debug_profile_read(shard_t sh, int kind, double* total_ms, int* launches) {
-  if (!sh || !total_ms || !launches || kind < 0 || kind >= PK_N) return fail(SHARD_EINVAL, "bad argument");
+int shard_debug_phase_times(shard_t sh, double* us, int n) {
+  if (!sh || !us || n < 1) return fail(SHARD_EINVAL, "bad argument");
   CUDA_TRY(cudaSetDevice(sh->device));
-  double t = 0.0;
-  int n = 0;
-  std::vector<std::pair<int, std::pair<cudaEvent_t, cudaEvent_t>>> keep;
-  for (auto& u : sh->ev_used) {
-    if (u.first != kind) {
-      keep.push_back(u);
-      continue;
-    }
-    CUDA_TRY(cudaEventSynchronize(u.second.second));
-    float ms = 0.f;
-    CUDA_TRY(cudaEventElapsedTime(&ms, u.second.first, u.second.second));
-    t += ms;
-    ++n;
-    sh->ev_pool.push_back(u.second.first);
-    sh->ev_pool.push_back(u.second.second);
-  }
-  sh->ev_used.swap(keep);
-  *total_ms = t;
-  *launches = n;
-  return SHARD_OK;
+  CUDA_TRY(cudaDeviceSynchronize());
+  std::vector<unsigned long long> t(sh->n_barriers + 1);
+  CUDA_TRY(cudaMemcpy(t.data(), sh->phase_clock, sizeof(unsigned long long) * t.size(), cudaMemcpyDeviceToHost));
+  const int k = std::min(n, sh->n_barriers);
+  for (int i = 0; i < k; ++i) us[i] = (double)(t[i + 1] - t[i]) * 1e-3;
+  return k;
 }
 
 }  // extern "C"

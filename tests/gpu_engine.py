@@ -19,11 +19,9 @@ def to_dev(a: np.ndarray, dtype=None) -> torch.Tensor:
 
 
 class GpuShard:
-    def __init__(self, shape, weights, graph: bool = True, pdl: bool = True):
+    def __init__(self, shape, weights):
         self.shape = shape
         self.h = pkg.shard_create(pkg.make_config(shape), weights.layers, weights.embedding)
-        pkg.shard_set_option(self.h, pkg.SHARD_OPT_GRAPH, int(graph))
-        pkg.shard_set_option(self.h, pkg.SHARD_OPT_PDL, int(pdl))
 
     def close(self):
         if self.h:

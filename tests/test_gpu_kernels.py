@@ -17,7 +17,7 @@ SHAPES = {
     # one layer of the 8B stage: every projection shape of the workload
     "8b-1layer": synth.ShardShape("8b-1layer", 1, 4096, 32, 8, 128, 14336, 128, 0.02, 0, 1e-5, 500000.0, 4096),
     # ragged: K not a multiple of 128, F not a multiple of 8, group 64
-    "ragged": synth.ShardShape("ragged", 1, 200, 4, 4, 32, 333, 64, 0.02, 0, 1e-5, 10000.0, 256),
+    "ragged": synth.ShardShape("ragged", 1, 200, 4, 4, 64, 333, 64, 0.02, 0, 1e-5, 10000.0, 256),
 }
 
 

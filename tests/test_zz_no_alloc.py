@@ -53,8 +53,8 @@ def test_noalloc_matches_allocating_path_on_consecutive_calls(shape):
 
 
 def test_noalloc_refuses_requests_beyond_its_fixed_scratch():
-    # a 64K-wide down projection: 16 padded activation rows alone need 2 MiB
-    shape = synth.ShardShape("wide-ffn", 1, 64, 1, 1, 64, 65536, 128, 0.02, 0, 1e-5, 10000.0, 64)
+    # a 160K-wide down projection: 16 padded activation rows alone need 5 MiB
+    shape = synth.ShardShape("wide-ffn", 1, 64, 1, 1, 64, 163840, 128, 0.02, 0, 1e-5, 10000.0, 64)
     w = synth.make_weights(shape, 5)
     h = pkg.shard_create(pkg.make_config(shape), w.layers, w.embedding)
     try:
