@@ -12,26 +12,21 @@ constexpr int kCtasPerSm = 1;
 
 template <int NT, int GPU>
 constexpr size_t smem_bytes() {
-  return (size_t)kW * kRingSlots * Geom<GPU>::kUnitBytes + (size_t)kW * kRingSlots * sizeof(uint64_t) +
-         (size_t)kW * 1024 * sizeof(float);
+  return (size_t)kW * kRingSlots * Geom<GPU>::kUnitBytes + (size_t)kW * kRingSlots * sizeof(uint64_t);
 }
 
 template <int NT, int GPU>
 __global__ void __launch_bounds__(kW * 32) gemv_kernel(const GemvArgs a) {
   extern __shared__ __align__(128) uint8_t smem[];
   __shared__ OpDesc s_op[1];
-  __shared__ int s_red_cnt, s_red_seg;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
     s_op[0] = OpDesc{a.units, a.n_rb, a.upr};
-    s_red_cnt = 0;
-    s_red_seg = 0;
   }
   __syncthreads();
   const size_t ring_bytes = (size_t)kW * kRingSlots * Geom<GPU>::kUnitBytes;
   uint8_t* ring = smem + (size_t)warp * kRingSlots * Geom<GPU>::kUnitBytes;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + ring_bytes) + warp * kRingSlots;
-  float* red = reinterpret_cast<float*>(smem + ring_bytes + (size_t)kW * kRingSlots * sizeof(uint64_t));
   WarpStream<GPU> ws;
   ws.init(s_op, 1, blockIdx.x, gridDim.x, warp, ring, bars, lane);
   ws.fill(lane);
@@ -44,9 +39,6 @@ __global__ void __launch_bounds__(kW * 32) gemv_kernel(const GemvArgs a) {
   p.skip = a.sp ? (a.sp->abort_step != 0) : false;
   p.partials = a.partials;
   p.counters = a.counters;
-  p.red = red;
-  p.red_cnt = &s_red_cnt;
-  p.red_seg = &s_red_seg;
   p.status = a.status;
   p.sp = a.sp;
   p.ep = a.ep;
@@ -94,7 +86,7 @@ int gemv_grid(int nt, int num_sms) {
 
 int gemv_warps_per_cta() { return kW; }
 
-size_t gemv_partials_floats(int grid) { return (size_t)grid * 2 * 1024; }
+size_t gemv_partials_floats(int grid) { return (size_t)grid * kW * 2 * kPieceFloats; }
 
 cudaError_t launch_gemv(const GemvArgs& a, int nt, int group, int grid, cudaStream_t s, bool pdl) {
   if (nt == 1) {

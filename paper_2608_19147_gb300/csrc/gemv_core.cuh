@@ -2,29 +2,29 @@
 // kernel and the standalone projection kernel.
 //
 // Work split.  The unit stream of a projection (n_rb row-blocks x upr units,
-// see kernels.h) is cut into gridDim.x contiguous ranges, one per CTA, so
-// every CTA streams the same number of bytes; inside a CTA, warp w takes
-// every kCtaWarps-th unit of the range starting at w.  Each warp owns a ring
-// of kRingSlots shared-memory slots that its lane 0 fills with bulk copies
-// (TMA, non-tensor), one unit per slot, completion tracked by one mbarrier
-// per slot.  Because the weights never depend on earlier work, a warp's ring
-// runs ahead through the *sequence* of projections it will process (the
-// step's q|k|v, o, gate|up, down of every layer): while the warp waits for
-// other work, its next projection's weights are already in flight.
+// see kernels.h) is cut into contiguous runs, one per warp of the grid
+// (warp g = cta * kCtaWarps + warp), so every warp streams the same number of
+// bytes and keeps its sums in registers for as long as its run stays inside
+// one row-block.  Each warp owns a ring of kRingSlots shared-memory slots that
+// its lane 0 fills with bulk copies (TMA, non-tensor), one unit per slot,
+// completion tracked by one mbarrier per slot.  Because the weights never
+// depend on earlier work, a warp's ring runs ahead through the *sequence* of
+// projections it will process (the step's q|k|v, o, gate|up, down of every
+// layer): while the warp waits for other work, its next projection's weights
+// are already in flight.
 //
 // Per unit, a lane turns each 32-bit code word into the four registers of its
 // m16n8k16 A fragment -- (q - z) exactly, in fp16 -- and multiplies them with
 // the activations (the B fragment) on the tensor cores, accumulating in fp32;
 // the fp16 group scale multiplies the fp32 group sum.
 //
-// Reduction.  A CTA's range covers a few row-block segments.  At the end of
-// each segment every warp leaves its partial sums in shared memory; the last
-// warp to arrive (shared-memory counter) adds the kCtaWarps pieces in warp
-// order.  A row-block wholly inside the CTA's range is then finished at once;
-// the pieces of a row-block split between CTAs go to a scratch buffer and the
-// last CTA to arrive (global counter) adds them in CTA order.  Both orders
-// are fixed, so results are deterministic and do not depend on the token
-// count M.
+// Reduction.  A row-block lying wholly inside one warp's run is finished by
+// that warp (epilogue straight from the accumulator registers).  A row-block
+// split between warps gets one piece per warp, stored in the accumulator
+// fragment layout; the last warp to arrive (global counter, acquire-release)
+// adds the pieces in warp order and runs the epilogue.  No warp ever waits
+// for another inside a projection, and the fixed order makes results
+// deterministic and independent of the token count M.
 #pragma once
 #include "common.cuh"
 
@@ -76,18 +76,18 @@ struct WarpStream {
   int f_op, f_u, f_end;
   const uint8_t* f_units;
   uint32_t n_filled, n_used;
+  uint64_t policy;  // L2 evict-first: each weight byte is read once per step
   bool timed_out;
 
-  __device__ __forceinline__ void cta_range(int op, int& cb, int& ce) const {
+  // Run [wb, we) of this warp in op's unit stream.
+  __device__ __forceinline__ void warp_range(int op, int& wb, int& we) const {
     const int T = ops[op].n_rb * ops[op].upr;
-    cb = part_start(T, cta, n_cta);
-    ce = part_start(T, cta + 1, n_cta);
+    const int g = cta * kCtaWarps + warp, nw = n_cta * kCtaWarps;
+    wb = part_start(T, g, nw);
+    we = part_start(T, g + 1, nw);
   }
   __device__ __forceinline__ void open_op(int op) {
-    int cb, ce;
-    cta_range(op, cb, ce);
-    f_u = cb + warp;
-    f_end = ce;
+    warp_range(op, f_u, f_end);
     f_units = ops[op].units;
   }
   // lane 0 initialises the slot barriers; the warp is synced after.
@@ -101,6 +101,7 @@ struct WarpStream {
     ring = ring_;
     bars = bars_;
     n_filled = n_used = 0;
+    policy = l2_policy_evict_first();
     timed_out = false;
     f_op = 0;
     f_u = f_end = 0;
@@ -120,12 +121,12 @@ struct WarpStream {
         open_op(f_op);
       }
       const uint8_t* src = f_units + (size_t)f_u * UB;
-      f_u += kCtaWarps;
+      ++f_u;
       if (lane == 0) {
         const int slot = n_filled % kRingSlots;
         fence_proxy_async_smem();
         mbar_arrive_expect_tx(&bars[slot], UB);
-        bulk_g2s(ring + (size_t)slot * UB, src, UB, &bars[slot]);
+        bulk_g2s_hint(ring + (size_t)slot * UB, src, UB, &bars[slot], policy);
       }
       ++n_filled;
     }
@@ -303,17 +304,17 @@ struct GemvPhase {
   const uint16_t* act;  // fp16 [M][act_ld]
   int act_ld, M;
   bool skip;            // consume the weights but compute nothing (aborted step)
-  float* partials;      // [gridDim.x][2][64][16] pieces of split row-blocks
+  float* partials;      // [n_cta * kCtaWarps][2][kPieceFloats] pieces of split row-blocks
   int* counters;        // [n_rb], zero, self-resetting
-  float* red;           // shared: [kCtaWarps][64][16] warp pieces of one segment
-  int* red_cnt;         // shared: arrivals at the current segment (0 at phase start)
-  int* red_seg;         // shared: segment number the buffer is open for (0 at phase start)
   int* status;
   const StepParams* sp;
   EpiArgs ep;
 };
 
-// Loads the B fragments of unit (ku) for tokens gid (and gid + 8).
+// Floats of one stored piece: [token][64 rows] for up to kMaxTokens tokens.
+constexpr int kPieceFloats = kMaxTokens * kRowsPerBlock;
+
+// Loads the B fragments of input unit ku for tokens gid (and gid + 8).
 template <int NT>
 __device__ __forceinline__ void load_act(uint4 (&act)[NT][2][2], const uint16_t* actp, int act_ld, int M, bool skip,
                                          int ku, int lane) {
@@ -331,115 +332,111 @@ __device__ __forceinline__ void load_act(uint4 (&act)[NT][2][2], const uint16_t*
   }
 }
 
-// End of one row-block segment of a CTA (the cold path): called by every
-// warp of the CTA after leaving its partial sums in shared memory.  The last
-// warp to arrive sums the pieces and finishes the row-block, or hands its
-// piece to the last CTA to arrive at the row-block.  Work items of the
-// reducing warp are (row pair, token): item i takes rows
-// lo = (i % 32 / 8) * 16 + i % 8 and lo + 8 for token i / 32.  The items of a
-// lane (at most kMaxTokens / 2 ... kMaxTokens) are processed together so
-// that their global loads are in flight at the same time.
-static __device__ __noinline__ void segment_end(const GemvPhase& p, int segno, int rb, bool whole, int slot, int cta,
-                                                int n_cta, int T, int rb_begin, int rb_end, int lane) {
-  __syncwarp();
-  int last = 0;
-  if (lane == 0) {
-    __threadfence_block();
-    last = (atomicAdd(p.red_cnt, 1) == kCtaWarps - 1);
-  }
-  last = __shfl_sync(0xffffffffu, last, 0);
-  if (!last) return;
-  __threadfence_block();
+// Finishes row-block rb from the stored pieces of warps g_first..g_last (the
+// cold path): for each token, adds the pieces in warp order, then runs the
+// epilogue.  Lane L takes the row pair lo = (L / 8) * 16 + L % 8 and lo + 8 --
+// a rotary or gate/up pair.  The loads of kBatch pieces are in flight at once.
+static __device__ __noinline__ void finish_rowblock(const GemvPhase& p, int rb, int g_first, int g_last, int T, int nw,
+                                                    int upr, int lane) {
+  constexpr int kBatch = 16;
+  const int rb_begin = rb * upr;
   const int lo = (lane >> 3) * 16 + (lane & 7);
-  const int M = p.M;
-  float vlo[kMaxTokens], vhi[kMaxTokens];
+  for (int m = 0; m < p.M; ++m) {
+    float vlo = 0.f, vhi = 0.f;
+    for (int g0 = g_first; g0 <= g_last; g0 += kBatch) {
+      float a[kBatch], b[kBatch];
 #pragma unroll
-  for (int m = 0; m < kMaxTokens; ++m) {
-    vlo[m] = vhi[m] = 0.f;
-    if (m < M) {
+      for (int i = 0; i < kBatch; ++i) {
+        const int gg = g0 + i;
+        a[i] = b[i] = 0.f;
+        if (gg <= g_last) {
+          const int s0 = part_start(T, gg, nw);
+          if (part_start(T, gg + 1, nw) > s0) {  // non-empty run
+            const float* pc = p.partials + ((size_t)gg * 2 + (s0 < rb_begin ? 1 : 0)) * kPieceFloats + m * kRowsPerBlock;
+            a[i] = __ldcg(pc + lo);
+            b[i] = __ldcg(pc + lo + 8);
+          }
+        }
+      }
 #pragma unroll
-      for (int w = 0; w < kCtaWarps; ++w) {
-        vlo[m] += p.red[(size_t)w * 1024 + lo * 16 + m];
-        vhi[m] += p.red[(size_t)w * 1024 + (lo + 8) * 16 + m];
+      for (int i = 0; i < kBatch; ++i) {
+        vlo += a[i];
+        vhi += b[i];
       }
     }
+    epilogue_pair(p.ep, p.sp, rb * kRowsPerBlock + lo, m, vlo, vhi);
   }
-  // reopen the buffer for the next segment
-  __syncwarp();
-  if (lane == 0) {
-    *reinterpret_cast<volatile int*>(p.red_cnt) = 0;
-    __threadfence_block();
-    *reinterpret_cast<volatile int*>(p.red_seg) = segno + 1;
-  }
-  if (whole) {
+}
+
+// End of one row-block segment of a warp's run.  The piece is stored (slot
+// 0: the run's first segment, slot 1: a later one); a whole row-block is
+// finished at once, a split one by the last of its contributing warps.
+template <int NT>
+__device__ __forceinline__ void piece_end(const GemvPhase& p, const float (&tot)[4][NT][4], int rb, bool whole, int slot,
+                                          int g, int nw, int T, int upr, int lane) {
+  const int gid = lane >> 2, tig = lane & 3;
+  float* mine = p.partials + ((size_t)g * 2 + slot) * kPieceFloats;
 #pragma unroll
-    for (int m = 0; m < kMaxTokens; ++m)
-      if (m < M) epilogue_pair(p.ep, p.sp, rb * kRowsPerBlock + lo, m, vlo[m], vhi[m]);
+  for (int rt = 0; rt < 4; ++rt)
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+      for (int c = 0; c < 2; ++c) {
+        const int m = nt * 8 + 2 * tig + c;
+        if (m < p.M) {
+          __stcg(mine + m * kRowsPerBlock + rt * 16 + gid, tot[rt][nt][c]);
+          __stcg(mine + m * kRowsPerBlock + rt * 16 + gid + 8, tot[rt][nt][2 + c]);
+        }
+      }
+  __syncwarp();
+  if (whole) {
+    finish_rowblock(p, rb, g, g, T, nw, upr, lane);
     return;
   }
-  float* mine_g = p.partials + ((size_t)cta * 2 + slot) * 1024;
-#pragma unroll
-  for (int m = 0; m < kMaxTokens; ++m)
-    if (m < M) {
-      mine_g[lo * 16 + m] = vlo[m];
-      mine_g[(lo + 8) * 16 + m] = vhi[m];
-    }
+  const int rb_begin = rb * upr, rb_end = rb_begin + upr;
+  // warp owning unit x: the largest g with part_start(T, g, nw) <= x
+  const int g_first = static_cast<int>(((long long)(rb_begin + 1) * nw + T - 1) / T - 1);
+  const int g_last = static_cast<int>(((long long)rb_end * nw + T - 1) / T - 1);
+  // with T < nw every non-empty run holds one unit
+  const int expected = (T >= nw) ? (g_last - g_first + 1) : upr;
+  // The warp barrier above orders every lane's piece stores before lane 0's
+  // release; lane 0's acquire is ordered before the merge loads by the warp
+  // barrier below.
+  int last = 0;
+  if (lane == 0) last = (atom_add_acq_rel(&p.counters[rb], 1) == expected - 1);
+  last = __shfl_sync(0xffffffffu, last, 0);
+  if (!last) return;
   __syncwarp();
-  auto cta_of = [&](int uu) { return static_cast<int>(((long long)(uu + 1) * n_cta + T - 1) / T - 1); };
-  const int c_first = cta_of(rb_begin), c_last = cta_of(rb_end - 1);
-  const int expected = (T >= n_cta) ? (c_last - c_first + 1) : (rb_end - rb_begin);
-  int glast = 0;
-  if (lane == 0) glast = (atom_add_acq_rel(&p.counters[rb], 1) == expected - 1);
-  glast = __shfl_sync(0xffffffffu, glast, 0);
-  if (!glast) return;
-#pragma unroll
-  for (int m = 0; m < kMaxTokens; ++m) vlo[m] = vhi[m] = 0.f;
-  for (int cc = c_first; cc <= c_last; ++cc) {
-    const int s0 = part_start(T, cc, n_cta), s1 = part_start(T, cc + 1, n_cta);
-    if (s1 <= s0) continue;  // empty range
-    const float* pc = p.partials + ((size_t)cc * 2 + ((s0 < rb_begin) ? 1 : 0)) * 1024;
-    float a[kMaxTokens], b[kMaxTokens];
-#pragma unroll
-    for (int m = 0; m < kMaxTokens; ++m) {
-      a[m] = (m < M) ? __ldcg(pc + lo * 16 + m) : 0.f;
-      b[m] = (m < M) ? __ldcg(pc + (lo + 8) * 16 + m) : 0.f;
-    }
-#pragma unroll
-    for (int m = 0; m < kMaxTokens; ++m) {
-      vlo[m] += a[m];
-      vhi[m] += b[m];
-    }
-  }
-#pragma unroll
-  for (int m = 0; m < kMaxTokens; ++m)
-    if (m < M) epilogue_pair(p.ep, p.sp, rb * kRowsPerBlock + lo, m, vlo[m], vhi[m]);
+  finish_rowblock(p, rb, g_first, g_last, T, nw, upr, lane);
   if (lane == 0) p.counters[rb] = 0;
 }
 
-// One projection for one warp of a CTA: consume the warp's units from the
-// stream (which must be positioned at this op), then take part in the
-// reduction of every row-block segment of the CTA's range.
+// One projection for one warp: consume the warp's run of units from the
+// stream (which must be positioned at this op) and finish or hand on each
+// row-block segment of it.
+//
+// Not inlined: the step's four projections run this one copy of the code, so
+// it stays in the instruction cache.  The stream state is worked on in a
+// local copy (registers) and written back at the end.
 template <int NT, int GPU>
-__device__ __forceinline__ void gemv_phase(WarpStream<GPU>& ws, int op, const GemvPhase& p, int lane) {
-  int cb, ce;
-  ws.cta_range(op, cb, ce);
-  if (cb >= ce) return;
+__device__ __noinline__ void gemv_phase(WarpStream<GPU>& ws_io, int op, const GemvPhase& p, int lane) {
+  WarpStream<GPU> ws = ws_io;
+  int wb, we;
+  ws.warp_range(op, wb, we);
+  if (wb >= we) return;
   const int upr = ws.ops[op].upr;
   const int T = ws.ops[op].n_rb * upr;
-  const int gid = lane >> 2, tig = lane & 3;
+  const int g = ws.cta * kCtaWarps + ws.warp, nw = ws.n_cta * kCtaWarps;
   const uint16_t* actp = p.act;
   const int act_ld = p.act_ld, M = p.M;
   const bool skip = p.skip;
-  int u = cb + ws.warp;  // this warp's next unit
-  int rb = cb / upr;
-  int ku = u - rb * upr;  // input unit of u within its row-block (may pass upr)
-  while (ku >= upr) ku -= upr;
+  int rb = wb / upr;
+  int ku = wb - rb * upr;
   uint4 nxt[NT][2][2];
-  if (u < ce) load_act<NT>(nxt, actp, act_ld, M, skip, ku, lane);
-  int segno = 0;
-  for (int seg = cb; seg < ce; ++segno, ++rb) {
-    const int rb_begin = rb * upr, rb_end = rb_begin + upr;
-    const int seg_end = ce < rb_end ? ce : rb_end;
+  load_act<NT>(nxt, actp, act_ld, M, skip, ku, lane);
+  for (int u = wb; u < we; ++rb) {
+    const int seg_begin = u, rb_end = (rb + 1) * upr;
+    const int seg_end = we < rb_end ? we : rb_end;
     float tot[4][NT][4];
 #pragma unroll
     for (int rt = 0; rt < 4; ++rt)
@@ -447,7 +444,7 @@ __device__ __forceinline__ void gemv_phase(WarpStream<GPU>& ws, int op, const Ge
       for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
         for (int q = 0; q < 4; ++q) tot[rt][nt][q] = 0.f;
-    for (; u < seg_end; u += kCtaWarps) {
+    for (; u < seg_end; ++u) {
       uint4 cur[NT][2][2];
 #pragma unroll
       for (int nt = 0; nt < NT; ++nt)
@@ -455,44 +452,18 @@ __device__ __forceinline__ void gemv_phase(WarpStream<GPU>& ws, int op, const Ge
         for (int kc = 0; kc < 2; ++kc)
 #pragma unroll
           for (int h = 0; h < 2; ++h) cur[nt][kc][h] = nxt[nt][kc][h];
-      ku += kCtaWarps;
-      while (ku >= upr) ku -= upr;
-      if (u + kCtaWarps < ce) load_act<NT>(nxt, actp, act_ld, M, skip, ku, lane);
+      if (++ku == upr) ku = 0;
+      if (u + 1 < we) load_act<NT>(nxt, actp, act_ld, M, skip, ku, lane);
       const uint8_t* U = ws.acquire();
       if (!skip && !ws.timed_out) mma_unit<NT, GPU>(U, cur, tot, lane);
       ws.release(lane);
     }
     if (!skip) {
-      if (lane == 0) {
-        uint32_t it = 0;
-        while (*reinterpret_cast<volatile int*>(p.red_seg) != segno) {
-          if (++it > (1u << 22)) {
-            atomicOr(p.status, ST_WAIT_TIMEOUT);
-            break;
-          }
-          __nanosleep(32);
-        }
-      }
-      __syncwarp();
-      float* mine = p.red + (size_t)ws.warp * 1024;
-#pragma unroll
-      for (int rt = 0; rt < 4; ++rt)
-#pragma unroll
-        for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-          for (int c = 0; c < 2; ++c) {
-            const int m = nt * 8 + 2 * tig + c;
-            if (m < M) {
-              mine[(rt * 16 + gid) * 16 + m] = tot[rt][nt][c];
-              mine[(rt * 16 + gid + 8) * 16 + m] = tot[rt][nt][2 + c];
-            }
-          }
-      const bool whole = (seg == rb_begin && seg_end == rb_end);
-      const int slot = (cb < rb_begin) ? 1 : 0;
-      segment_end(p, segno, rb, whole, slot, ws.cta, ws.n_cta, T, rb_begin, rb_end, lane);
+      const bool whole = (seg_begin == rb * upr && seg_end == rb_end);
+      piece_end<NT>(p, tot, rb, whole, seg_begin == wb ? 0 : 1, g, nw, T, upr, lane);
     }
-    seg = seg_end;
   }
+  ws_io = ws;
 }
 
 }  // namespace shard

@@ -134,7 +134,7 @@ struct GemvArgs {
   int act_ld;
   int M;                // tokens when sp == nullptr
   const StepParams* sp; // step parameters (nullptr on the standalone path)
-  float* partials;      // [grid][2][64][16] fp32 scratch
+  float* partials;      // [grid warps][2][piece] fp32 scratch, gemv_partials_floats(grid)
   int* counters;        // [n_rb] zero-initialised, self-resetting
   int* status;
   EpiArgs ep;
@@ -189,7 +189,7 @@ struct StepKernelArgs {
   uint16_t* act_attn;        // [16][Kp_dq]
   uint16_t* act_f;           // [16][Kp_F]
   float* q;                  // [16][Hq*d]
-  float* partials;           // projection pieces [grid][2][64][16]
+  float* partials;           // projection pieces, gemv_partials_floats(grid)
   int* counters;             // [max row-blocks]
   uint16_t* kpool;           // [L][n_rows][Hkv][cap][d]
   uint16_t* vpool;

@@ -356,8 +356,7 @@ int shard_create(const shard_config* cfg, const shard_weights_host* w, shard_t* 
   CUDA_TRY(cudaMalloc(&sh->q, sizeof(float) * kMaxTokens * sh->dq));
   for (int nt = 1; nt <= 2; ++nt) sh->grid[nt] = gemv_grid(nt, sh->num_sms);
   {
-    const size_t step_pieces = (size_t)sh->num_sms * 2 * 1024;
-    const size_t n = std::max(gemv_partials_floats(std::max(sh->grid[1], sh->grid[2])), step_pieces);
+    const size_t n = gemv_partials_floats(std::max(std::max(sh->grid[1], sh->grid[2]), sh->num_sms));
     CUDA_TRY(cudaMalloc(&sh->partials, sizeof(float) * n));
   }
   CUDA_TRY(cudaMalloc(&sh->counters, sizeof(int) * sh->max_rb));

@@ -28,11 +28,9 @@ template <int GPU>
 struct StepSmem {
   static constexpr size_t kRing = (size_t)kWarps * kRingSlots * Geom<GPU>::kUnitBytes;
   static constexpr size_t kBars = (size_t)kWarps * kRingSlots * sizeof(uint64_t);
-  // union: attention query staging / projection reduction buffer
+  // attention query staging
   static constexpr size_t kQ = (size_t)kWarps * kQGroup * 128 * sizeof(float);  // d <= 128
-  static constexpr size_t kRed = (size_t)kWarps * 1024 * sizeof(float);
-  static constexpr size_t kUnion = kQ > kRed ? kQ : kRed;
-  static constexpr size_t kFixed = kRing + kBars + kUnion;  // + the op table (4L entries)
+  static constexpr size_t kFixed = kRing + kBars + kQ;  // + the op table (4L entries)
   static size_t total(int n_layers) { return kFixed + (size_t)4 * n_layers * sizeof(OpDesc); }
 };
 
@@ -54,13 +52,10 @@ __device__ __forceinline__ void red_release_add(unsigned long long* p, unsigned 
   asm volatile("red.release.gpu.global.add.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
 }
 
-// Also resets the CTA's projection-reduction state for the next phase.
 __device__ void grid_sync(unsigned long long* ctr, unsigned long long& target, int* status,
-                          unsigned long long* clock, int& nsync, int* red_cnt, int* red_seg) {
+                          unsigned long long* clock, int& nsync) {
   __syncthreads();
   if (threadIdx.x == 0) {
-    *red_cnt = 0;
-    *red_seg = 0;
     target += gridDim.x;
     red_release_add(ctr, 1ULL);
     // bounded: after ~2^22 polls, or once any CTA has given up, stop waiting
@@ -470,20 +465,14 @@ __device__ __noinline__ void attn_merge_warp(const AttnView& a, const StepParams
 template <int NT, int GPU, int DPL>
 __global__ void __launch_bounds__(kThreads, 1) step_kernel(const StepKernelArgs a) {
   extern __shared__ __align__(128) uint8_t smem[];
-  __shared__ int s_red_cnt, s_red_seg;
   using SS = StepSmem<GPU>;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int gw = blockIdx.x * kWarps + warp, NW = gridDim.x * kWarps;
   uint8_t* ring = smem + (size_t)warp * kRingSlots * Geom<GPU>::kUnitBytes;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + SS::kRing) + warp * kRingSlots;
-  float* uni = reinterpret_cast<float*>(smem + SS::kRing + SS::kBars);
-  float* qs = uni + (size_t)warp * kQGroup * 128;
+  float* qs = reinterpret_cast<float*>(smem + SS::kRing + SS::kBars) + (size_t)warp * kQGroup * 128;
   OpDesc* s_ops = reinterpret_cast<OpDesc*>(smem + SS::kFixed);
   for (int i = threadIdx.x; i < 4 * a.L; i += kThreads) s_ops[i] = a.ops[i];
-  if (threadIdx.x == 0) {
-    s_red_cnt = 0;
-    s_red_seg = 0;
-  }
   __syncthreads();
   unsigned long long target = a.barrier_base;
   int nsync = 1;
@@ -494,7 +483,7 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const StepKernelArgs 
   ws.fill(lane);
 
   if (blockIdx.x == 0) prologue_cta(a.pro);
-  grid_sync(a.barrier, target, a.status, a.phase_clock, nsync, &s_red_cnt, &s_red_seg);
+  grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
 
   const StepParams* sp = a.pro.sp;
   const bool skip = __ldcg(&sp->abort_step) != 0;
@@ -509,9 +498,6 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const StepKernelArgs 
     gp.skip = skip;
     gp.partials = a.partials;
     gp.counters = a.counters;
-    gp.red = uni;
-    gp.red_cnt = &s_red_cnt;
-    gp.red_seg = &s_red_seg;
     gp.status = a.status;
     gp.sp = sp;
     gp.ep.kind = epi;
@@ -532,9 +518,9 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const StepKernelArgs 
     const uint16_t* nrm = a.norms + (size_t)l * 2 * a.H;
     // attention block
     if (!skip) rmsnorm_cta(a.x, a.H, nrm, a.eps, a.act_h, a.Kp_H, M);
-    grid_sync(a.barrier, target, a.status, a.phase_clock, nsync, &s_red_cnt, &s_red_seg);
+    grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
     gemv(4 * l + 0, EPI_QKV, a.act_h, a.Kp_H, l);
-    grid_sync(a.barrier, target, a.status, a.phase_clock, nsync, &s_red_cnt, &s_red_seg);
+    grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
     if (!skip) {
       AttnView av{};
       av.q = a.q;
@@ -555,7 +541,7 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const StepKernelArgs 
         int b, hk, c;
         if (decode_item(sp, a.Hkv, item, b, hk, c)) attn_partial_warp<DPL>(av, sp, b, hk, c, qs, lane);
       }
-      grid_sync(a.barrier, target, a.status, a.phase_clock, nsync, &s_red_cnt, &s_red_seg);
+      grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
       // merge items: (b, hk, query)
       const int G = a.Hq / a.Hkv;
       total = 0;
@@ -571,18 +557,18 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const StepKernelArgs 
         attn_merge_warp<DPL>(av, sp, b, r / Qb, r % Qb, lane);
       }
     } else {
-      grid_sync(a.barrier, target, a.status, a.phase_clock, nsync, &s_red_cnt, &s_red_seg);
+      grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
     }
-    grid_sync(a.barrier, target, a.status, a.phase_clock, nsync, &s_red_cnt, &s_red_seg);
+    grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
     gemv(4 * l + 1, EPI_RESID, a.act_attn, a.Kp_dq, l);
-    grid_sync(a.barrier, target, a.status, a.phase_clock, nsync, &s_red_cnt, &s_red_seg);
+    grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
     // MLP block
     if (!skip) rmsnorm_cta(a.x, a.H, nrm + a.H, a.eps, a.act_h, a.Kp_H, M);
-    grid_sync(a.barrier, target, a.status, a.phase_clock, nsync, &s_red_cnt, &s_red_seg);
+    grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
     gemv(4 * l + 2, EPI_SWIGLU, a.act_h, a.Kp_H, l);
-    grid_sync(a.barrier, target, a.status, a.phase_clock, nsync, &s_red_cnt, &s_red_seg);
+    grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
     gemv(4 * l + 3, EPI_RESID, a.act_f, a.Kp_F, l);
-    if (l + 1 < a.L) grid_sync(a.barrier, target, a.status, a.phase_clock, nsync, &s_red_cnt, &s_red_seg);
+    if (l + 1 < a.L) grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
   }
   if (ws.timed_out && lane == 0) atomicOr(a.status, ST_WAIT_TIMEOUT);
 }
