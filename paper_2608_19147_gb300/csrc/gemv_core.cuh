@@ -53,8 +53,16 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
-// Start of part i of n of a stream of T units (T * n < 2^63).
-__device__ __forceinline__ int part_start(int T, int i, int n) { return static_cast<int>((long long)T * i / n); }
+// Start of part i of n of a stream of T units.  32-bit arithmetic: the host
+// checks (T + 1) * n < 2^32 for every projection when a shard is created.
+__device__ __forceinline__ int part_start(int T, int i, int n) {
+  return static_cast<int>(static_cast<uint32_t>(T) * static_cast<uint32_t>(i) / static_cast<uint32_t>(n));
+}
+// The part owning unit x: the largest i with part_start(T, i, n) <= x.
+__device__ __forceinline__ int part_of(int T, int x, int n) {
+  return static_cast<int>((static_cast<uint32_t>(x + 1) * static_cast<uint32_t>(n) + static_cast<uint32_t>(T) - 1u) /
+                          static_cast<uint32_t>(T)) - 1;
+}
 
 __device__ __forceinline__ int atom_add_acq_rel(int* p, int v) {
   int old;
@@ -336,11 +344,18 @@ __device__ __forceinline__ void load_act(uint4 (&act)[NT][2][2], const uint16_t*
 // cold path): for each token, adds the pieces in warp order, then runs the
 // epilogue.  Lane L takes the row pair lo = (L / 8) * 16 + L % 8 and lo + 8 --
 // a rotary or gate/up pair.  The loads of kBatch pieces are in flight at once.
+//
+// Which slot holds a warp's piece: every contributor after the first started
+// its run inside the row-block (slot 0); the first contributor used slot 1
+// if its run started before the row-block.  When T < nw some runs are empty
+// and each non-empty run is a single unit.
 static __device__ __noinline__ void finish_rowblock(const GemvPhase& p, int rb, int g_first, int g_last, int T, int nw,
                                                     int upr, int lane) {
   constexpr int kBatch = 16;
   const int rb_begin = rb * upr;
   const int lo = (lane >> 3) * 16 + (lane & 7);
+  const bool dense = T >= nw;
+  const size_t first_off = ((size_t)g_first * 2 + (part_start(T, g_first, nw) < rb_begin ? 1 : 0)) * kPieceFloats;
   for (int m = 0; m < p.M; ++m) {
     float vlo = 0.f, vhi = 0.f;
     for (int g0 = g_first; g0 <= g_last; g0 += kBatch) {
@@ -349,13 +364,12 @@ static __device__ __noinline__ void finish_rowblock(const GemvPhase& p, int rb, 
       for (int i = 0; i < kBatch; ++i) {
         const int gg = g0 + i;
         a[i] = b[i] = 0.f;
-        if (gg <= g_last) {
-          const int s0 = part_start(T, gg, nw);
-          if (part_start(T, gg + 1, nw) > s0) {  // non-empty run
-            const float* pc = p.partials + ((size_t)gg * 2 + (s0 < rb_begin ? 1 : 0)) * kPieceFloats + m * kRowsPerBlock;
-            a[i] = __ldcg(pc + lo);
-            b[i] = __ldcg(pc + lo + 8);
-          }
+        bool live = gg <= g_last;
+        if (live && !dense) live = part_start(T, gg + 1, nw) > part_start(T, gg, nw);
+        if (live) {
+          const float* pc = p.partials + (gg == g_first ? first_off : (size_t)gg * 2 * kPieceFloats) + m * kRowsPerBlock;
+          a[i] = __ldcg(pc + lo);
+          b[i] = __ldcg(pc + lo + 8);
         }
       }
 #pragma unroll
@@ -394,9 +408,7 @@ __device__ __forceinline__ void piece_end(const GemvPhase& p, const float (&tot)
     return;
   }
   const int rb_begin = rb * upr, rb_end = rb_begin + upr;
-  // warp owning unit x: the largest g with part_start(T, g, nw) <= x
-  const int g_first = static_cast<int>(((long long)(rb_begin + 1) * nw + T - 1) / T - 1);
-  const int g_last = static_cast<int>(((long long)rb_end * nw + T - 1) / T - 1);
+  const int g_first = part_of(T, rb_begin, nw), g_last = part_of(T, rb_end - 1, nw);
   // with T < nw every non-empty run holds one unit
   const int expected = (T >= nw) ? (g_last - g_first + 1) : upr;
   // The warp barrier above orders every lane's piece stores before lane 0's

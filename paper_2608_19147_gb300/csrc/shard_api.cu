@@ -248,6 +248,9 @@ int shard_create(const shard_config* cfg, const shard_weights_host* w, shard_t* 
       op.group = c.group;
       op.bytes = (size_t)op.n_rb * op.upr * ub;
       op.dims = OpDims{k, sh->Hq, sh->Hkv, sh->d, sh->F, sh->H};
+      // the device splits the unit stream with 32-bit arithmetic
+      if (((uint64_t)op.n_rb * op.upr + 1) * ((uint64_t)sh->num_sms * gemv_warps_per_cta()) >= (1ull << 32))
+        return fail(SHARD_EUNSUPPORTED, "a projection has too many units for this GPU's warp count");
       total += op.bytes;
       sh->max_rb = std::max(sh->max_rb, op.n_rb);
     }

@@ -14,6 +14,8 @@
 //
 // Barrier waits are bounded: a wait that runs out sets a status bit and
 // proceeds (the step's results are then reported invalid) instead of hanging.
+#include <type_traits>
+
 #include "gemv_core.cuh"
 
 namespace shard {
@@ -21,15 +23,14 @@ namespace {
 
 constexpr int kWarps = kCtaWarps;
 constexpr int kThreads = kWarps * 32;
-constexpr int kQGroup = 8;        // queries staged per warp at a time
 constexpr int kChunk = 32;        // cache entries per attention item (one per lane)
 
 template <int GPU>
 struct StepSmem {
   static constexpr size_t kRing = (size_t)kWarps * kRingSlots * Geom<GPU>::kUnitBytes;
   static constexpr size_t kBars = (size_t)kWarps * kRingSlots * sizeof(uint64_t);
-  // attention query staging
-  static constexpr size_t kQ = (size_t)kWarps * kQGroup * 128 * sizeof(float);  // d <= 128
+  // attention item area (AttnSmem)
+  static constexpr size_t kQ = 32 * 1024;
   static constexpr size_t kFixed = kRing + kBars + kQ;  // + the op table (4L entries)
   static size_t total(int n_layers) { return kFixed + (size_t)4 * n_layers * sizeof(OpDesc); }
 };
@@ -224,11 +225,14 @@ __device__ __noinline__ void rmsnorm_cta(const float* x, int H, const uint16_t* 
 
 // ---------------------------------------------------------------------------
 // Attention.  Item = (request b, kv head hk, chunk c of kChunk entries); one
-// warp per item.  Lane j scores entry j0 + j against every query of the item
-// (the request's new tokens x the kv head's query heads), then lanes switch
-// to owning head dims for the value sum.  Each item writes (max, sum of exp,
-// unnormalised output) per query; the merge phase combines chunks in order.
+// CTA per item.  Each item writes (max, sum of exp, unnormalised output) per
+// query (the request's new tokens x the kv head's query heads); the merge
+// phase combines a request's chunks in order.
 // ---------------------------------------------------------------------------
+// A partial is (max, sum of exp, 2 unused, unnormalised output[d]): the
+// output starts 16-byte aligned.
+__host__ __device__ constexpr int part_stride(int d) { return d + 4; }
+
 struct AttnView {
   const float* q;
   const uint16_t* kpool;
@@ -255,207 +259,220 @@ __device__ __forceinline__ bool decode_item(const StepParams* sp, int Hkv, int i
   return false;
 }
 
-template <int DPL>  // head dims per lane (d = 32 * DPL)
-__device__ __noinline__ void attn_partial_warp(const AttnView& a, const StepParams* sp, int b, int hk, int c, float* qs,
-                                               int lane) {
-  constexpr int d = 32 * DPL;
-  constexpr int KV8 = d / 8;  // 16-byte pieces per K row
+__device__ __forceinline__ float2 h2f2(uint32_t u) {
+  __half2 h;
+  memcpy(&h, &u, sizeof(h));
+  return __half22float2(h);
+}
+
+// Shared-memory layout of one attention item.
+template <int DPL>
+struct AttnSmem {
+  static constexpr int d = 32 * DPL;
+  static constexpr int kKld = d + 8;  // padded K row (halves): consecutive rows start on different banks
+  static constexpr int kQg = 16;      // queries per group
+  static constexpr size_t kK = (size_t)kChunk * kKld * 2;
+  static constexpr size_t kV = (size_t)kChunk * d * 2;
+  static constexpr size_t kQ = (size_t)kQg * d * 4;
+  static constexpr size_t kP = (size_t)kQg * kChunk * 4;
+  static constexpr size_t kBytes = kK + kV + kQ + kP + 2 * kChunk * sizeof(int);
+};
+
+// One item, processed by the whole CTA:
+//   1. the chunk's slots (beam table) and mask bits;
+//   2. its K and V rows and the first query group into shared memory, every
+//      load of a thread in flight at once;
+//   3. scores: warp w takes queries w, w + kWarps, ...; lane = entry; the
+//      softmax pieces (max, sum of exp) per query across the lanes;
+//   4. values: thread = (query, pair of head dims), sum over the entries.
+template <int DPL>
+__device__ __noinline__ void attn_item_cta(const AttnView& a, const StepParams* sp, int b, int hk, int c,
+                                           uint8_t* area) {
+  using S = AttnSmem<DPL>;
+  constexpr int d = S::d, KP = d / 8;  // 16-byte pieces per row
+  uint16_t* Ks = reinterpret_cast<uint16_t*>(area);
+  uint16_t* Vs = reinterpret_cast<uint16_t*>(area + S::kK);
+  float* qsm = reinterpret_cast<float*>(area + S::kK + S::kV);
+  float* ps = reinterpret_cast<float*>(area + S::kK + S::kV + S::kQ);
+  int* slot_s = reinterpret_cast<int*>(area + S::kK + S::kV + S::kQ + S::kP);
+  int* vis_s = slot_s + kChunk;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int L = sp->req_len[b], P = sp->req_P[b];
   const int tok0 = sp->req_tok0[b], nb = sp->req_tok0[b + 1] - tok0;
   const int G = a.Hq / a.Hkv, Q = nb * G;
   const int j0 = c * kChunk, nj = min(kChunk, L - j0);
-  const int jg = j0 + lane;
-  const bool in_range = lane < nj;
-  int slot = 0;
-  bool visible_base = false;
-  if (in_range) {
-    slot = __ldcg(sp->bt + (size_t)b * a.cap + jg);
-    visible_base = __ldcg(sp->mask + (size_t)b * sp->mask_stride + jg) != 0;
-  }
-  const size_t krow = (((size_t)(slot / a.cap) * a.Hkv + hk) * a.cap + slot % a.cap) * d;
   const float scale = rsqrtf(static_cast<float>(d));
-  float* part = a.part + ((((size_t)b * a.Hkv + hk) * a.n_chunks + c) * a.qmax) * (d + 2);
-  // this lane's K row, all pieces in flight at once
-  uint4 kw[KV8];
-  const uint4* kr = reinterpret_cast<const uint4*>(a.kpool + krow);
-#pragma unroll
-  for (int t = 0; t < KV8; ++t) kw[t] = in_range ? __ldcg(kr + t) : make_uint4(0, 0, 0, 0);
-  for (int q0 = 0; q0 < Q; q0 += kQGroup) {
-    const int qn = min(kQGroup, Q - q0);
-    // stage this group's queries (fp32) in the warp's shared area
-    __syncwarp();
-    {
-      float qv[kQGroup * DPL];
-#pragma unroll
-      for (int i = 0; i < kQGroup; ++i)
-#pragma unroll
-        for (int u = 0; u < DPL; ++u) {
-          const int qi = q0 + i, t = u * 32 + lane;
-          qv[i * DPL + u] = (i < qn) ? __ldcg(a.q + (size_t)(tok0 + qi / G) * a.Hq * d + (hk * G + qi % G) * d + t) : 0.f;
-        }
-#pragma unroll
-      for (int i = 0; i < kQGroup; ++i)
-#pragma unroll
-        for (int u = 0; u < DPL; ++u) qs[i * d + u * 32 + lane] = qv[i * DPL + u];
+  float* part = a.part + ((((size_t)b * a.Hkv + hk) * a.n_chunks + c) * a.qmax) * part_stride(d);
+  // query qi of the item is head hk * G + qi % G of token tok0 + qi / G
+  auto q_src = [&](int qi) { return a.q + (size_t)(tok0 + qi / G) * a.Hq * d + (hk * G + qi % G) * d; };
+
+  if (tid < kChunk) {
+    int slot = 0, vis = 0;
+    if (tid < nj) {
+      slot = __ldcg(sp->bt + (size_t)b * a.cap + j0 + tid);
+      vis = __ldcg(sp->mask + (size_t)b * sp->mask_stride + j0 + tid) != 0;
     }
-    __syncwarp();
-    // scores: lane = entry
-    float s[kQGroup];
+    slot_s[tid] = slot;
+    vis_s[tid] = vis;
+  }
+  __syncthreads();
+  {
+    constexpr int kRowPieces = kChunk * KP;
+    constexpr int kPer = (2 * kRowPieces + kThreads - 1) / kThreads;
+    constexpr int kQPieces = S::kQg * d / 4;
+    constexpr int kQPer = (kQPieces + kThreads - 1) / kThreads;
+    const int qn0 = min(S::kQg, Q);
+    uint4 v[kPer];
+    float4 qv[kQPer];
 #pragma unroll
-    for (int i = 0; i < kQGroup; ++i) s[i] = 0.f;
-#pragma unroll
-    for (int t8 = 0; t8 < KV8; ++t8) {
-      const uint32_t kk[4] = {kw[t8].x, kw[t8].y, kw[t8].z, kw[t8].w};
-      float kf[8];
-#pragma unroll
-      for (int v = 0; v < 4; ++v) {
-        kf[2 * v] = h2f(static_cast<uint16_t>(kk[v] & 0xFFFFu));
-        kf[2 * v + 1] = h2f(static_cast<uint16_t>(kk[v] >> 16));
-      }
-#pragma unroll
-      for (int i = 0; i < kQGroup; ++i) {
-        if (i < qn) {
-          const float4 qa = *reinterpret_cast<const float4*>(qs + i * d + t8 * 8);
-          const float4 qb = *reinterpret_cast<const float4*>(qs + i * d + t8 * 8 + 4);
-          s[i] = fmaf(qa.x, kf[0], s[i]);
-          s[i] = fmaf(qa.y, kf[1], s[i]);
-          s[i] = fmaf(qa.z, kf[2], s[i]);
-          s[i] = fmaf(qa.w, kf[3], s[i]);
-          s[i] = fmaf(qb.x, kf[4], s[i]);
-          s[i] = fmaf(qb.y, kf[5], s[i]);
-          s[i] = fmaf(qb.z, kf[6], s[i]);
-          s[i] = fmaf(qb.w, kf[7], s[i]);
-        }
+    for (int i = 0; i < kPer; ++i) {
+      const int pi = tid + i * kThreads, r = (pi % kRowPieces) / KP;
+      v[i] = make_uint4(0, 0, 0, 0);
+      if (pi < 2 * kRowPieces && r < nj) {
+        const int sl = slot_s[r];
+        const size_t row = (((size_t)(sl / a.cap) * a.Hkv + hk) * a.cap + sl % a.cap) * d;
+        v[i] = __ldcg(reinterpret_cast<const uint4*>((pi >= kRowPieces ? a.vpool : a.kpool) + row) + pi % KP);
       }
     }
-    // softmax pieces per query (entries across lanes)
-    float p[kQGroup];
 #pragma unroll
-    for (int i = 0; i < kQGroup; ++i) {
-      p[i] = 0.f;
-      if (i >= qn) continue;
-      const int qi = q0 + i;
-      const bool vis = in_range && visible_base && jg <= P + qi / G;
-      const float v = vis ? s[i] * scale : -INFINITY;
-      float mx = v;
+    for (int i = 0; i < kQPer; ++i) {
+      const int pi = tid + i * kThreads, qi = pi / (d / 4);
+      qv[i] = (pi < kQPieces && qi < qn0) ? __ldcg(reinterpret_cast<const float4*>(q_src(qi)) + pi % (d / 4))
+                                          : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int i = 0; i < kPer; ++i) {
+      const int pi = tid + i * kThreads, r = (pi % kRowPieces) / KP;
+      if (pi < 2 * kRowPieces) {
+        uint4* dst = pi >= kRowPieces ? reinterpret_cast<uint4*>(Vs + r * d) : reinterpret_cast<uint4*>(Ks + r * S::kKld);
+        dst[pi % KP] = v[i];
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < kQPer; ++i) {
+      const int pi = tid + i * kThreads;
+      if (pi < kQPieces) reinterpret_cast<float4*>(qsm)[pi] = qv[i];
+    }
+  }
+  for (int q0 = 0; q0 < Q; q0 += S::kQg) {
+    const int qn = min(S::kQg, Q - q0);
+    if (q0 > 0) {
+      __syncthreads();
+      for (int pi = tid; pi < qn * (d / 4); pi += kThreads)
+        reinterpret_cast<float4*>(qsm)[pi] =
+            __ldcg(reinterpret_cast<const float4*>(q_src(q0 + pi / (d / 4))) + pi % (d / 4));
+    }
+    __syncthreads();
+    for (int qi = warp; qi < qn; qi += kWarps) {
+      const float* qq = qsm + qi * d;
+      const uint16_t* kr = Ks + lane * S::kKld;
+      float s = 0.f;
+#pragma unroll 4
+      for (int t = 0; t < KP; ++t) {
+        const uint4 kk = *reinterpret_cast<const uint4*>(kr + t * 8);
+        const float4 qa = *reinterpret_cast<const float4*>(qq + t * 8);
+        const float4 qb = *reinterpret_cast<const float4*>(qq + t * 8 + 4);
+        float2 f = h2f2(kk.x);
+        s = fmaf(qa.x, f.x, s);
+        s = fmaf(qa.y, f.y, s);
+        f = h2f2(kk.y);
+        s = fmaf(qa.z, f.x, s);
+        s = fmaf(qa.w, f.y, s);
+        f = h2f2(kk.z);
+        s = fmaf(qb.x, f.x, s);
+        s = fmaf(qb.y, f.y, s);
+        f = h2f2(kk.w);
+        s = fmaf(qb.z, f.x, s);
+        s = fmaf(qb.w, f.y, s);
+      }
+      const int q = q0 + qi;
+      const bool vis = lane < nj && vis_s[lane] && j0 + lane <= P + q / G;
+      const float val = vis ? s * scale : -INFINITY;
+      float mx = val;
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-      const float e = vis ? expf(v - mx) : 0.f;
+      const float e = vis ? expf(val - mx) : 0.f;
       float l = e;
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
-      p[i] = e;
+      ps[qi * kChunk + lane] = e;
       if (lane == 0) {
-        part[(size_t)qi * (d + 2)] = mx;
-        part[(size_t)qi * (d + 2) + 1] = l;
+        part[(size_t)q * part_stride(d)] = mx;
+        part[(size_t)q * part_stride(d) + 1] = l;
       }
     }
-    // values: lane owns dims [DPL*lane, DPL*lane + DPL); rows in batches of 8,
-    // the next batch in flight while one is summed
-    float acc[kQGroup][DPL];
-#pragma unroll
-    for (int i = 0; i < kQGroup; ++i)
-#pragma unroll
-      for (int u = 0; u < DPL; ++u) acc[i][u] = 0.f;
-    auto load_v = [&](int jb, uint32_t (&vw)[8][DPL / 2]) {
-#pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        const int sj = __shfl_sync(0xffffffffu, slot, (jb + u) & 31);
-        if (jb + u < nj) {
-          const size_t vrow = (((size_t)(sj / a.cap) * a.Hkv + hk) * a.cap + sj % a.cap) * d;
-          if constexpr (DPL == 4) {
-            const uint2 t = __ldcg(reinterpret_cast<const uint2*>(a.vpool + vrow) + lane);
-            vw[u][0] = t.x;
-            vw[u][DPL / 2 - 1] = t.y;
-          } else {
-            vw[u][0] = __ldcg(reinterpret_cast<const uint32_t*>(a.vpool + vrow) + lane);
-          }
-        } else {
-#pragma unroll
-          for (int v = 0; v < DPL / 2; ++v) vw[u][v] = 0u;
-        }
+    __syncthreads();
+    for (int w = tid; w < qn * (d / 2); w += kThreads) {
+      const int qi = w / (d / 2), dp = w % (d / 2);
+      const float* pq = ps + qi * kChunk;
+      float o0 = 0.f, o1 = 0.f;
+#pragma unroll 8
+      for (int e = 0; e < kChunk; ++e) {  // rows past nj are zero with weight zero
+        const float pe = pq[e];
+        const float2 vf = h2f2(*reinterpret_cast<const uint32_t*>(Vs + e * d + 2 * dp));
+        o0 = fmaf(pe, vf.x, o0);
+        o1 = fmaf(pe, vf.y, o1);
       }
-    };
-    uint32_t vbuf[2][8][DPL / 2];
-    load_v(0, vbuf[0]);
-#pragma unroll 1
-    for (int jb = 0, cur = 0; jb < nj; jb += 8, cur ^= 1) {
-      if (jb + 8 < nj) {
-        if (cur == 0) load_v(jb + 8, vbuf[1]);
-        else load_v(jb + 8, vbuf[0]);
-      }
-#pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        float vf[DPL];
-#pragma unroll
-        for (int v = 0; v < DPL / 2; ++v) {
-          const uint32_t x = cur == 0 ? vbuf[0][u][v] : vbuf[1][u][v];
-          vf[2 * v] = h2f(static_cast<uint16_t>(x & 0xFFFFu));
-          vf[2 * v + 1] = h2f(static_cast<uint16_t>(x >> 16));
-        }
-#pragma unroll
-        for (int i = 0; i < kQGroup; ++i) {
-          const float pj = __shfl_sync(0xffffffffu, p[i], (jb + u) & 31);
-#pragma unroll
-          for (int v = 0; v < DPL; ++v) acc[i][v] = fmaf(pj, vf[v], acc[i][v]);
-        }
-      }
-    }
-#pragma unroll
-    for (int i = 0; i < kQGroup; ++i) {
-      if (i >= qn) continue;
-      float* o = part + (size_t)(q0 + i) * (d + 2) + 2 + DPL * lane;
-#pragma unroll
-      for (int u = 0; u < DPL; ++u) o[u] = acc[i][u];
+      *reinterpret_cast<float2*>(part + (size_t)(q0 + qi) * part_stride(d) + 4 + 2 * dp) = make_float2(o0, o1);
     }
   }
+  __syncthreads();  // the area is reused by the next item
 }
 
-// Merge of one (request, kv head, query): chunks in order.  Lane c holds
-// chunk c's max and sum; the outputs are summed with all loads in flight.
+// Merge of one (request, kv head, query): chunks in order, kMergeBatch at a
+// time with all their loads in flight; lane c of a batch holds chunk c's max
+// and sum, each lane DPL output dims.  The running result is rescaled when a
+// batch raises the maximum (online softmax).
 template <int DPL>
 __device__ __noinline__ void attn_merge_warp(const AttnView& a, const StepParams* sp, int b, int hk, int qi, int lane) {
   constexpr int d = 32 * DPL;
+  constexpr int kMergeBatch = 16;
+  using VecT = typename std::conditional<DPL == 4, float4, float2>::type;
   const int L = sp->req_len[b], tok0 = sp->req_tok0[b];
   const int G = a.Hq / a.Hkv;
   const int nc = n_chunks_of(L);
-  const float* base = a.part + (((size_t)b * a.Hkv + hk) * a.n_chunks) * a.qmax * (d + 2) + (size_t)qi * (d + 2);
-  const size_t cstride = (size_t)a.qmax * (d + 2);
-  float M = -INFINITY;
-  for (int c = lane; c < nc; c += 32) M = fmaxf(M, __ldcg(base + c * cstride));
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-  float den = 0.f, num[DPL];
+  const size_t cstride = (size_t)a.qmax * part_stride(d);
+  const float* base = a.part + (((size_t)b * a.Hkv + hk) * a.n_chunks) * cstride + (size_t)qi * part_stride(d);
+  float M = -INFINITY, den = 0.f, num[DPL];
 #pragma unroll
   for (int u = 0; u < DPL; ++u) num[u] = 0.f;
-  for (int c0 = 0; c0 < nc; c0 += 32) {
-    // lane c: weight of chunk c0 + c
-    float wl = 0.f, ll = 0.f;
-    if (c0 + lane < nc) {
-      const float mc = __ldcg(base + (c0 + lane) * cstride);
-      ll = __ldcg(base + (c0 + lane) * cstride + 1);
-      wl = (mc == -INFINITY) ? 0.f : expf(mc - M);
+  for (int c0 = 0; c0 < nc; c0 += kMergeBatch) {
+    float mc = -INFINITY, lc = 0.f;
+    if (lane < kMergeBatch && c0 + lane < nc) {
+      const float2 ml = __ldcg(reinterpret_cast<const float2*>(base + (size_t)(c0 + lane) * cstride));
+      mc = ml.x;
+      lc = ml.y;
     }
-    float dl = ll * wl;
+    VecT ov[kMergeBatch];
+#pragma unroll
+    for (int u = 0; u < kMergeBatch; ++u) {
+      if (c0 + u < nc) {
+        ov[u] = __ldcg(reinterpret_cast<const VecT*>(base + (size_t)(c0 + u) * cstride + 4) + lane);
+      } else {
+        ov[u] = VecT{};
+      }
+    }
+    float bm = mc;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) bm = fmaxf(bm, __shfl_xor_sync(0xffffffffu, bm, o));
+    const float Mn = fmaxf(M, bm);
+    const float alpha = (M == -INFINITY) ? 0.f : expf(M - Mn);
+    den *= alpha;
+#pragma unroll
+    for (int u = 0; u < DPL; ++u) num[u] *= alpha;
+    const float wl = (mc == -INFINITY) ? 0.f : expf(mc - Mn);
+    float dl = lc * wl;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) dl += __shfl_xor_sync(0xffffffffu, dl, o);
     den += dl;
-    const int n = min(32, nc - c0);
-    for (int cb = 0; cb < n; cb += 8) {
-      float ov[8][DPL];
 #pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        const float* pc = base + (size_t)(c0 + cb + u) * cstride + 2 + DPL * lane;
+    for (int u = 0; u < kMergeBatch; ++u) {
+      const float w = __shfl_sync(0xffffffffu, wl, u);
+      const float* f = reinterpret_cast<const float*>(&ov[u]);
 #pragma unroll
-        for (int v = 0; v < DPL; ++v) ov[u][v] = (cb + u < n) ? __ldcg(pc + v) : 0.f;
-      }
-#pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        const float w = __shfl_sync(0xffffffffu, wl, (cb + u) & 31);
-#pragma unroll
-        for (int v = 0; v < DPL; ++v) num[v] = fmaf(ov[u][v], w, num[v]);
-      }
+      for (int v = 0; v < DPL; ++v) num[v] = fmaf(f[v], w, num[v]);
     }
+    M = Mn;
   }
   uint16_t* out = a.out + (size_t)(tok0 + qi / G) * a.out_ld + (hk * G + qi % G) * d + DPL * lane;
 #pragma unroll
@@ -470,7 +487,8 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const StepKernelArgs 
   const int gw = blockIdx.x * kWarps + warp, NW = gridDim.x * kWarps;
   uint8_t* ring = smem + (size_t)warp * kRingSlots * Geom<GPU>::kUnitBytes;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + SS::kRing) + warp * kRingSlots;
-  float* qs = reinterpret_cast<float*>(smem + SS::kRing + SS::kBars) + (size_t)warp * kQGroup * 128;
+  uint8_t* att_area = smem + SS::kRing + SS::kBars;
+  static_assert(AttnSmem<DPL>::kBytes <= SS::kQ, "attention area too small");
   OpDesc* s_ops = reinterpret_cast<OpDesc*>(smem + SS::kFixed);
   for (int i = threadIdx.x; i < 4 * a.L; i += kThreads) s_ops[i] = a.ops[i];
   __syncthreads();
@@ -537,9 +555,9 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const StepKernelArgs 
       av.out_ld = a.Kp_dq;
       int total = 0;
       for (int b = 0; b < sp->B; ++b) total += a.Hkv * n_chunks_of(sp->req_len[b]);
-      for (int item = gw; item < total; item += NW) {
+      for (int item = blockIdx.x; item < total; item += gridDim.x) {
         int b, hk, c;
-        if (decode_item(sp, a.Hkv, item, b, hk, c)) attn_partial_warp<DPL>(av, sp, b, hk, c, qs, lane);
+        if (decode_item(sp, a.Hkv, item, b, hk, c)) attn_item_cta<DPL>(av, sp, b, hk, c, att_area);
       }
       grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
       // merge items: (b, hk, query)
@@ -600,7 +618,7 @@ cudaError_t setup_t() {
 int step_barriers(int n_layers) { return 8 * n_layers; }
 
 size_t step_attention_part_floats(int B, int Hkv, int n_chunks, int G, int d) {
-  return (size_t)B * Hkv * n_chunks * (kMaxTokens * G) * (d + 2);
+  return (size_t)B * Hkv * n_chunks * (kMaxTokens * G) * part_stride(d);
 }
 
 cudaError_t step_setup(int group, int head_dim) {
