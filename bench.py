@@ -63,7 +63,6 @@ CONFIGS = {
     "tiny": dict(shape=synth.TINY, prefill=72, steps_per_request=256, rows=1, n=1, tokens=True,
                  workload="tiny 2L h256 decode: 72-token prefill, 1 token/step"),
 }
-PHASES = ["norm1", "qkv", "attention", "attention_merge", "o", "norm2", "gate_up", "down"]
 
 
 def log(*a):
@@ -363,18 +362,19 @@ def run_gpu(args, rank: int, world: int):
     prof_K = min(K, 64)
     pplan = Plan(args.config, prof_K, SEED + 2)
     pst, pd = load_states(pplan), stage(pplan)
-    n_ph = 8 * shape.n_layers
+    PHASES = list(pkg.PHASES)
+    n_ph = len(PHASES) * shape.n_layers
     acc = np.zeros(n_ph)
     for t in range(prof_K):
         run_steps_one(pplan, pst, pd, t)
         acc += np.array(pkg.shard_debug_phase_times(sh, shape.n_layers))
     acc /= prof_K
-    # times[0] is the prologue, then the eight phases of every layer (the
-    # last layer's down phase ends with the kernel, not at a barrier)
+    # times[0] is the prologue, then the phases of every layer (the last
+    # layer's down phase ends with the kernel, not at a barrier)
     phases = {"prologue": {"total_us_per_step": float(acc[0])}}
     lay = acc[1:].tolist() + [0.0]
     for i, name in enumerate(PHASES):
-        v = np.array(lay[i::8])
+        v = np.array(lay[i::len(PHASES)])
         phases[name] = {"avg_us_per_layer": float(v.mean()), "total_us_per_step": float(v.sum())}
     for name, kind in (("qkv", "qkv"), ("o", "o"), ("gate_up", "gate_up"), ("down", "down")):
         t_us = phases[name]["avg_us_per_layer"]

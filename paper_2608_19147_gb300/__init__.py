@@ -28,7 +28,7 @@ EXPORTS = ("shard_create", "shard_destroy", "kv_state_alloc", "kv_state_free", "
            "kv_state_read", "kv_state_length", "kv_trim", "shard_step", "shard_step_host", "shard_sync_status",
            "shard_last_error", "shard_debug_op_info", "shard_debug_unpack", "shard_debug_gemv",
            "shard_debug_phase_times", "shard_gemv_noalloc")
-PHASES = ("norm1", "qkv", "attention", "attention_merge", "o", "norm2", "gate_up", "down")
+PHASES = ("qkv", "attention", "attention_merge", "o", "gate_up", "down")  # qkv and gate_up include their RMSNorm
 
 
 class ShardError(RuntimeError):
@@ -227,8 +227,9 @@ def shard_debug_gemv(shard: int, layer: int, op: int, x: int, M: int, y: int, y_
 
 def shard_debug_phase_times(shard: int, n_layers: int):
     """Durations (microseconds) of the last step's phases: the prologue, then
-    per layer the eight phases named in PHASES."""
-    n = 8 * n_layers
+    per layer the phases named in PHASES (the last layer's last phase ends
+    with the kernel, not at a barrier, and is not included)."""
+    n = len(PHASES) * n_layers
     buf = (ctypes.c_double * n)()
     k = load_library().shard_debug_phase_times(shard, buf, n)
     if k < 0:

@@ -16,34 +16,41 @@ constexpr size_t smem_bytes() {
 }
 
 template <int NT, int GPU>
-__global__ void __launch_bounds__(kW * 32) gemv_kernel(const GemvArgs a) {
+__global__ void __launch_bounds__(kW * 32) gemv_kernel(const __grid_constant__ GemvArgs a) {
   extern __shared__ __align__(128) uint8_t smem[];
   __shared__ OpDesc s_op[1];
+  __shared__ GemvPhase s_gp;
+  __shared__ WarpStream<GPU> s_ws[kW];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
     s_op[0] = OpDesc{a.units, a.n_rb, a.upr};
+    GemvPhase p{};
+    p.act = a.act;
+    p.act_ld = a.act_ld;
+    p.M = a.sp ? a.sp->M : a.M;
+    p.skip = a.sp ? (a.sp->abort_step != 0) : false;
+    p.partials = a.partials;
+    p.counters = a.counters;
+    p.status = a.status;
+    p.sp = a.sp;
+    p.ep = a.ep;
+    s_gp = p;
   }
   __syncthreads();
   const size_t ring_bytes = (size_t)kW * kRingSlots * Geom<GPU>::kUnitBytes;
   uint8_t* ring = smem + (size_t)warp * kRingSlots * Geom<GPU>::kUnitBytes;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + ring_bytes) + warp * kRingSlots;
-  WarpStream<GPU> ws;
-  ws.init(s_op, 1, blockIdx.x, gridDim.x, warp, ring, bars, lane);
-  ws.fill(lane);
+  {
+    WarpStream<GPU> ws;
+    ws.init(s_op, 1, blockIdx.x, gridDim.x, warp, ring, bars, lane);
+    ws.fill(lane);
+    if (lane == 0) s_ws[warp] = ws;
+    __syncwarp();
+  }
   pdl_launch_dependents();
   pdl_wait();
-  GemvPhase p{};
-  p.act = a.act;
-  p.act_ld = a.act_ld;
-  p.M = a.sp ? a.sp->M : a.M;
-  p.skip = a.sp ? (a.sp->abort_step != 0) : false;
-  p.partials = a.partials;
-  p.counters = a.counters;
-  p.status = a.status;
-  p.sp = a.sp;
-  p.ep = a.ep;
-  gemv_phase<NT, GPU>(ws, 0, p, lane);
-  if (ws.timed_out && lane == 0) atomicOr(a.status, ST_WAIT_TIMEOUT);
+  gemv_phase<NT, GPU>(&s_ws[warp], 0, &s_gp, 0, lane);
+  if (s_ws[warp].timed_out && lane == 0) atomicOr(a.status, ST_WAIT_TIMEOUT);
 }
 
 template <int NT, int GPU>

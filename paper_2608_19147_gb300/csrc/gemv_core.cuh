@@ -84,7 +84,6 @@ struct WarpStream {
   int f_op, f_u, f_end;
   const uint8_t* f_units;
   uint32_t n_filled, n_used;
-  uint64_t policy;  // L2 evict-first: each weight byte is read once per step
   bool timed_out;
 
   // Run [wb, we) of this warp in op's unit stream.
@@ -109,7 +108,6 @@ struct WarpStream {
     ring = ring_;
     bars = bars_;
     n_filled = n_used = 0;
-    policy = l2_policy_evict_first();
     timed_out = false;
     f_op = 0;
     f_u = f_end = 0;
@@ -134,7 +132,8 @@ struct WarpStream {
         const int slot = n_filled % kRingSlots;
         fence_proxy_async_smem();
         mbar_arrive_expect_tx(&bars[slot], UB);
-        bulk_g2s_hint(ring + (size_t)slot * UB, src, UB, &bars[slot], policy);
+        // L2 evict-first: each weight byte is read once per step
+        bulk_g2s_hint(ring + (size_t)slot * UB, src, UB, &bars[slot], l2_policy_evict_first());
       }
       ++n_filled;
     }
@@ -238,9 +237,11 @@ __device__ __forceinline__ void mma_unit(const uint8_t* __restrict__ U, const ui
 __device__ __forceinline__ float silu(float v) { return v / (1.f + expf(-v)); }
 
 // Epilogue of one (row R_lo, row R_lo + 8, token m) pair of a finished
-// row-block: rotary pairs and gate/up pairs sit on these two rows.
-__device__ __forceinline__ void epilogue_pair(const EpiArgs& e, const StepParams* sp, int Rlo, int m, float vlo,
-                                              float vhi) {
+// row-block: rotary pairs and gate/up pairs sit on these two rows.  Returns
+// the sum of squares of the residual values written (EPI_RESID), else 0.
+__device__ __forceinline__ float epilogue_pair(const EpiArgs& e, const StepParams* sp, int layer, int Rlo, int m,
+                                               float vlo, float vhi) {
+  float ss = 0.f;
   const OpDims& o = e.dims;
   const int Rhi = Rlo + 8;
   switch (e.kind) {
@@ -266,7 +267,7 @@ __device__ __forceinline__ void epilogue_pair(const EpiArgs& e, const StepParams
           q[i] = olo;
           q[half + i] = ohi;
         } else {
-          uint16_t* k = e.kpool + (((size_t)prow * o.Hkv + head) * e.cap + ppos) * o.d;
+          uint16_t* k = e.kpool + (size_t)layer * e.layer_stride + (((size_t)prow * o.Hkv + head) * e.cap + ppos) * o.d;
           k[i] = f2h(olo);
           k[half + i] = f2h(ohi);
         }
@@ -278,7 +279,8 @@ __device__ __forceinline__ void epilogue_pair(const EpiArgs& e, const StepParams
         for (int u = 0; u < 2; ++u) {
           if (rv[u] < o.Hkv * o.d) {
             const int head = rv[u] / o.d, dim = rv[u] % o.d;
-            e.vpool[(((size_t)prow * o.Hkv + head) * e.cap + ppos) * o.d + dim] = f2h(vv[u]);
+            e.vpool[(size_t)layer * e.layer_stride + (((size_t)prow * o.Hkv + head) * e.cap + ppos) * o.d + dim] =
+                f2h(vv[u]);
           }
         }
       }
@@ -293,7 +295,8 @@ __device__ __forceinline__ void epilogue_pair(const EpiArgs& e, const StepParams
           float* xp = e.x + (size_t)m * o.H + rr[u];
           const float nx = __ldcg(xp) + vv[u];
           *xp = nx;
-          if (e.write_out) sp->hidden_out[(size_t)m * o.H + rr[u]] = f2h(nx);
+          ss = fmaf(nx, nx, ss);
+          if (e.out_layer == layer) sp->hidden_out[(size_t)m * o.H + rr[u]] = f2h(nx);
         }
       }
       break;
@@ -306,6 +309,7 @@ __device__ __forceinline__ void epilogue_pair(const EpiArgs& e, const StepParams
     default:
       break;
   }
+  return ss;
 }
 
 struct GemvPhase {
@@ -349,8 +353,9 @@ __device__ __forceinline__ void load_act(uint4 (&act)[NT][2][2], const uint16_t*
 // its run inside the row-block (slot 0); the first contributor used slot 1
 // if its run started before the row-block.  When T < nw some runs are empty
 // and each non-empty run is a single unit.
-static __device__ __noinline__ void finish_rowblock(const GemvPhase& p, int rb, int g_first, int g_last, int T, int nw,
-                                                    int upr, int lane) {
+static __device__ __noinline__ void finish_rowblock(const GemvPhase* pp, int layer, int rb, int g_first, int g_last,
+                                                    int T, int nw, int upr, int lane) {
+  const GemvPhase& p = *pp;
   constexpr int kBatch = 16;
   const int rb_begin = rb * upr;
   const int lo = (lane >> 3) * 16 + (lane & 7);
@@ -378,7 +383,12 @@ static __device__ __noinline__ void finish_rowblock(const GemvPhase& p, int rb, 
         vhi += b[i];
       }
     }
-    epilogue_pair(p.ep, p.sp, rb * kRowsPerBlock + lo, m, vlo, vhi);
+    float ss = epilogue_pair(p.ep, p.sp, layer, rb * kRowsPerBlock + lo, m, vlo, vhi);
+    if (p.ep.ss) {  // the row-block's sum of squares of the new residual, for the next RMSNorm
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+      if (lane == 0) p.ep.ss[rb * kMaxTokens + m] = ss;
+    }
   }
 }
 
@@ -386,8 +396,9 @@ static __device__ __noinline__ void finish_rowblock(const GemvPhase& p, int rb, 
 // 0: the run's first segment, slot 1: a later one); a whole row-block is
 // finished at once, a split one by the last of its contributing warps.
 template <int NT>
-__device__ __forceinline__ void piece_end(const GemvPhase& p, const float (&tot)[4][NT][4], int rb, bool whole, int slot,
-                                          int g, int nw, int T, int upr, int lane) {
+__device__ __forceinline__ void piece_end(const GemvPhase* pp, int layer, const float (&tot)[4][NT][4], int rb, bool whole,
+                                          int slot, int g, int nw, int T, int upr, int lane) {
+  const GemvPhase& p = *pp;
   const int gid = lane >> 2, tig = lane & 3;
   float* mine = p.partials + ((size_t)g * 2 + slot) * kPieceFloats;
 #pragma unroll
@@ -404,7 +415,7 @@ __device__ __forceinline__ void piece_end(const GemvPhase& p, const float (&tot)
       }
   __syncwarp();
   if (whole) {
-    finish_rowblock(p, rb, g, g, T, nw, upr, lane);
+    finish_rowblock(pp, layer, rb, g, g, T, nw, upr, lane);
     return;
   }
   const int rb_begin = rb * upr, rb_end = rb_begin + upr;
@@ -419,7 +430,7 @@ __device__ __forceinline__ void piece_end(const GemvPhase& p, const float (&tot)
   last = __shfl_sync(0xffffffffu, last, 0);
   if (!last) return;
   __syncwarp();
-  finish_rowblock(p, rb, g_first, g_last, T, nw, upr, lane);
+  finish_rowblock(pp, layer, rb, g_first, g_last, T, nw, upr, lane);
   if (lane == 0) p.counters[rb] = 0;
 }
 
@@ -428,11 +439,15 @@ __device__ __forceinline__ void piece_end(const GemvPhase& p, const float (&tot)
 // row-block segment of it.
 //
 // Not inlined: the step's four projections run this one copy of the code, so
-// it stays in the instruction cache.  The stream state is worked on in a
-// local copy (registers) and written back at the end.
+// it stays in the instruction cache.  The stream state and the phase
+// arguments live in shared memory (ws_io, pp): nothing crosses the call
+// through the stack, whose local memory would miss the small L1 left next to
+// the weight rings.  The stream state is worked on in registers and written
+// back at the end.
 template <int NT, int GPU>
-__device__ __noinline__ void gemv_phase(WarpStream<GPU>& ws_io, int op, const GemvPhase& p, int lane) {
-  WarpStream<GPU> ws = ws_io;
+__device__ __noinline__ void gemv_phase(WarpStream<GPU>* ws_io, int op, const GemvPhase* pp, int layer, int lane) {
+  WarpStream<GPU> ws = *ws_io;
+  const GemvPhase& p = *pp;
   int wb, we;
   ws.warp_range(op, wb, we);
   if (wb >= we) return;
@@ -472,10 +487,12 @@ __device__ __noinline__ void gemv_phase(WarpStream<GPU>& ws_io, int op, const Ge
     }
     if (!skip) {
       const bool whole = (seg_begin == rb * upr && seg_end == rb_end);
-      piece_end<NT>(p, tot, rb, whole, seg_begin == wb ? 0 : 1, g, nw, T, upr, lane);
+      piece_end<NT>(pp, layer, tot, rb, whole, seg_begin == wb ? 0 : 1, g, nw, T, upr, lane);
     }
   }
-  ws_io = ws;
+  __syncwarp();
+  if (lane == 0) *ws_io = ws;
+  __syncwarp();
 }
 
 }  // namespace shard

@@ -117,12 +117,14 @@ struct EpiArgs {
   float* y;  // EPI_STORE: y[m][natural row], row stride y_ld
   int y_ld;
   float* q;                   // EPI_QKV: q fp32 [M][Hq*d]
-  uint16_t* kpool;            // EPI_QKV: this layer's K pool [n_rows][Hkv][cap][d]
+  uint16_t* kpool;            // EPI_QKV: layer 0's K pool [n_rows][Hkv][cap][d]; layer l at + l * layer_stride
   uint16_t* vpool;
+  size_t layer_stride;
   int cap;
   const float2* rope;         // [max_position][d/2] (cos, sin)
   float* x;                   // EPI_RESID: residual [M][H]
-  int write_out;              // EPI_RESID: also write fp16(x) to sp->hidden_out
+  float* ss;                  // EPI_RESID (or nullptr): per row-block sums of squares of x [n_rb][16]
+  int out_layer;              // EPI_RESID: in this layer also write fp16(x) to sp->hidden_out (-1: never)
   uint16_t* h;                // EPI_SWIGLU: fp16 [M][h_ld]
   int h_ld;
 };
@@ -166,6 +168,7 @@ struct PrologueArgs {
   int cap, max_position, vocab, H;
   const uint16_t* embedding;
   float* x;              // residual [M][H]
+  float* ss;             // per 64-row block sums of squares of x [n_rb_H][16]
   int* status;
   StepParams* sp;
 };
@@ -185,6 +188,7 @@ struct StepKernelArgs {
   const uint16_t* norms;     // [L][2][H]
   const float2* rope;        // [max_position][d/2]
   float* x;                  // residual [16][H]
+  float* ss;                 // per 64-row block sums of squares of x [n_rb_H][16]
   uint16_t* act_h;           // [16][Kp_H]
   uint16_t* act_attn;        // [16][Kp_dq]
   uint16_t* act_f;           // [16][Kp_F]
@@ -195,11 +199,11 @@ struct StepKernelArgs {
   uint16_t* vpool;
   size_t layer_stride;
   int cap, n_chunks;         // attention items are 32 entries
-  float* attn_part;          // [B][Hkv][n_chunks][16*G][d+2]
+  float* attn_part;          // [B][Hkv][n_chunks][16*G][d+4]
   int* status;
   unsigned long long* barrier;         // grid-barrier counter (monotonic)
   unsigned long long barrier_base;     // its value when this launch starts
-  unsigned long long* phase_clock;     // [8L + 1] globaltimer at each barrier
+  unsigned long long* phase_clock;     // [step_barriers(L) + 1] globaltimer at each barrier
 };
 // One-time attribute setup of the step kernel variants for a group size and
 // head dim; number of grid barriers per step; launch (cooperative, one CTA

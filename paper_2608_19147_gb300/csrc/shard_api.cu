@@ -78,6 +78,7 @@ struct shard_s {
   float2* rope = nullptr;          // [max_position][d/2]
   // per-step work buffers (one set per shard)
   float* x = nullptr;              // [16][H]
+  float* ss = nullptr;             // [n_rb_H][16] per 64-row block sums of squares of x
   uint16_t* act_h = nullptr;       // [16][Kp_H]
   uint16_t* act_attn = nullptr;    // [16][Kp_dq]
   uint16_t* act_f = nullptr;       // [16][Kp_F]
@@ -350,6 +351,7 @@ int shard_create(const shard_config* cfg, const shard_weights_host* w, shard_t* 
 
   // Work buffers.
   CUDA_TRY(cudaMalloc(&sh->x, sizeof(float) * kMaxTokens * sh->H));
+  CUDA_TRY(cudaMalloc(&sh->ss, sizeof(float) * kMaxTokens * ((sh->H + kRowsPerBlock - 1) / kRowsPerBlock)));
   CUDA_TRY(cudaMalloc(&sh->act_h, sizeof(uint16_t) * kMaxTokens * sh->Kp_H));
   CUDA_TRY(cudaMalloc(&sh->act_attn, sizeof(uint16_t) * kMaxTokens * sh->Kp_dq));
   CUDA_TRY(cudaMalloc(&sh->act_f, sizeof(uint16_t) * kMaxTokens * sh->Kp_F));
@@ -396,6 +398,7 @@ int shard_destroy(shard_t sh) {
   cudaFree(sh->embedding);
   cudaFree(sh->rope);
   cudaFree(sh->x);
+  cudaFree(sh->ss);
   cudaFree(sh->act_h);
   cudaFree(sh->act_attn);
   cudaFree(sh->act_f);
@@ -640,6 +643,7 @@ int shard_step(shard_t sh, kvstate_t st, const uint16_t* hidden_in, const int32_
   pa.H = sh->H;
   pa.embedding = sh->embedding;
   pa.x = sh->x;
+  pa.ss = sh->ss;
   pa.status = sh->status;
   pa.sp = sh->sp;
   StepKernelArgs ka{};
@@ -658,6 +662,7 @@ int shard_step(shard_t sh, kvstate_t st, const uint16_t* hidden_in, const int32_
   ka.norms = sh->norms;
   ka.rope = sh->rope;
   ka.x = sh->x;
+  ka.ss = sh->ss;
   ka.act_h = sh->act_h;
   ka.act_attn = sh->act_attn;
   ka.act_f = sh->act_f;

@@ -2,10 +2,13 @@
 //
 // One CTA per SM, kCtaWarps warps.  The step runs as a sequence of phases separated
 // by grid-wide barriers:
-//   prologue (CTA 0) | for each layer: RMSNorm | q|k|v projection (+RoPE,
+//   prologue (CTA 0) | for each layer: RMSNorm + q|k|v projection (+RoPE,
 //   K/V append) | attention partials | attention merge | o projection
-//   (+residual) | RMSNorm | gate|up projection (+SwiGLU) | down projection
+//   (+residual) | RMSNorm + gate|up projection (+SwiGLU) | down projection
 //   (+residual; the last layer writes hidden_out).
+// Each RMSNorm is computed by every CTA at the start of the projection that
+// consumes it, from per-row-block sums of squares left by the residual's
+// producer, so it needs no barrier of its own.
 // Every warp owns a ring of weight slots (gemv_core.cuh) that streams, in
 // order, all the projection units the warp will process during the step.
 // The ring refills as soon as a slot is consumed, independent of the
@@ -47,6 +50,12 @@ __device__ __forceinline__ unsigned long long globaltimer() {
   unsigned long long t;
   asm volatile("mov.u64 %0, %globaltimer;" : "=l"(t));
   return t;
+}
+
+__device__ __forceinline__ float2 h2f2(uint32_t u) {
+  __half2 h;
+  memcpy(&h, &u, sizeof(h));
+  return __half22float2(h);
 }
 
 __device__ __forceinline__ void red_release_add(unsigned long long* p, unsigned long long v) {
@@ -146,13 +155,29 @@ __device__ __noinline__ void prologue_cta(const PrologueArgs& a) {
     a.bt_dst[(size_t)b * a.cap + s_P[b] + i] = b * a.cap + a.cursor[b] + i;
   }
   if (tid < a.B) a.lens[tid] = s_len[tid];
-  const size_t n = (size_t)a.M * a.H;
-  for (size_t e = tid; e < n; e += nth) {
-    const int m = static_cast<int>(e / a.H);
-    const size_t k = e % a.H;
-    const uint16_t h =
-        a.hidden_in ? __ldcg(a.hidden_in + e) : a.embedding[(size_t)__ldcg(a.token_ids + m) * a.H + k];
-    a.x[e] = h2f(h);
+  // residual x: warp per (token, 64-row block), which also leaves the
+  // block's sum of squares for the first RMSNorm
+  {
+    const int n_rb = (a.H + kRowsPerBlock - 1) / kRowsPerBlock;
+    const int lane = tid & 31;
+    for (int it = tid >> 5; it < a.M * n_rb; it += nth >> 5) {
+      const int m = it / n_rb, rb = it % n_rb;
+      const uint16_t* src = a.hidden_in ? a.hidden_in + (size_t)m * a.H
+                                        : a.embedding + (size_t)__ldcg(a.token_ids + m) * a.H;
+      float ss = 0.f;
+#pragma unroll
+      for (int r = 0; r < kRowsPerBlock; r += 32) {
+        const int k = rb * kRowsPerBlock + r + lane;
+        if (k < a.H) {
+          const float v = h2f(a.hidden_in ? __ldcg(src + k) : src[k]);
+          a.x[(size_t)m * a.H + k] = v;
+          ss = fmaf(v, v, ss);
+        }
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+      if (lane == 0) a.ss[rb * kMaxTokens + m] = ss;
+    }
   }
   if (tid == 0) {
     StepParams* sp = a.sp;
@@ -179,48 +204,55 @@ __device__ __noinline__ void prologue_cta(const PrologueArgs& a) {
 }
 
 // ---------------------------------------------------------------------------
-// RMSNorm: CTA m < M normalises token m (sum of squares in a fixed order).
+// RMSNorm, run by every CTA at the start of the projection that consumes it.
+// r[m] = 1 / sqrt(mean(x[m]^2) + eps) from the per-row-block sums of squares
+// that the residual's producer left (added in a fixed order, so every CTA
+// gets the same r); then act = fp16(x * r * w).  Every CTA writes the whole
+// act -- the same bits -- so its own warps can start as soon as it is done.
+// H is a multiple of 4.
 // ---------------------------------------------------------------------------
-__device__ __noinline__ void rmsnorm_cta(const float* x, int H, const uint16_t* w, float eps, uint16_t* out,
-                                         int out_ld, int M) {
-  __shared__ float s_part[kWarps];
-  __shared__ float s_r;
-  constexpr int kPer = 24;  // values per thread held in registers (H <= 24 * kThreads)
-  for (int m = blockIdx.x; m < M; m += gridDim.x) {
-    const float* xm = x + (size_t)m * H;
-    float v[kPer];
+__device__ __noinline__ void rmsnorm_cta(const float* x, int H, const uint16_t* w, float eps, const float* ss,
+                                         uint16_t* out, int out_ld, int M) {
+  __shared__ float s_r[kMaxTokens];
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int n_rb = (H + kRowsPerBlock - 1) / kRowsPerBlock;
+  for (int m = warp; m < M; m += kWarps) {
+    float t = 0.f;
+    for (int rb = lane; rb < n_rb; rb += 32) t += __ldcg(ss + rb * kMaxTokens + m);
 #pragma unroll
-    for (int i = 0; i < kPer; ++i) {
-      const int k = threadIdx.x + i * kThreads;
-      v[i] = k < H ? __ldcg(xm + k) : 0.f;
-    }
-    float ss = 0.f;
-#pragma unroll
-    for (int i = 0; i < kPer; ++i) ss = fmaf(v[i], v[i], ss);
-    for (int k = threadIdx.x + kPer * kThreads; k < H; k += kThreads) {
-      const float t = __ldcg(xm + k);
-      ss = fmaf(t, t, ss);
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
-    if ((threadIdx.x & 31) == 0) s_part[threadIdx.x >> 5] = ss;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-      float t = 0.f;
-      for (int i = 0; i < kWarps; ++i) t += s_part[i];
-      s_r = rsqrtf(t / H + eps);
-    }
-    __syncthreads();
-    const float r = s_r;
-    uint16_t* o = out + (size_t)m * out_ld;
-#pragma unroll
-    for (int i = 0; i < kPer; ++i) {
-      const int k = threadIdx.x + i * kThreads;
-      if (k < H) o[k] = f2h(v[i] * r * h2f(w[k]));
-    }
-    for (int k = threadIdx.x + kPer * kThreads; k < H; k += kThreads) o[k] = f2h(__ldcg(xm + k) * r * h2f(w[k]));
-    __syncthreads();
+    for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+    if (lane == 0) s_r[m] = rsqrtf(t / H + eps);
   }
+  __syncthreads();
+  constexpr int kBatch = 4;  // float4 pieces per thread in flight
+  const int H4 = H / 4, n4 = M * H4;
+  for (int i0 = tid; i0 < n4; i0 += kBatch * kThreads) {
+    float4 xv[kBatch];
+    uint2 wv[kBatch];
+#pragma unroll
+    for (int j = 0; j < kBatch; ++j) {
+      const int i = i0 + j * kThreads;
+      if (i < n4) {
+        xv[j] = __ldcg(reinterpret_cast<const float4*>(x) + i);
+        wv[j] = *reinterpret_cast<const uint2*>(w + 4 * (i % H4));
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < kBatch; ++j) {
+      const int i = i0 + j * kThreads;
+      if (i < n4) {
+        const int m = i / H4, k = 4 * (i % H4);
+        const float r = s_r[m];
+        const float2 w01 = h2f2(wv[j].x), w23 = h2f2(wv[j].y);
+        uint16_t* o = out + (size_t)m * out_ld + k;
+        o[0] = f2h(xv[j].x * r * w01.x);
+        o[1] = f2h(xv[j].y * r * w01.y);
+        o[2] = f2h(xv[j].z * r * w23.x);
+        o[3] = f2h(xv[j].w * r * w23.y);
+      }
+    }
+  }
+  __syncthreads();
 }
 
 // ---------------------------------------------------------------------------
@@ -235,8 +267,9 @@ __host__ __device__ constexpr int part_stride(int d) { return d + 4; }
 
 struct AttnView {
   const float* q;
-  const uint16_t* kpool;
+  const uint16_t* kpool;  // layer 0; layer l at + l * layer_stride
   const uint16_t* vpool;
+  size_t layer_stride;
   int cap, Hq, Hkv, d, n_chunks, qmax;
   float* part;
   uint16_t* out;
@@ -257,12 +290,6 @@ __device__ __forceinline__ bool decode_item(const StepParams* sp, int Hkv, int i
     item -= per;
   }
   return false;
-}
-
-__device__ __forceinline__ float2 h2f2(uint32_t u) {
-  __half2 h;
-  memcpy(&h, &u, sizeof(h));
-  return __half22float2(h);
 }
 
 // Shared-memory layout of one attention item.
@@ -286,8 +313,11 @@ struct AttnSmem {
 //      softmax pieces (max, sum of exp) per query across the lanes;
 //   4. values: thread = (query, pair of head dims), sum over the entries.
 template <int DPL>
-__device__ __noinline__ void attn_item_cta(const AttnView& a, const StepParams* sp, int b, int hk, int c,
+__device__ __noinline__ void attn_item_cta(const AttnView* ap, int layer, const StepParams* sp, int b, int hk, int c,
                                            uint8_t* area) {
+  const AttnView& a = *ap;
+  const uint16_t* kpool = a.kpool + (size_t)layer * a.layer_stride;
+  const uint16_t* vpool = a.vpool + (size_t)layer * a.layer_stride;
   using S = AttnSmem<DPL>;
   constexpr int d = S::d, KP = d / 8;  // 16-byte pieces per row
   uint16_t* Ks = reinterpret_cast<uint16_t*>(area);
@@ -331,7 +361,7 @@ __device__ __noinline__ void attn_item_cta(const AttnView& a, const StepParams* 
       if (pi < 2 * kRowPieces && r < nj) {
         const int sl = slot_s[r];
         const size_t row = (((size_t)(sl / a.cap) * a.Hkv + hk) * a.cap + sl % a.cap) * d;
-        v[i] = __ldcg(reinterpret_cast<const uint4*>((pi >= kRowPieces ? a.vpool : a.kpool) + row) + pi % KP);
+        v[i] = __ldcg(reinterpret_cast<const uint4*>((pi >= kRowPieces ? vpool : kpool) + row) + pi % KP);
       }
     }
 #pragma unroll
@@ -424,7 +454,8 @@ __device__ __noinline__ void attn_item_cta(const AttnView& a, const StepParams* 
 // and sum, each lane DPL output dims.  The running result is rescaled when a
 // batch raises the maximum (online softmax).
 template <int DPL>
-__device__ __noinline__ void attn_merge_warp(const AttnView& a, const StepParams* sp, int b, int hk, int qi, int lane) {
+__device__ __noinline__ void attn_merge_warp(const AttnView* ap, const StepParams* sp, int b, int hk, int qi, int lane) {
+  const AttnView& a = *ap;
   constexpr int d = 32 * DPL;
   constexpr int kMergeBatch = 16;
   using VecT = typename std::conditional<DPL == 4, float4, float2>::type;
@@ -480,8 +511,11 @@ __device__ __noinline__ void attn_merge_warp(const AttnView& a, const StepParams
 }
 
 template <int NT, int GPU, int DPL>
-__global__ void __launch_bounds__(kThreads, 1) step_kernel(const StepKernelArgs a) {
+__global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant__ StepKernelArgs a) {
   extern __shared__ __align__(128) uint8_t smem[];
+  __shared__ GemvPhase s_gp[4];            // per projection kind: q|k|v, o, gate|up, down
+  __shared__ WarpStream<GPU> s_ws[kWarps];  // each warp's weight stream, between phases
+  __shared__ AttnView s_av;
   using SS = StepSmem<GPU>;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int gw = blockIdx.x * kWarps + warp, NW = gridDim.x * kWarps;
@@ -495,10 +529,13 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const StepKernelArgs 
   unsigned long long target = a.barrier_base;
   int nsync = 1;
   if (threadIdx.x == 0 && blockIdx.x == 0) a.phase_clock[0] = globaltimer();
-
-  WarpStream<GPU> ws;
-  ws.init(s_ops, 4 * a.L, blockIdx.x, gridDim.x, warp, ring, bars, lane);
-  ws.fill(lane);
+  {
+    WarpStream<GPU> ws;
+    ws.init(s_ops, 4 * a.L, blockIdx.x, gridDim.x, warp, ring, bars, lane);
+    ws.fill(lane);
+    if (lane == 0) s_ws[warp] = ws;
+    __syncwarp();
+  }
 
   if (blockIdx.x == 0) prologue_cta(a.pro);
   grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
@@ -506,58 +543,64 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const StepKernelArgs 
   const StepParams* sp = a.pro.sp;
   const bool skip = __ldcg(&sp->abort_step) != 0;
   const int M = a.pro.M;
-
-  // Per-phase arguments are built where they are used (short live ranges).
-  auto gemv = [&](int op, int epi, const uint16_t* act, int act_ld, int l) {
+  if (threadIdx.x < 4) {
+    const int k = threadIdx.x;
     GemvPhase gp{};
-    gp.act = act;
-    gp.act_ld = act_ld;
+    gp.act = k == 0 || k == 2 ? a.act_h : k == 1 ? a.act_attn : a.act_f;
+    gp.act_ld = k == 0 || k == 2 ? a.Kp_H : k == 1 ? a.Kp_dq : a.Kp_F;
     gp.M = M;
     gp.skip = skip;
     gp.partials = a.partials;
     gp.counters = a.counters;
     gp.status = a.status;
     gp.sp = sp;
-    gp.ep.kind = epi;
-    gp.ep.dims = OpDims{op & 3, a.Hq, a.Hkv, a.d, a.F, a.H};
+    gp.ep.kind = k == 0 ? EPI_QKV : k == 2 ? EPI_SWIGLU : EPI_RESID;
+    gp.ep.dims = OpDims{k, a.Hq, a.Hkv, a.d, a.F, a.H};
     gp.ep.q = a.q;
-    gp.ep.kpool = a.kpool + (size_t)l * a.layer_stride;
-    gp.ep.vpool = a.vpool + (size_t)l * a.layer_stride;
+    gp.ep.kpool = a.kpool;
+    gp.ep.vpool = a.vpool;
+    gp.ep.layer_stride = a.layer_stride;
     gp.ep.cap = a.cap;
     gp.ep.rope = a.rope;
     gp.ep.x = a.x;
-    gp.ep.write_out = (op == 4 * a.L - 1) ? 1 : 0;
+    gp.ep.ss = (k == 1 || k == 3) ? a.ss : nullptr;
+    gp.ep.out_layer = k == 3 ? a.L - 1 : -1;
     gp.ep.h = a.act_f;
     gp.ep.h_ld = a.Kp_F;
-    gemv_phase<NT, GPU>(ws, op, gp, lane);
-  };
+    s_gp[k] = gp;
+  }
+  if (threadIdx.x == 32) {
+    AttnView av{};
+    av.q = a.q;
+    av.kpool = a.kpool;
+    av.vpool = a.vpool;
+    av.layer_stride = a.layer_stride;
+    av.cap = a.cap;
+    av.Hq = a.Hq;
+    av.Hkv = a.Hkv;
+    av.d = a.d;
+    av.n_chunks = a.n_chunks;
+    av.qmax = kMaxTokens * (a.Hq / a.Hkv);
+    av.part = a.attn_part;
+    av.out = a.act_attn;
+    av.out_ld = a.Kp_dq;
+    s_av = av;
+  }
+  __syncthreads();
+  auto gemv = [&](int op, int l) { gemv_phase<NT, GPU>(&s_ws[warp], op, &s_gp[op & 3], l, lane); };
 
   for (int l = 0; l < a.L; ++l) {
     const uint16_t* nrm = a.norms + (size_t)l * 2 * a.H;
     // attention block
-    if (!skip) rmsnorm_cta(a.x, a.H, nrm, a.eps, a.act_h, a.Kp_H, M);
-    grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
-    gemv(4 * l + 0, EPI_QKV, a.act_h, a.Kp_H, l);
+    if (!skip) rmsnorm_cta(a.x, a.H, nrm, a.eps, a.ss, a.act_h, a.Kp_H, M);
+    gemv(4 * l + 0, l);
     grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
     if (!skip) {
-      AttnView av{};
-      av.q = a.q;
-      av.kpool = a.kpool + (size_t)l * a.layer_stride;
-      av.vpool = a.vpool + (size_t)l * a.layer_stride;
-      av.cap = a.cap;
-      av.Hq = a.Hq;
-      av.Hkv = a.Hkv;
-      av.d = a.d;
-      av.n_chunks = a.n_chunks;
-      av.qmax = kMaxTokens * (a.Hq / a.Hkv);
-      av.part = a.attn_part;
-      av.out = a.act_attn;
-      av.out_ld = a.Kp_dq;
       int total = 0;
       for (int b = 0; b < sp->B; ++b) total += a.Hkv * n_chunks_of(sp->req_len[b]);
       for (int item = blockIdx.x; item < total; item += gridDim.x) {
         int b, hk, c;
-        if (decode_item(sp, a.Hkv, item, b, hk, c)) attn_item_cta<DPL>(av, sp, b, hk, c, att_area);
+        if (decode_item(sp, a.Hkv, item, b, hk, c)) attn_item_cta<DPL>(&s_av, l, sp, b, hk, c, att_area);
       }
       grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
       // merge items: (b, hk, query)
@@ -572,23 +615,22 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const StepKernelArgs 
           r -= per;
         }
         const int Qb = (sp->req_tok0[b + 1] - sp->req_tok0[b]) * G;
-        attn_merge_warp<DPL>(av, sp, b, r / Qb, r % Qb, lane);
+        attn_merge_warp<DPL>(&s_av, sp, b, r / Qb, r % Qb, lane);
       }
     } else {
       grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
     }
     grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
-    gemv(4 * l + 1, EPI_RESID, a.act_attn, a.Kp_dq, l);
+    gemv(4 * l + 1, l);
     grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
     // MLP block
-    if (!skip) rmsnorm_cta(a.x, a.H, nrm + a.H, a.eps, a.act_h, a.Kp_H, M);
+    if (!skip) rmsnorm_cta(a.x, a.H, nrm + a.H, a.eps, a.ss, a.act_h, a.Kp_H, M);
+    gemv(4 * l + 2, l);
     grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
-    gemv(4 * l + 2, EPI_SWIGLU, a.act_h, a.Kp_H, l);
-    grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
-    gemv(4 * l + 3, EPI_RESID, a.act_f, a.Kp_F, l);
+    gemv(4 * l + 3, l);
     if (l + 1 < a.L) grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
   }
-  if (ws.timed_out && lane == 0) atomicOr(a.status, ST_WAIT_TIMEOUT);
+  if (s_ws[warp].timed_out && lane == 0) atomicOr(a.status, ST_WAIT_TIMEOUT);
 }
 
 template <int NT, int GPU, int DPL>
@@ -615,7 +657,7 @@ cudaError_t setup_t() {
 
 }  // namespace
 
-int step_barriers(int n_layers) { return 8 * n_layers; }
+int step_barriers(int n_layers) { return 6 * n_layers; }
 
 size_t step_attention_part_floats(int B, int Hkv, int n_chunks, int G, int d) {
   return (size_t)B * Hkv * n_chunks * (kMaxTokens * G) * part_stride(d);
