@@ -30,7 +30,7 @@ __global__ void __launch_bounds__(kW * 32) gemv_kernel(const __grid_constant__ G
     p.M = a.sp ? a.sp->M : a.M;
     p.skip = a.sp ? (a.sp->abort_step != 0) : false;
     p.partials = a.partials;
-    p.counters = a.counters;
+    p.flags = a.flags;
     p.status = a.status;
     p.sp = a.sp;
     p.ep = a.ep;
@@ -49,7 +49,7 @@ __global__ void __launch_bounds__(kW * 32) gemv_kernel(const __grid_constant__ G
   }
   pdl_launch_dependents();
   pdl_wait();
-  gemv_phase<NT, GPU>(&s_ws[warp], 0, &s_gp, 0, lane);
+  gemv_phase<NT, GPU>(&s_ws[warp], 0, &s_gp, 0, a.epoch, lane);
   if (s_ws[warp].timed_out && lane == 0) atomicOr(a.status, ST_WAIT_TIMEOUT);
 }
 
@@ -94,6 +94,8 @@ int gemv_grid(int nt, int num_sms) {
 int gemv_warps_per_cta() { return kW; }
 
 size_t gemv_partials_floats(int grid) { return (size_t)grid * kW * 2 * kPieceFloats; }
+
+size_t gemv_flags_count(int grid) { return (size_t)grid * kW * 2; }
 
 cudaError_t launch_gemv(const GemvArgs& a, int nt, int group, int grid, cudaStream_t s, bool pdl) {
   if (nt == 1) {

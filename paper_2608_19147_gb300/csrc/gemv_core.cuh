@@ -19,11 +19,13 @@
 // the fp16 group scale multiplies the fp32 group sum.
 //
 // Reduction.  A row-block lying wholly inside one warp's run is finished by
-// that warp (epilogue straight from the accumulator registers).  A row-block
-// split between warps gets one piece per warp, stored in the accumulator
-// fragment layout; the last warp to arrive (global counter, acquire-release)
-// adds the pieces in warp order and runs the epilogue.  No warp ever waits
-// for another inside a projection, and the fixed order makes results
+// that warp.  A row-block split between warps gets one piece per warp; each
+// contributor stores its piece and publishes it with a release-store of the
+// launch's epoch into its flag, never waiting.  The warp that owns the
+// row-block's last unit, after its own run, waits (acquire loads, all
+// contributors polled at once, bounded) for the other flags, adds the pieces
+// in warp order and runs the epilogue.  Waits only ever point to lower warp
+// indices, so they cannot form a cycle; the fixed order makes results
 // deterministic and independent of the token count M.
 #pragma once
 #include "common.cuh"
@@ -68,6 +70,14 @@ __device__ __forceinline__ int atom_add_acq_rel(int* p, int v) {
   int old;
   asm volatile("atom.add.acq_rel.gpu.global.s32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
   return old;
+}
+__device__ __forceinline__ void st_release_u32(unsigned* p, unsigned v) {
+  asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ unsigned ld_acquire_u32(const unsigned* p) {
+  unsigned v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
 }
 
 // ---------------------------------------------------------------------------
@@ -239,8 +249,9 @@ __device__ __forceinline__ float silu(float v) { return v / (1.f + expf(-v)); }
 // Epilogue of one (row R_lo, row R_lo + 8, token m) pair of a finished
 // row-block: rotary pairs and gate/up pairs sit on these two rows.  Returns
 // the sum of squares of the residual values written (EPI_RESID), else 0.
+// xlo, xhi: the residual's current values at the two rows (EPI_RESID).
 __device__ __forceinline__ float epilogue_pair(const EpiArgs& e, const StepParams* sp, int layer, int Rlo, int m,
-                                               float vlo, float vhi) {
+                                               float vlo, float vhi, float xlo, float xhi) {
   float ss = 0.f;
   const OpDims& o = e.dims;
   const int Rhi = Rlo + 8;
@@ -288,12 +299,12 @@ __device__ __forceinline__ float epilogue_pair(const EpiArgs& e, const StepParam
     }
     case EPI_RESID: {
       const int rr[2] = {Rlo, Rhi};
-      const float vv[2] = {vlo, vhi};
+      const float vv[2] = {vlo, vhi}, xv[2] = {xlo, xhi};
 #pragma unroll
       for (int u = 0; u < 2; ++u) {
         if (rr[u] < o.H) {
           float* xp = e.x + (size_t)m * o.H + rr[u];
-          const float nx = __ldcg(xp) + vv[u];
+          const float nx = xv[u] + vv[u];
           *xp = nx;
           ss = fmaf(nx, nx, ss);
           if (e.out_layer == layer) sp->hidden_out[(size_t)m * o.H + rr[u]] = f2h(nx);
@@ -317,7 +328,7 @@ struct GemvPhase {
   int act_ld, M;
   bool skip;            // consume the weights but compute nothing (aborted step)
   float* partials;      // [n_cta * kCtaWarps][2][kPieceFloats] pieces of split row-blocks
-  int* counters;        // [n_rb], zero, self-resetting
+  unsigned* flags;      // [n_cta * kCtaWarps][2] epoch of the piece last published in each slot
   int* status;
   const StepParams* sp;
   EpiArgs ep;
@@ -345,9 +356,12 @@ __device__ __forceinline__ void load_act(uint4 (&act)[NT][2][2], const uint16_t*
 }
 
 // Finishes row-block rb from the stored pieces of warps g_first..g_last (the
-// cold path): for each token, adds the pieces in warp order, then runs the
-// epilogue.  Lane L takes the row pair lo = (L / 8) * 16 + L % 8 and lo + 8 --
-// a rotary or gate/up pair.  The loads of kBatch pieces are in flight at once.
+// cold path), then runs the epilogue.  Lane L = rg + 8 * pg loads, as
+// float4s, the four row pairs (R0 + i, R0 + 8 + i), R0 = 16 * (rg / 2) +
+// 4 * (rg % 2), of the pieces g_first + pg, + pg + 4, ... and adds them in
+// that order; two butterfly levels over pg then give every lane of the row
+// group the same totals, and lane L finishes the pair R0 + pg (a rotary or
+// gate/up pair).  The order is fixed, so the result is deterministic.
 //
 // Which slot holds a warp's piece: every contributor after the first started
 // its run inside the row-block (slot 0); the first contributor used slot 1
@@ -356,34 +370,55 @@ __device__ __forceinline__ void load_act(uint4 (&act)[NT][2][2], const uint16_t*
 static __device__ __noinline__ void finish_rowblock(const GemvPhase* pp, int layer, int rb, int g_first, int g_last,
                                                     int T, int nw, int upr, int lane) {
   const GemvPhase& p = *pp;
-  constexpr int kBatch = 16;
+  constexpr int kPerLane = 8;  // pieces per lane and batch (32 per batch over the 4 piece groups)
   const int rb_begin = rb * upr;
-  const int lo = (lane >> 3) * 16 + (lane & 7);
+  const int rg = lane & 7, pg = lane >> 3;
+  const int R0 = 16 * (rg >> 1) + 4 * (rg & 1);
+  const int R = rb * kRowsPerBlock + R0 + pg;
   const bool dense = T >= nw;
   const size_t first_off = ((size_t)g_first * 2 + (part_start(T, g_first, nw) < rb_begin ? 1 : 0)) * kPieceFloats;
   for (int m = 0; m < p.M; ++m) {
-    float vlo = 0.f, vhi = 0.f;
-    for (int g0 = g_first; g0 <= g_last; g0 += kBatch) {
-      float a[kBatch], b[kBatch];
+    // the residual's current values, loaded with the pieces
+    float xlo = 0.f, xhi = 0.f;
+    if (p.ep.kind == EPI_RESID) {
+      if (R < p.ep.dims.H) xlo = __ldcg(p.ep.x + (size_t)m * p.ep.dims.H + R);
+      if (R + 8 < p.ep.dims.H) xhi = __ldcg(p.ep.x + (size_t)m * p.ep.dims.H + R + 8);
+    }
+    float4 slo = make_float4(0.f, 0.f, 0.f, 0.f), shi = slo;
+    for (int g0 = g_first + pg; g0 <= g_last; g0 += 4 * kPerLane) {
+      float4 a[kPerLane], b[kPerLane];
 #pragma unroll
-      for (int i = 0; i < kBatch; ++i) {
-        const int gg = g0 + i;
-        a[i] = b[i] = 0.f;
+      for (int i = 0; i < kPerLane; ++i) {
+        const int gg = g0 + 4 * i;
+        a[i] = b[i] = make_float4(0.f, 0.f, 0.f, 0.f);
         bool live = gg <= g_last;
         if (live && !dense) live = part_start(T, gg + 1, nw) > part_start(T, gg, nw);
         if (live) {
           const float* pc = p.partials + (gg == g_first ? first_off : (size_t)gg * 2 * kPieceFloats) + m * kRowsPerBlock;
-          a[i] = __ldcg(pc + lo);
-          b[i] = __ldcg(pc + lo + 8);
+          a[i] = __ldcg(reinterpret_cast<const float4*>(pc + R0));
+          b[i] = __ldcg(reinterpret_cast<const float4*>(pc + R0 + 8));
         }
       }
 #pragma unroll
-      for (int i = 0; i < kBatch; ++i) {
-        vlo += a[i];
-        vhi += b[i];
+      for (int i = 0; i < kPerLane; ++i) {
+        slo.x += a[i].x; slo.y += a[i].y; slo.z += a[i].z; slo.w += a[i].w;
+        shi.x += b[i].x; shi.y += b[i].y; shi.z += b[i].z; shi.w += b[i].w;
       }
     }
-    float ss = epilogue_pair(p.ep, p.sp, layer, rb * kRowsPerBlock + lo, m, vlo, vhi);
+#pragma unroll
+    for (int o = 8; o <= 16; o <<= 1) {
+      slo.x += __shfl_xor_sync(0xffffffffu, slo.x, o);
+      slo.y += __shfl_xor_sync(0xffffffffu, slo.y, o);
+      slo.z += __shfl_xor_sync(0xffffffffu, slo.z, o);
+      slo.w += __shfl_xor_sync(0xffffffffu, slo.w, o);
+      shi.x += __shfl_xor_sync(0xffffffffu, shi.x, o);
+      shi.y += __shfl_xor_sync(0xffffffffu, shi.y, o);
+      shi.z += __shfl_xor_sync(0xffffffffu, shi.z, o);
+      shi.w += __shfl_xor_sync(0xffffffffu, shi.w, o);
+    }
+    const float vlo = pg == 0 ? slo.x : pg == 1 ? slo.y : pg == 2 ? slo.z : slo.w;
+    const float vhi = pg == 0 ? shi.x : pg == 1 ? shi.y : pg == 2 ? shi.z : shi.w;
+    float ss = epilogue_pair(p.ep, p.sp, layer, R, m, vlo, vhi, xlo, xhi);
     if (p.ep.ss) {  // the row-block's sum of squares of the new residual, for the next RMSNorm
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
@@ -392,12 +427,43 @@ static __device__ __noinline__ void finish_rowblock(const GemvPhase* pp, int lay
   }
 }
 
-// End of one row-block segment of a warp's run.  The piece is stored (slot
-// 0: the run's first segment, slot 1: a later one); a whole row-block is
-// finished at once, a split one by the last of its contributing warps.
+// Merge of split row-block rb by the warp owning its last unit: wait until
+// every other contributor (g_first .. g_last - 1, non-empty runs) has
+// published its piece for this epoch, then finish the row-block.
+static __device__ __noinline__ void merge_rowblock(const GemvPhase* pp, int layer, int rb, int g_first, int g_last,
+                                                   int T, int nw, int upr, unsigned epoch, int lane) {
+  const GemvPhase& p = *pp;
+  const int rb_begin = rb * upr;
+  for (int g0 = g_first; g0 < g_last; g0 += 32) {
+    const int gg = g0 + lane;
+    if (gg < g_last) {
+      const int s0 = part_start(T, gg, nw);
+      if (part_start(T, gg + 1, nw) > s0) {  // non-empty run
+        const unsigned* f = p.flags + (size_t)gg * 2 + (gg == g_first && s0 < rb_begin ? 1 : 0);
+        uint32_t it = 0;
+        while (ld_acquire_u32(f) != epoch) {
+          if (++it > (1u << 22)) {
+            atomicOr(p.status, ST_WAIT_TIMEOUT);
+            break;
+          }
+          __nanosleep(32);
+        }
+      }
+    }
+  }
+  __syncwarp();
+  finish_rowblock(pp, layer, rb, g_first, g_last, T, nw, upr, lane);
+}
+
+// End of one row-block segment of a warp's run: store the piece (slot 0:
+// the run's first segment, slot 1: a later one) and publish it.  A whole
+// row-block is finished at once; a split one is merged by the owner of its
+// last unit after that warp's run (gemv_phase) -- the owner itself (owner
+// set) publishes nothing.
 template <int NT>
 __device__ __forceinline__ void piece_end(const GemvPhase* pp, int layer, const float (&tot)[4][NT][4], int rb, bool whole,
-                                          int slot, int g, int nw, int T, int upr, int lane) {
+                                          bool owner, int slot, int g, int nw, int T, int upr, unsigned epoch,
+                                          int lane) {
   const GemvPhase& p = *pp;
   const int gid = lane >> 2, tig = lane & 3;
   float* mine = p.partials + ((size_t)g * 2 + slot) * kPieceFloats;
@@ -418,20 +484,9 @@ __device__ __forceinline__ void piece_end(const GemvPhase* pp, int layer, const 
     finish_rowblock(pp, layer, rb, g, g, T, nw, upr, lane);
     return;
   }
-  const int rb_begin = rb * upr, rb_end = rb_begin + upr;
-  const int g_first = part_of(T, rb_begin, nw), g_last = part_of(T, rb_end - 1, nw);
-  // with T < nw every non-empty run holds one unit
-  const int expected = (T >= nw) ? (g_last - g_first + 1) : upr;
   // The warp barrier above orders every lane's piece stores before lane 0's
-  // release; lane 0's acquire is ordered before the merge loads by the warp
-  // barrier below.
-  int last = 0;
-  if (lane == 0) last = (atom_add_acq_rel(&p.counters[rb], 1) == expected - 1);
-  last = __shfl_sync(0xffffffffu, last, 0);
-  if (!last) return;
-  __syncwarp();
-  finish_rowblock(pp, layer, rb, g_first, g_last, T, nw, upr, lane);
-  if (lane == 0) p.counters[rb] = 0;
+  // release; the merging warp's acquire loads pair with it.
+  if (!owner && lane == 0) st_release_u32(p.flags + (size_t)g * 2 + slot, epoch);
 }
 
 // One projection for one warp: consume the warp's run of units from the
@@ -445,7 +500,8 @@ __device__ __forceinline__ void piece_end(const GemvPhase* pp, int layer, const 
 // the weight rings.  The stream state is worked on in registers and written
 // back at the end.
 template <int NT, int GPU>
-__device__ __noinline__ void gemv_phase(WarpStream<GPU>* ws_io, int op, const GemvPhase* pp, int layer, int lane) {
+__device__ __noinline__ void gemv_phase(WarpStream<GPU>* ws_io, int op, const GemvPhase* pp, int layer, unsigned epoch,
+                                        int lane) {
   WarpStream<GPU> ws = *ws_io;
   const GemvPhase& p = *pp;
   int wb, we;
@@ -487,12 +543,20 @@ __device__ __noinline__ void gemv_phase(WarpStream<GPU>* ws_io, int op, const Ge
     }
     if (!skip) {
       const bool whole = (seg_begin == rb * upr && seg_end == rb_end);
-      piece_end<NT>(pp, layer, tot, rb, whole, seg_begin == wb ? 0 : 1, g, nw, T, upr, lane);
+      piece_end<NT>(pp, layer, tot, rb, whole, seg_end == rb_end, seg_begin == wb ? 0 : 1, g, nw, T, upr, epoch,
+                    lane);
     }
   }
   __syncwarp();
   if (lane == 0) *ws_io = ws;
   __syncwarp();
+  if (!skip) {
+    // merge the split row-blocks whose last unit is this warp's
+    for (int r = wb / upr; r * upr + upr <= we; ++r) {
+      if (r * upr >= wb) continue;  // whole inside the run: already finished
+      merge_rowblock(pp, layer, r, part_of(T, r * upr, nw), g, T, nw, upr, epoch, lane);
+    }
+  }
 }
 
 }  // namespace shard

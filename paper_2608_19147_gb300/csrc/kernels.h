@@ -137,7 +137,8 @@ struct GemvArgs {
   int M;                // tokens when sp == nullptr
   const StepParams* sp; // step parameters (nullptr on the standalone path)
   float* partials;      // [grid warps][2][piece] fp32 scratch, gemv_partials_floats(grid)
-  int* counters;        // [n_rb] zero-initialised, self-resetting
+  unsigned* flags;      // [grid warps][2] piece flags (gemv_flags_count(grid)), zero-initialised
+  unsigned epoch;       // nonzero, different from every earlier launch on these flags
   int* status;
   EpiArgs ep;
 };
@@ -146,6 +147,7 @@ struct GemvArgs {
 // nt = 2: M <= 16).
 int gemv_grid(int nt, int num_sms);
 size_t gemv_partials_floats(int grid);
+size_t gemv_flags_count(int grid);
 cudaError_t launch_gemv(const GemvArgs& a, int nt, int group, int grid, cudaStream_t s, bool pdl);
 // One-time per-device kernel attribute setup (dynamic shared memory limits).
 cudaError_t gemv_setup();
@@ -194,12 +196,14 @@ struct StepKernelArgs {
   uint16_t* act_f;           // [16][Kp_F]
   float* q;                  // [16][Hq*d]
   float* partials;           // projection pieces, gemv_partials_floats(grid)
-  int* counters;             // [max row-blocks]
+  unsigned* flags;           // projection piece flags, gemv_flags_count(grid), zero-initialised
+  unsigned epoch_base;       // projection op of this launch publishes epoch_base + op (unique per launch)
   uint16_t* kpool;           // [L][n_rows][Hkv][cap][d]
   uint16_t* vpool;
   size_t layer_stride;
   int cap, n_chunks;         // attention items are 32 entries
   float* attn_part;          // [B][Hkv][n_chunks][16*G][d+4]
+  int* attn_cnt;             // [16][Hkv] finished chunks per (request, kv head); zero, self-resetting
   int* status;
   unsigned long long* barrier;         // grid-barrier counter (monotonic)
   unsigned long long barrier_base;     // its value when this launch starts

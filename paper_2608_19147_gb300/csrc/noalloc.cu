@@ -7,9 +7,10 @@
 // running while another thread holds the allocator, or a latency-critical
 // loop where an allocation's implicit device synchronisation is not
 // allowed.  Such a caller still owns its inputs and outputs; only the
-// kernel's scratch (the cross-CTA partial sums, the per-row-block arrival
-// counters and a zero-padded copy of the activations) moves into the static
-// array below, which every GPU that loads the library holds until exit.
+// kernel's scratch (the partial sums of split row-blocks, the flags that
+// publish them and a zero-padded copy of the activations) moves into the
+// static array below, which every GPU that loads the library holds until
+// exit.
 #include <algorithm>
 #include <cstdio>
 
@@ -20,14 +21,18 @@
 namespace shard {
 namespace {
 
-// 4 MiB: the padded activations (16 rows of up to 28672 inputs: 896 KiB), the
-// row-block counters (4 KiB for 1024 row-blocks) and the cross-CTA partial
-// sums of as many CTAs as fit in the rest (8 KiB per CTA).
+// 4 MiB: at a fixed offset the piece flags of up to kMaxGrid CTAs and a
+// status word, then the partial sums of as many CTAs as fit next to the
+// padded activations (16 rows of up to 28672 inputs: 896 KiB).  The flags
+// only ever hold epochs, which are unique per device, so they need no
+// clearing between calls.
 constexpr size_t kNoAllocScratchBytes = 4u << 20;
+constexpr int kMaxGrid = 256;
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 
 constexpr int kMaxDevices = 64;
 void* g_scratch_addr[kMaxDevices] = {};  // per-device address of g_noalloc_scratch
+unsigned g_epoch[kMaxDevices] = {};      // per-device last epoch used
 
 }  // namespace
 
@@ -62,21 +67,23 @@ int shard_gemv_noalloc(shard_t sh, int layer, int op, const uint16_t* x, int M, 
   }
   const PackedOp& p = *v.op;
   const int nt = M <= 8 ? 1 : 2;
-  // Scratch layout: [partials | counters | activations], 256-byte aligned
-  // parts.  The grid shrinks until its partials fit next to the rest.
-  const size_t cnt_bytes = ((size_t)(p.n_rb + 1) * sizeof(int) + 255) / 256 * 256;  // counters + status word
+  // Scratch layout: [flags + status word | partials | activations],
+  // 256-byte aligned parts.  The grid shrinks until its partials fit.
+  const size_t flag_bytes = ((gemv_flags_count(kMaxGrid) + 1) * sizeof(unsigned) + 255) / 256 * 256;
   const size_t act_bytes = (size_t)M * p.Kp * sizeof(uint16_t);
   const size_t per_cta = gemv_partials_floats(1) * sizeof(float);
   long long fit = 0;
-  if (cnt_bytes + act_bytes < kNoAllocScratchBytes) fit = (long long)((kNoAllocScratchBytes - cnt_bytes - act_bytes) / per_cta);
-  const int grid = static_cast<int>(std::min<long long>(std::min<long long>(nt == 1 ? v.grid_nt1 : v.grid_nt2, fit),
-                                                        (long long)p.n_rb * p.upr));
+  if (flag_bytes + act_bytes < kNoAllocScratchBytes)
+    fit = (long long)((kNoAllocScratchBytes - flag_bytes - act_bytes) / per_cta);
+  const int grid = static_cast<int>(std::min<long long>(
+      std::min<long long>(std::min<long long>(nt == 1 ? v.grid_nt1 : v.grid_nt2, kMaxGrid), fit),
+      (long long)p.n_rb * p.upr));
   const size_t part_bytes = (gemv_partials_floats(grid > 0 ? grid : 0) * sizeof(float) + 255) / 256 * 256;
-  if (grid < 1 || part_bytes + cnt_bytes + act_bytes > kNoAllocScratchBytes) {
+  if (grid < 1 || flag_bytes + part_bytes + act_bytes > kNoAllocScratchBytes) {
     snprintf(g_msg, sizeof(g_msg),
-             "shard_gemv_noalloc: needs %zu bytes of scratch for M=%d, K=%d and %d row-blocks plus %zu per CTA; "
+             "shard_gemv_noalloc: needs %zu bytes of scratch for M=%d and K=%d plus %zu per CTA; "
              "the fixed array has %zu",
-             cnt_bytes + act_bytes, M, p.K, p.n_rb, per_cta, kNoAllocScratchBytes);
+             flag_bytes + act_bytes, M, p.K, per_cta, kNoAllocScratchBytes);
     return shard_noalloc_fail(SHARD_ECAPACITY, g_msg);
   }
   if (y_ld < v.rows) {
@@ -100,13 +107,19 @@ int shard_gemv_noalloc(shard_t sh, int layer, int op, const uint16_t* x, int M, 
     g_scratch_addr[v.device] = ptr;
   }
   unsigned char* base = static_cast<unsigned char*>(g_scratch_addr[v.device]);
-  float* partials = reinterpret_cast<float*>(base);
-  int* counters = reinterpret_cast<int*>(base + part_bytes);
-  uint16_t* act = reinterpret_cast<uint16_t*>(base + part_bytes + cnt_bytes);
+  unsigned* flags = reinterpret_cast<unsigned*>(base);
+  int* status = reinterpret_cast<int*>(flags + gemv_flags_count(kMaxGrid));
+  float* partials = reinterpret_cast<float*>(base + flag_bytes);
+  uint16_t* act = reinterpret_cast<uint16_t*>(base + flag_bytes + part_bytes);
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
-  // The array keeps the previous call's contents: zero the arrival counters
-  // and the activation padding; partial sums are written before being read.
-  e = cudaMemsetAsync(counters, 0, cnt_bytes, s);
+  // The array keeps the previous call's contents: zero the status word and
+  // the activation padding; partial sums are written before being read.
+  if (g_epoch[v.device] == 0xFFFFFFFFu) {  // wrap-around: clear the flags first
+    e = cudaMemsetAsync(flags, 0, flag_bytes, s);
+    g_epoch[v.device] = 0;
+  }
+  const unsigned epoch = ++g_epoch[v.device];
+  if (e == cudaSuccess) e = cudaMemsetAsync(status, 0, sizeof(int), s);
   if (e == cudaSuccess) e = cudaMemsetAsync(act, 0, act_bytes, s);
   if (e == cudaSuccess)
     e = cudaMemcpy2DAsync(act, sizeof(uint16_t) * p.Kp, x, sizeof(uint16_t) * p.K, sizeof(uint16_t) * p.K, M,
@@ -124,8 +137,9 @@ int shard_gemv_noalloc(shard_t sh, int layer, int op, const uint16_t* x, int M, 
   g.M = M;
   g.sp = nullptr;
   g.partials = partials;
-  g.counters = counters;
-  g.status = counters + p.n_rb;
+  g.flags = flags;
+  g.epoch = epoch;
+  g.status = status;
   g.ep.kind = EPI_STORE;
   g.ep.dims = p.dims;
   g.ep.y = y;

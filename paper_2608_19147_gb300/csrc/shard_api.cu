@@ -79,12 +79,14 @@ struct shard_s {
   // per-step work buffers (one set per shard)
   float* x = nullptr;              // [16][H]
   float* ss = nullptr;             // [n_rb_H][16] per 64-row block sums of squares of x
+  int* attn_cnt = nullptr;         // [16][Hkv] attention chunks finished per (request, kv head)
   uint16_t* act_h = nullptr;       // [16][Kp_H]
   uint16_t* act_attn = nullptr;    // [16][Kp_dq]
   uint16_t* act_f = nullptr;       // [16][Kp_F]
   float* q = nullptr;              // [16][dq]
   float* partials = nullptr;
-  int* counters = nullptr;
+  unsigned* flags = nullptr;        // projection piece flags
+  unsigned epoch = 1;               // next epoch for the flags
   int max_rb = 0;
   int* status = nullptr;           // device status word
   int* status_host = nullptr;      // pinned mirror (copied after each step)
@@ -179,6 +181,20 @@ int op_K(int kind, const shard_s& s) {
 }
 
 int nt_for(int M) { return M <= 8 ? 1 : 2; }
+
+// Reserves n consecutive flag epochs (never 0).  On wrap-around (after 2^32
+// epochs) the flags are cleared first, so no stale flag can match.
+unsigned next_epochs(shard_s* sh, unsigned n) {
+  if (sh->epoch > 0xFFFFFFFFu - n) {
+    cudaDeviceSynchronize();
+    cudaMemset(sh->flags, 0, sizeof(unsigned) * gemv_flags_count(std::max(std::max(sh->grid[1], sh->grid[2]), sh->num_sms)));
+    cudaDeviceSynchronize();
+    sh->epoch = 1;
+  }
+  const unsigned e = sh->epoch;
+  sh->epoch += n;
+  return e;
+}
 
 int check_pending_status(shard_s* sh) {
   const int bits = *reinterpret_cast<volatile int*>(sh->status_host);
@@ -352,6 +368,8 @@ int shard_create(const shard_config* cfg, const shard_weights_host* w, shard_t* 
   // Work buffers.
   CUDA_TRY(cudaMalloc(&sh->x, sizeof(float) * kMaxTokens * sh->H));
   CUDA_TRY(cudaMalloc(&sh->ss, sizeof(float) * kMaxTokens * ((sh->H + kRowsPerBlock - 1) / kRowsPerBlock)));
+  CUDA_TRY(cudaMalloc(&sh->attn_cnt, sizeof(int) * kMaxRequests * sh->Hkv));
+  CUDA_TRY(cudaMemset(sh->attn_cnt, 0, sizeof(int) * kMaxRequests * sh->Hkv));
   CUDA_TRY(cudaMalloc(&sh->act_h, sizeof(uint16_t) * kMaxTokens * sh->Kp_H));
   CUDA_TRY(cudaMalloc(&sh->act_attn, sizeof(uint16_t) * kMaxTokens * sh->Kp_dq));
   CUDA_TRY(cudaMalloc(&sh->act_f, sizeof(uint16_t) * kMaxTokens * sh->Kp_F));
@@ -364,8 +382,11 @@ int shard_create(const shard_config* cfg, const shard_weights_host* w, shard_t* 
     const size_t n = gemv_partials_floats(std::max(std::max(sh->grid[1], sh->grid[2]), sh->num_sms));
     CUDA_TRY(cudaMalloc(&sh->partials, sizeof(float) * n));
   }
-  CUDA_TRY(cudaMalloc(&sh->counters, sizeof(int) * sh->max_rb));
-  CUDA_TRY(cudaMemset(sh->counters, 0, sizeof(int) * sh->max_rb));
+  {
+    const size_t nf = gemv_flags_count(std::max(std::max(sh->grid[1], sh->grid[2]), sh->num_sms));
+    CUDA_TRY(cudaMalloc(&sh->flags, sizeof(unsigned) * nf));
+    CUDA_TRY(cudaMemset(sh->flags, 0, sizeof(unsigned) * nf));
+  }
   CUDA_TRY(cudaMalloc(&sh->status, sizeof(int)));
   CUDA_TRY(cudaMemset(sh->status, 0, sizeof(int)));
   CUDA_TRY(cudaHostAlloc(&sh->status_host, sizeof(int), cudaHostAllocDefault));
@@ -399,12 +420,13 @@ int shard_destroy(shard_t sh) {
   cudaFree(sh->rope);
   cudaFree(sh->x);
   cudaFree(sh->ss);
+  cudaFree(sh->attn_cnt);
   cudaFree(sh->act_h);
   cudaFree(sh->act_attn);
   cudaFree(sh->act_f);
   cudaFree(sh->q);
   cudaFree(sh->partials);
-  cudaFree(sh->counters);
+  cudaFree(sh->flags);
   cudaFree(sh->status);
   cudaFree(sh->sp);
   cudaFree(sh->dstage);
@@ -668,13 +690,15 @@ int shard_step(shard_t sh, kvstate_t st, const uint16_t* hidden_in, const int32_
   ka.act_f = sh->act_f;
   ka.q = sh->q;
   ka.partials = sh->partials;
-  ka.counters = sh->counters;
+  ka.flags = sh->flags;
+  ka.epoch_base = next_epochs(sh, 4 * sh->L);
   ka.kpool = st->k;
   ka.vpool = st->v;
   ka.layer_stride = st->layer_stride;
   ka.cap = st->cap;
   ka.n_chunks = st->n_chunks;
   ka.attn_part = st->attn_part;
+  ka.attn_cnt = sh->attn_cnt;
   ka.status = sh->status;
   ka.barrier = sh->barrier;
   ka.barrier_base = sh->barrier_base;
@@ -817,7 +841,8 @@ int shard_debug_gemv(shard_t sh, int layer, int op, const uint16_t* x, int M, fl
   g.M = M;
   g.sp = nullptr;
   g.partials = sh->partials;
-  g.counters = sh->counters;
+  g.flags = sh->flags;
+  g.epoch = next_epochs(sh, 1);
   g.status = sh->status;
   g.ep.kind = EPI_STORE;
   g.ep.dims = p.dims;

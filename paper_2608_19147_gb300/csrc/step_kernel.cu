@@ -3,9 +3,9 @@
 // One CTA per SM, kCtaWarps warps.  The step runs as a sequence of phases separated
 // by grid-wide barriers:
 //   prologue (CTA 0) | for each layer: RMSNorm + q|k|v projection (+RoPE,
-//   K/V append) | attention partials | attention merge | o projection
-//   (+residual) | RMSNorm + gate|up projection (+SwiGLU) | down projection
-//   (+residual; the last layer writes hidden_out).
+//   K/V append) | attention (chunk partials; the last chunk's CTA merges) |
+//   o projection (+residual) | RMSNorm + gate|up projection (+SwiGLU) |
+//   down projection (+residual; the last layer writes hidden_out).
 // Each RMSNorm is computed by every CTA at the start of the projection that
 // consumes it, from per-row-block sums of squares left by the residual's
 // producer, so it needs no barrier of its own.
@@ -258,8 +258,8 @@ __device__ __noinline__ void rmsnorm_cta(const float* x, int H, const uint16_t* 
 // ---------------------------------------------------------------------------
 // Attention.  Item = (request b, kv head hk, chunk c of kChunk entries); one
 // CTA per item.  Each item writes (max, sum of exp, unnormalised output) per
-// query (the request's new tokens x the kv head's query heads); the merge
-// phase combines a request's chunks in order.
+// query (the request's new tokens x the kv head's query heads); the CTA that
+// finishes the last chunk of (b, hk) combines the chunks in order.
 // ---------------------------------------------------------------------------
 // A partial is (max, sum of exp, 2 unused, unnormalised output[d]): the
 // output starts 16-byte aligned.
@@ -272,6 +272,7 @@ struct AttnView {
   size_t layer_stride;
   int cap, Hq, Hkv, d, n_chunks, qmax;
   float* part;
+  int* cnt;  // finished chunks per (request, kv head)
   uint16_t* out;
   int out_ld;
 };
@@ -305,13 +306,76 @@ struct AttnSmem {
   static constexpr size_t kBytes = kK + kV + kQ + kP + 2 * kChunk * sizeof(int);
 };
 
+// Merge of one (request, kv head, query): chunks in order, kMergeBatch at a
+// time with all their loads in flight; lane c of a batch holds chunk c's max
+// and sum, each lane DPL output dims.  The running result is rescaled when a
+// batch raises the maximum (online softmax).
+template <int DPL>
+__device__ __noinline__ void attn_merge_warp(const AttnView* ap, const StepParams* sp, int b, int hk, int qi, int lane) {
+  const AttnView& a = *ap;
+  constexpr int d = 32 * DPL;
+  constexpr int kMergeBatch = 16;
+  using VecT = typename std::conditional<DPL == 4, float4, float2>::type;
+  const int L = sp->req_len[b], tok0 = sp->req_tok0[b];
+  const int G = a.Hq / a.Hkv;
+  const int nc = n_chunks_of(L);
+  const size_t cstride = (size_t)a.qmax * part_stride(d);
+  const float* base = a.part + (((size_t)b * a.Hkv + hk) * a.n_chunks) * cstride + (size_t)qi * part_stride(d);
+  float M = -INFINITY, den = 0.f, num[DPL];
+#pragma unroll
+  for (int u = 0; u < DPL; ++u) num[u] = 0.f;
+  for (int c0 = 0; c0 < nc; c0 += kMergeBatch) {
+    float mc = -INFINITY, lc = 0.f;
+    if (lane < kMergeBatch && c0 + lane < nc) {
+      const float2 ml = __ldcg(reinterpret_cast<const float2*>(base + (size_t)(c0 + lane) * cstride));
+      mc = ml.x;
+      lc = ml.y;
+    }
+    VecT ov[kMergeBatch];
+#pragma unroll
+    for (int u = 0; u < kMergeBatch; ++u) {
+      if (c0 + u < nc) {
+        ov[u] = __ldcg(reinterpret_cast<const VecT*>(base + (size_t)(c0 + u) * cstride + 4) + lane);
+      } else {
+        ov[u] = VecT{};
+      }
+    }
+    float bm = mc;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) bm = fmaxf(bm, __shfl_xor_sync(0xffffffffu, bm, o));
+    const float Mn = fmaxf(M, bm);
+    const float alpha = (M == -INFINITY) ? 0.f : expf(M - Mn);
+    den *= alpha;
+#pragma unroll
+    for (int u = 0; u < DPL; ++u) num[u] *= alpha;
+    const float wl = (mc == -INFINITY) ? 0.f : expf(mc - Mn);
+    float dl = lc * wl;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) dl += __shfl_xor_sync(0xffffffffu, dl, o);
+    den += dl;
+#pragma unroll
+    for (int u = 0; u < kMergeBatch; ++u) {
+      const float w = __shfl_sync(0xffffffffu, wl, u);
+      const float* f = reinterpret_cast<const float*>(&ov[u]);
+#pragma unroll
+      for (int v = 0; v < DPL; ++v) num[v] = fmaf(f[v], w, num[v]);
+    }
+    M = Mn;
+  }
+  uint16_t* out = a.out + (size_t)(tok0 + qi / G) * a.out_ld + (hk * G + qi % G) * d + DPL * lane;
+#pragma unroll
+  for (int u = 0; u < DPL; ++u) out[u] = f2h(num[u] / den);
+}
+
 // One item, processed by the whole CTA:
 //   1. the chunk's slots (beam table) and mask bits;
 //   2. its K and V rows and the first query group into shared memory, every
 //      load of a thread in flight at once;
 //   3. scores: warp w takes queries w, w + kWarps, ...; lane = entry; the
 //      softmax pieces (max, sum of exp) per query across the lanes;
-//   4. values: thread = (query, pair of head dims), sum over the entries.
+//   4. values: thread = (query, pair of head dims), sum over the entries;
+//   5. the CTA that finishes the last chunk of (request, kv head) -- an
+//      acquire-release counter -- merges its queries, one warp each.
 template <int DPL>
 __device__ __noinline__ void attn_item_cta(const AttnView* ap, int layer, const StepParams* sp, int b, int hk, int c,
                                            uint8_t* area) {
@@ -446,68 +510,14 @@ __device__ __noinline__ void attn_item_cta(const AttnView* ap, int layer, const 
       *reinterpret_cast<float2*>(part + (size_t)(q0 + qi) * part_stride(d) + 4 + 2 * dp) = make_float2(o0, o1);
     }
   }
-  __syncthreads();  // the area is reused by the next item
-}
-
-// Merge of one (request, kv head, query): chunks in order, kMergeBatch at a
-// time with all their loads in flight; lane c of a batch holds chunk c's max
-// and sum, each lane DPL output dims.  The running result is rescaled when a
-// batch raises the maximum (online softmax).
-template <int DPL>
-__device__ __noinline__ void attn_merge_warp(const AttnView* ap, const StepParams* sp, int b, int hk, int qi, int lane) {
-  const AttnView& a = *ap;
-  constexpr int d = 32 * DPL;
-  constexpr int kMergeBatch = 16;
-  using VecT = typename std::conditional<DPL == 4, float4, float2>::type;
-  const int L = sp->req_len[b], tok0 = sp->req_tok0[b];
-  const int G = a.Hq / a.Hkv;
-  const int nc = n_chunks_of(L);
-  const size_t cstride = (size_t)a.qmax * part_stride(d);
-  const float* base = a.part + (((size_t)b * a.Hkv + hk) * a.n_chunks) * cstride + (size_t)qi * part_stride(d);
-  float M = -INFINITY, den = 0.f, num[DPL];
-#pragma unroll
-  for (int u = 0; u < DPL; ++u) num[u] = 0.f;
-  for (int c0 = 0; c0 < nc; c0 += kMergeBatch) {
-    float mc = -INFINITY, lc = 0.f;
-    if (lane < kMergeBatch && c0 + lane < nc) {
-      const float2 ml = __ldcg(reinterpret_cast<const float2*>(base + (size_t)(c0 + lane) * cstride));
-      mc = ml.x;
-      lc = ml.y;
-    }
-    VecT ov[kMergeBatch];
-#pragma unroll
-    for (int u = 0; u < kMergeBatch; ++u) {
-      if (c0 + u < nc) {
-        ov[u] = __ldcg(reinterpret_cast<const VecT*>(base + (size_t)(c0 + u) * cstride + 4) + lane);
-      } else {
-        ov[u] = VecT{};
-      }
-    }
-    float bm = mc;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) bm = fmaxf(bm, __shfl_xor_sync(0xffffffffu, bm, o));
-    const float Mn = fmaxf(M, bm);
-    const float alpha = (M == -INFINITY) ? 0.f : expf(M - Mn);
-    den *= alpha;
-#pragma unroll
-    for (int u = 0; u < DPL; ++u) num[u] *= alpha;
-    const float wl = (mc == -INFINITY) ? 0.f : expf(mc - Mn);
-    float dl = lc * wl;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) dl += __shfl_xor_sync(0xffffffffu, dl, o);
-    den += dl;
-#pragma unroll
-    for (int u = 0; u < kMergeBatch; ++u) {
-      const float w = __shfl_sync(0xffffffffu, wl, u);
-      const float* f = reinterpret_cast<const float*>(&ov[u]);
-#pragma unroll
-      for (int v = 0; v < DPL; ++v) num[v] = fmaf(f[v], w, num[v]);
-    }
-    M = Mn;
+  __shared__ int s_last;
+  __syncthreads();  // the item's partials are written; the area is reused by the next item
+  if (tid == 0) s_last = atom_add_acq_rel(&a.cnt[b * a.Hkv + hk], 1) == n_chunks_of(L) - 1;
+  __syncthreads();
+  if (s_last) {
+    for (int qi = warp; qi < Q; qi += kWarps) attn_merge_warp<DPL>(ap, sp, b, hk, qi, lane);
+    if (tid == 0) a.cnt[b * a.Hkv + hk] = 0;
   }
-  uint16_t* out = a.out + (size_t)(tok0 + qi / G) * a.out_ld + (hk * G + qi % G) * d + DPL * lane;
-#pragma unroll
-  for (int u = 0; u < DPL; ++u) out[u] = f2h(num[u] / den);
 }
 
 template <int NT, int GPU, int DPL>
@@ -518,7 +528,6 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
   __shared__ AttnView s_av;
   using SS = StepSmem<GPU>;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int gw = blockIdx.x * kWarps + warp, NW = gridDim.x * kWarps;
   uint8_t* ring = smem + (size_t)warp * kRingSlots * Geom<GPU>::kUnitBytes;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + SS::kRing) + warp * kRingSlots;
   uint8_t* att_area = smem + SS::kRing + SS::kBars;
@@ -551,7 +560,7 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
     gp.M = M;
     gp.skip = skip;
     gp.partials = a.partials;
-    gp.counters = a.counters;
+    gp.flags = a.flags;
     gp.status = a.status;
     gp.sp = sp;
     gp.ep.kind = k == 0 ? EPI_QKV : k == 2 ? EPI_SWIGLU : EPI_RESID;
@@ -582,12 +591,13 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
     av.n_chunks = a.n_chunks;
     av.qmax = kMaxTokens * (a.Hq / a.Hkv);
     av.part = a.attn_part;
+    av.cnt = a.attn_cnt;
     av.out = a.act_attn;
     av.out_ld = a.Kp_dq;
     s_av = av;
   }
   __syncthreads();
-  auto gemv = [&](int op, int l) { gemv_phase<NT, GPU>(&s_ws[warp], op, &s_gp[op & 3], l, lane); };
+  auto gemv = [&](int op, int l) { gemv_phase<NT, GPU>(&s_ws[warp], op, &s_gp[op & 3], l, a.epoch_base + op, lane); };
 
   for (int l = 0; l < a.L; ++l) {
     const uint16_t* nrm = a.norms + (size_t)l * 2 * a.H;
@@ -602,23 +612,6 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
         int b, hk, c;
         if (decode_item(sp, a.Hkv, item, b, hk, c)) attn_item_cta<DPL>(&s_av, l, sp, b, hk, c, att_area);
       }
-      grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
-      // merge items: (b, hk, query)
-      const int G = a.Hq / a.Hkv;
-      total = 0;
-      for (int b = 0; b < sp->B; ++b) total += a.Hkv * (sp->req_tok0[b + 1] - sp->req_tok0[b]) * G;
-      for (int item = gw; item < total; item += NW) {
-        int r = item, b = 0;
-        for (; b < sp->B; ++b) {
-          const int per = a.Hkv * (sp->req_tok0[b + 1] - sp->req_tok0[b]) * G;
-          if (r < per) break;
-          r -= per;
-        }
-        const int Qb = (sp->req_tok0[b + 1] - sp->req_tok0[b]) * G;
-        attn_merge_warp<DPL>(&s_av, sp, b, r / Qb, r % Qb, lane);
-      }
-    } else {
-      grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
     }
     grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
     gemv(4 * l + 1, l);
@@ -657,7 +650,7 @@ cudaError_t setup_t() {
 
 }  // namespace
 
-int step_barriers(int n_layers) { return 6 * n_layers; }
+int step_barriers(int n_layers) { return 5 * n_layers; }
 
 size_t step_attention_part_floats(int B, int Hkv, int n_chunks, int G, int d) {
   return (size_t)B * Hkv * n_chunks * (kMaxTokens * G) * part_stride(d);
