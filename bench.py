@@ -25,6 +25,7 @@ line.
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import hashlib
 import json
 import math
@@ -78,9 +79,9 @@ class Plan:
     position ids, the attention mask rows, beam_idx and token ids or hidden
     states; per-row prefill lengths; the byte counts of the step."""
 
-    def __init__(self, cfg_name: str, K: int, seed: int, request0: int = 0):
+    def __init__(self, cfg_name: str, K: int, seed: int, request0: int = 0, shape=None):
         c = CONFIGS[cfg_name]
-        self.name, self.c, self.shape = cfg_name, c, c["shape"]
+        self.name, self.c, self.shape = cfg_name, c, (shape or c["shape"])
         s = self.shape
         self.B = c["rows"]
         self.n = c["n"]
@@ -247,6 +248,15 @@ def profiled_traffic(kind: str, cfg: str):
     return None
 
 
+def stage_shape(args):
+    """The configuration's stage, or its first --layers layers (a shallower
+    slice of the same kernel, used for profiling captures)."""
+    shape = CONFIGS[args.config]["shape"]
+    if args.layers and args.layers != shape.n_layers:
+        shape = dataclasses.replace(shape, name="%s-first%dL" % (shape.name, args.layers), n_layers=args.layers)
+    return shape
+
+
 def run_gpu(args, rank: int, world: int):
     import torch
 
@@ -260,14 +270,14 @@ def run_gpu(args, rank: int, world: int):
 
         dist.init_process_group("nccl", device_id=dev)
     c = CONFIGS[args.config]
-    shape = c["shape"]
+    shape = stage_shape(args)
     K, W = args.steps, max(3, args.warmup)
     threads = max(1, (os.cpu_count() or 1) // max(1, int(os.environ.get("LOCAL_WORLD_SIZE", world))))
     t_gen = time.time()
     weights = synth.make_weights(shape, SEED, threads=threads)
     log("weights generated in %.1fs (%.2f GB packed)" % (time.time() - t_gen, weights.packed_bytes() / 1e9))
-    plan = Plan(args.config, K, SEED)
-    warm = Plan(args.config, W, SEED + 1)
+    plan = Plan(args.config, K, SEED, shape=shape)
+    warm = Plan(args.config, W, SEED + 1, shape=shape)
     sh = pkg.shard_create(pkg.make_config(shape), weights.layers, weights.embedding)
     stream = torch.cuda.current_stream(dev)
     sptr = stream.cuda_stream
@@ -360,7 +370,7 @@ def run_gpu(args, rank: int, world: int):
     # ---- per-phase times: the step kernel's barrier timestamps, averaged
     # over a pass of the same workload (one step, then read, per step) ----
     prof_K = min(K, 64)
-    pplan = Plan(args.config, prof_K, SEED + 2)
+    pplan = Plan(args.config, prof_K, SEED + 2, shape=shape)
     pst, pd = load_states(pplan), stage(pplan)
     PHASES = list(pkg.PHASES)
     n_ph = len(PHASES) * shape.n_layers
@@ -384,7 +394,7 @@ def run_gpu(args, rank: int, world: int):
         pkg.kv_state_free(st)
 
     # ---- end to end through the host-buffer entry point ----
-    eplan = Plan(args.config, K, SEED + 3)
+    eplan = Plan(args.config, K, SEED + 3, shape=shape)
     est = load_states(eplan)
     out = np.empty((eplan.M, shape.hidden), np.uint16)
     h2d = d2h = 0
@@ -438,7 +448,8 @@ def run_gpu(args, rank: int, world: int):
         "dtype": "w4a16 (uint4 weights, fp16 activations, fp32 accumulate)",
         "data": "synthetic (seeded Gaussian weights quantised to uint4; no checkpoints available)",
         "config": {
-            "workload": c["workload"],
+            "workload": c["workload"] + ("" if shape.n_layers == c["shape"].n_layers else
+                                         " [profiling slice: first %d layers only]" % shape.n_layers),
             "shard": "%s: %d layers, hidden %d, %dq/%dkv heads, head_dim %d, ffn %d, group %d" % (
                 shape.name, shape.n_layers, shape.hidden, shape.n_heads, shape.n_kv_heads, shape.head_dim, shape.ffn,
                 shape.group),
@@ -459,7 +470,7 @@ def run_gpu(args, rank: int, world: int):
             "frac": step_bytes / (ms / K * 1e6) / peak,
             "peak_note": "%s: MEASURED_PEAKS.json hbm_gbs (a copy bandwidth); achieved = algorithmic bytes per "
                          "launch / CUDA-event time of the timed launches" % peak_note,
-            "traffic": profiled_traffic("step", args.config),
+            "traffic": profiled_traffic("step", args.config) if shape.n_layers == c["shape"].n_layers else None,
             "frac_of_8tbs_nominal": step_bytes / (ms / K * 1e6) / 8000.0,
         },
         "phases": phases,
@@ -540,6 +551,8 @@ def main():
     ap.add_argument("--config", default="8b-decode", choices=list(CONFIGS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=20.0)
+    ap.add_argument("--layers", type=int, default=0,
+                    help="run only the stage's first N layers (profiling captures); default: the whole stage")
     args = ap.parse_args()
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
