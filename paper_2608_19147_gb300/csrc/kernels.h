@@ -201,7 +201,7 @@ struct StepKernelArgs {
   uint16_t* kpool;           // [L][n_rows][Hkv][cap][d]
   uint16_t* vpool;
   size_t layer_stride;
-  int cap, n_chunks;         // attention items are 32 entries
+  int cap, n_chunks;         // items per row at kAttnChunkMin entries (the partials layout)
   float* attn_part;          // [B][Hkv][n_chunks][16*G][d+4]
   int* attn_cnt;             // [16][Hkv] finished chunks per (request, kv head); zero, self-resetting
   int* status;
@@ -216,7 +216,8 @@ cudaError_t step_setup(int group, int head_dim);
 int step_barriers(int n_layers);
 cudaError_t launch_step(const StepKernelArgs& a, int nt, int group, int grid, cudaStream_t s);
 size_t step_attention_part_floats(int B, int Hkv, int n_chunks, int G, int d);
-constexpr int kAttnChunk = 32;
+constexpr int kAttnChunk = 64;     // most cache entries per attention item
+constexpr int kAttnChunkMin = 32;  // fewest (partials are laid out for this many per item)
 
 // Weight repacking (one fused op; all source pointers device).
 // Source matrices of a fused op (q, k, v for OP_QKV; gate, up for OP_GU; one

@@ -117,7 +117,7 @@ struct kvstate_s {
   std::vector<int> cursor, len_host;
   bool shared = false;    // rows may share entries (a beam gather ran)
   bool poisoned = false;  // a step aborted on the device
-  int n_chunks = 0;       // attention items per row (32 entries each)
+  int n_chunks = 0;       // attention items per row at the smallest item size (kAttnChunkMin)
   float* attn_part = nullptr;
 };
 
@@ -452,7 +452,7 @@ int kv_state_alloc(shard_t sh, int n_rows, int capacity, kvstate_t* out) {
   const size_t pool = st->layer_stride * sh->L;
   st->cursor.assign(n_rows, 0);
   st->len_host.assign(n_rows, 0);
-  st->n_chunks = (capacity + kAttnChunk - 1) / kAttnChunk;
+  st->n_chunks = (capacity + kAttnChunkMin - 1) / kAttnChunkMin;
   int rc = SHARD_OK;
   auto chk = [&](cudaError_t e) {
     if (e != cudaSuccess && rc == SHARD_OK)

@@ -26,14 +26,14 @@ namespace {
 
 constexpr int kWarps = kCtaWarps;
 constexpr int kThreads = kWarps * 32;
-constexpr int kChunk = 32;        // cache entries per attention item (one per lane)
+constexpr int kChunk = kAttnChunk;  // most cache entries per attention item (two per lane)
 
 template <int GPU>
 struct StepSmem {
   static constexpr size_t kRing = (size_t)kWarps * kRingSlots * Geom<GPU>::kUnitBytes;
   static constexpr size_t kBars = (size_t)kWarps * kRingSlots * sizeof(uint64_t);
   // attention item area (AttnSmem)
-  static constexpr size_t kQ = 32 * 1024;
+  static constexpr size_t kQ = 48 * 1024;
   static constexpr size_t kFixed = kRing + kBars + kQ;  // + the op table (4L entries)
   static size_t total(int n_layers) { return kFixed + (size_t)4 * n_layers * sizeof(OpDesc); }
 };
@@ -56,6 +56,15 @@ __device__ __forceinline__ float2 h2f2(uint32_t u) {
   __half2 h;
   memcpy(&h, &u, sizeof(h));
   return __half22float2(h);
+}
+
+__device__ __forceinline__ void red_release_add_s32(int* p, int v) {
+  asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ int ld_acquire_s32(const int* p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
 }
 
 __device__ __forceinline__ void red_release_add(unsigned long long* p, unsigned long long v) {
@@ -256,10 +265,16 @@ __device__ __noinline__ void rmsnorm_cta(const float* x, int H, const uint16_t* 
 }
 
 // ---------------------------------------------------------------------------
-// Attention.  Item = (request b, kv head hk, chunk c of kChunk entries); one
-// CTA per item.  Each item writes (max, sum of exp, unnormalised output) per
-// query (the request's new tokens x the kv head's query heads); the CTA that
-// finishes the last chunk of (b, hk) combines the chunks in order.
+// Attention.  Item = (request b, kv head hk, chunk c of cs entries); one CTA
+// per item, items dealt round-robin.  cs is 32 when that gives no more items
+// than CTAs (short caches: more parallel items), else 64 (long caches: fewer
+// rounds and merges).  Each item writes (max, sum of exp,
+// unnormalised output) per query (the request's new tokens x the kv head's
+// query heads).  With several items per CTA, after its items the CTA that
+// took the last chunk of (b, hk) waits for the chunk count and combines the
+// chunks in order, so the merges are spread over CTAs and never delay
+// anyone's items; with one item per CTA at most, the CTA that finishes the
+// last chunk merges at once.
 // ---------------------------------------------------------------------------
 // A partial is (max, sum of exp, 2 unused, unnormalised output[d]): the
 // output starts 16-byte aligned.
@@ -273,24 +288,87 @@ struct AttnView {
   int cap, Hq, Hkv, d, n_chunks, qmax;
   float* part;
   int* cnt;  // finished chunks per (request, kv head)
+  int cs;    // entries per item this step: kAttnChunkMin, or kChunk when that gives more items than CTAs
+  int last_merges;  // at most one item per CTA: the CTA finishing the last chunk merges at once
   uint16_t* out;
   int out_ld;
 };
 
-__device__ __forceinline__ int n_chunks_of(int L) { return (L + kChunk - 1) / kChunk; }
+__device__ __forceinline__ int n_chunks_of(int L, int cs) { return (L + cs - 1) / cs; }
 
 // Finds the item's (b, hk, c) from a flat index; false if past the end.
-__device__ __forceinline__ bool decode_item(const StepParams* sp, int Hkv, int item, int& b, int& hk, int& c) {
+__device__ __forceinline__ bool decode_item(const StepParams* sp, int Hkv, int cs, int item, int& b, int& hk, int& c) {
   for (b = 0; b < sp->B; ++b) {
-    const int per = Hkv * n_chunks_of(sp->req_len[b]);
+    const int per = Hkv * n_chunks_of(sp->req_len[b], cs);
     if (item < per) {
-      hk = item / n_chunks_of(sp->req_len[b]);
-      c = item % n_chunks_of(sp->req_len[b]);
+      hk = item / n_chunks_of(sp->req_len[b], cs);
+      c = item % n_chunks_of(sp->req_len[b], cs);
       return true;
     }
     item -= per;
   }
   return false;
+}
+
+// q (fp32, shared) . K row (fp16, shared) over KP 8-element pieces; the
+// two-row form scores rows k0 and k1 with one pass over q.
+__device__ __forceinline__ float dot_q_k(const float* qq, const uint16_t* k0r, int KP) {
+  float s0 = 0.f;
+#pragma unroll 4
+  for (int t = 0; t < KP; ++t) {
+    const uint4 k0 = *reinterpret_cast<const uint4*>(k0r + t * 8);
+    const float4 qa = *reinterpret_cast<const float4*>(qq + t * 8);
+    const float4 qb = *reinterpret_cast<const float4*>(qq + t * 8 + 4);
+    float2 f = h2f2(k0.x);
+    s0 = fmaf(qa.x, f.x, s0);
+    s0 = fmaf(qa.y, f.y, s0);
+    f = h2f2(k0.y);
+    s0 = fmaf(qa.z, f.x, s0);
+    s0 = fmaf(qa.w, f.y, s0);
+    f = h2f2(k0.z);
+    s0 = fmaf(qb.x, f.x, s0);
+    s0 = fmaf(qb.y, f.y, s0);
+    f = h2f2(k0.w);
+    s0 = fmaf(qb.z, f.x, s0);
+    s0 = fmaf(qb.w, f.y, s0);
+  }
+  return s0;
+}
+__device__ __forceinline__ float dot_q_k2(const float* qq, const uint16_t* k0r, const uint16_t* k1r, float& s1,
+                                          int KP) {
+  float s0 = 0.f;
+  s1 = 0.f;
+#pragma unroll 4
+  for (int t = 0; t < KP; ++t) {
+    const uint4 k0 = *reinterpret_cast<const uint4*>(k0r + t * 8);
+    const uint4 k1 = *reinterpret_cast<const uint4*>(k1r + t * 8);
+    const float4 qa = *reinterpret_cast<const float4*>(qq + t * 8);
+    const float4 qb = *reinterpret_cast<const float4*>(qq + t * 8 + 4);
+    float2 f = h2f2(k0.x), g = h2f2(k1.x);
+    s0 = fmaf(qa.x, f.x, s0);
+    s0 = fmaf(qa.y, f.y, s0);
+    s1 = fmaf(qa.x, g.x, s1);
+    s1 = fmaf(qa.y, g.y, s1);
+    f = h2f2(k0.y);
+    g = h2f2(k1.y);
+    s0 = fmaf(qa.z, f.x, s0);
+    s0 = fmaf(qa.w, f.y, s0);
+    s1 = fmaf(qa.z, g.x, s1);
+    s1 = fmaf(qa.w, g.y, s1);
+    f = h2f2(k0.z);
+    g = h2f2(k1.z);
+    s0 = fmaf(qb.x, f.x, s0);
+    s0 = fmaf(qb.y, f.y, s0);
+    s1 = fmaf(qb.x, g.x, s1);
+    s1 = fmaf(qb.y, g.y, s1);
+    f = h2f2(k0.w);
+    g = h2f2(k1.w);
+    s0 = fmaf(qb.z, f.x, s0);
+    s0 = fmaf(qb.w, f.y, s0);
+    s1 = fmaf(qb.z, g.x, s1);
+    s1 = fmaf(qb.w, g.y, s1);
+  }
+  return s0;
 }
 
 // Shared-memory layout of one attention item.
@@ -318,7 +396,7 @@ __device__ __noinline__ void attn_merge_warp(const AttnView* ap, const StepParam
   using VecT = typename std::conditional<DPL == 4, float4, float2>::type;
   const int L = sp->req_len[b], tok0 = sp->req_tok0[b];
   const int G = a.Hq / a.Hkv;
-  const int nc = n_chunks_of(L);
+  const int nc = n_chunks_of(L, a.cs);
   const size_t cstride = (size_t)a.qmax * part_stride(d);
   const float* base = a.part + (((size_t)b * a.Hkv + hk) * a.n_chunks) * cstride + (size_t)qi * part_stride(d);
   float M = -INFINITY, den = 0.f, num[DPL];
@@ -374,8 +452,9 @@ __device__ __noinline__ void attn_merge_warp(const AttnView* ap, const StepParam
 //   3. scores: warp w takes queries w, w + kWarps, ...; lane = entry; the
 //      softmax pieces (max, sum of exp) per query across the lanes;
 //   4. values: thread = (query, pair of head dims), sum over the entries;
-//   5. the CTA that finishes the last chunk of (request, kv head) -- an
-//      acquire-release counter -- merges its queries, one warp each.
+//   5. a release count of the finished chunk for its (request, kv head); when
+//      every CTA has at most one item, the CTA that counts the last chunk
+//      merges at once.
 template <int DPL>
 __device__ __noinline__ void attn_item_cta(const AttnView* ap, int layer, const StepParams* sp, int b, int hk, int c,
                                            uint8_t* area) {
@@ -394,7 +473,7 @@ __device__ __noinline__ void attn_item_cta(const AttnView* ap, int layer, const 
   const int L = sp->req_len[b], P = sp->req_P[b];
   const int tok0 = sp->req_tok0[b], nb = sp->req_tok0[b + 1] - tok0;
   const int G = a.Hq / a.Hkv, Q = nb * G;
-  const int j0 = c * kChunk, nj = min(kChunk, L - j0);
+  const int j0 = c * a.cs, nj = min(a.cs, L - j0);
   const float scale = rsqrtf(static_cast<float>(d));
   float* part = a.part + ((((size_t)b * a.Hkv + hk) * a.n_chunks + c) * a.qmax) * part_stride(d);
   // query qi of the item is head hk * G + qi % G of token tok0 + qi / G
@@ -459,37 +538,26 @@ __device__ __noinline__ void attn_item_cta(const AttnView* ap, int layer, const 
     __syncthreads();
     for (int qi = warp; qi < qn; qi += kWarps) {
       const float* qq = qsm + qi * d;
-      const uint16_t* kr = Ks + lane * S::kKld;
-      float s = 0.f;
-#pragma unroll 4
-      for (int t = 0; t < KP; ++t) {
-        const uint4 kk = *reinterpret_cast<const uint4*>(kr + t * 8);
-        const float4 qa = *reinterpret_cast<const float4*>(qq + t * 8);
-        const float4 qb = *reinterpret_cast<const float4*>(qq + t * 8 + 4);
-        float2 f = h2f2(kk.x);
-        s = fmaf(qa.x, f.x, s);
-        s = fmaf(qa.y, f.y, s);
-        f = h2f2(kk.y);
-        s = fmaf(qa.z, f.x, s);
-        s = fmaf(qa.w, f.y, s);
-        f = h2f2(kk.z);
-        s = fmaf(qb.x, f.x, s);
-        s = fmaf(qb.y, f.y, s);
-        f = h2f2(kk.w);
-        s = fmaf(qb.z, f.x, s);
-        s = fmaf(qb.w, f.y, s);
+      float s0, s1 = 0.f;
+      if (a.cs > 32) {
+        s0 = dot_q_k2(qq, Ks + lane * S::kKld, Ks + (lane + 32) * S::kKld, s1, KP);
+      } else {
+        s0 = dot_q_k(qq, Ks + lane * S::kKld, KP);
       }
       const int q = q0 + qi;
-      const bool vis = lane < nj && vis_s[lane] && j0 + lane <= P + q / G;
-      const float val = vis ? s * scale : -INFINITY;
-      float mx = val;
+      const int lim = P + q / G;  // causal limit of this query's token
+      const bool vis0 = lane < nj && vis_s[lane] && j0 + lane <= lim;
+      const bool vis1 = lane + 32 < nj && vis_s[lane + 32] && j0 + lane + 32 <= lim;
+      const float v0 = vis0 ? s0 * scale : -INFINITY, v1 = vis1 ? s1 * scale : -INFINITY;
+      float mx = fmaxf(v0, v1);
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-      const float e = vis ? expf(val - mx) : 0.f;
-      float l = e;
+      const float e0 = vis0 ? expf(v0 - mx) : 0.f, e1 = vis1 ? expf(v1 - mx) : 0.f;
+      float l = e0 + e1;
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
-      ps[qi * kChunk + lane] = e;
+      ps[qi * kChunk + lane] = e0;
+      ps[qi * kChunk + lane + 32] = e1;
       if (lane == 0) {
         part[(size_t)q * part_stride(d)] = mx;
         part[(size_t)q * part_stride(d) + 1] = l;
@@ -501,7 +569,7 @@ __device__ __noinline__ void attn_item_cta(const AttnView* ap, int layer, const 
       const float* pq = ps + qi * kChunk;
       float o0 = 0.f, o1 = 0.f;
 #pragma unroll 8
-      for (int e = 0; e < kChunk; ++e) {  // rows past nj are zero with weight zero
+      for (int e = 0; e < a.cs; ++e) {  // rows past nj are zero with weight zero
         const float pe = pq[e];
         const float2 vf = h2f2(*reinterpret_cast<const uint32_t*>(Vs + e * d + 2 * dp));
         o0 = fmaf(pe, vf.x, o0);
@@ -510,14 +578,46 @@ __device__ __noinline__ void attn_item_cta(const AttnView* ap, int layer, const 
       *reinterpret_cast<float2*>(part + (size_t)(q0 + qi) * part_stride(d) + 4 + 2 * dp) = make_float2(o0, o1);
     }
   }
+  // the item's partials are written (and the area is free for the next item);
+  // the release orders them before the count the merging CTA acquires
+  __syncthreads();
+  if (!a.last_merges) {
+    if (tid == 0) red_release_add_s32(&a.cnt[b * a.Hkv + hk], 1);
+    return;
+  }
   __shared__ int s_last;
-  __syncthreads();  // the item's partials are written; the area is reused by the next item
-  if (tid == 0) s_last = atom_add_acq_rel(&a.cnt[b * a.Hkv + hk], 1) == n_chunks_of(L) - 1;
+  if (tid == 0) s_last = atom_add_acq_rel(&a.cnt[b * a.Hkv + hk], 1) == n_chunks_of(L, a.cs) - 1;
   __syncthreads();
   if (s_last) {
     for (int qi = warp; qi < Q; qi += kWarps) attn_merge_warp<DPL>(ap, sp, b, hk, qi, lane);
+    __syncthreads();
     if (tid == 0) a.cnt[b * a.Hkv + hk] = 0;
   }
+}
+
+// Merge of (request b, kv head hk) by its designated CTA, after that CTA's
+// own items: wait until every chunk is counted (bounded), merge the queries
+// (one warp each), reset the count.
+template <int DPL>
+__device__ __noinline__ void attn_merge_cta(const AttnView* ap, const StepParams* sp, int b, int hk, int* status) {
+  const AttnView& a = *ap;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int L = sp->req_len[b], nb = sp->req_tok0[b + 1] - sp->req_tok0[b];
+  const int Q = nb * (a.Hq / a.Hkv);
+  if (tid == 0) {
+    uint32_t it = 0;
+    while (ld_acquire_s32(&a.cnt[b * a.Hkv + hk]) < n_chunks_of(L, a.cs)) {
+      if (++it > (1u << 22)) {
+        atomicOr(status, ST_WAIT_TIMEOUT);
+        break;
+      }
+      __nanosleep(64);
+    }
+  }
+  __syncthreads();
+  for (int qi = warp; qi < Q; qi += kWarps) attn_merge_warp<DPL>(ap, sp, b, hk, qi, lane);
+  __syncthreads();
+  if (tid == 0) a.cnt[b * a.Hkv + hk] = 0;
 }
 
 template <int NT, int GPU, int DPL>
@@ -592,6 +692,10 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
     av.qmax = kMaxTokens * (a.Hq / a.Hkv);
     av.part = a.attn_part;
     av.cnt = a.attn_cnt;
+    int items = 0;
+    for (int b = 0; b < sp->B; ++b) items += a.Hkv * n_chunks_of(sp->req_len[b], kAttnChunkMin);
+    av.cs = items > (int)gridDim.x ? kChunk : kAttnChunkMin;
+    av.last_merges = items <= (int)gridDim.x;
     av.out = a.act_attn;
     av.out_ld = a.Kp_dq;
     s_av = av;
@@ -607,10 +711,18 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
     grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
     if (!skip) {
       int total = 0;
-      for (int b = 0; b < sp->B; ++b) total += a.Hkv * n_chunks_of(sp->req_len[b]);
+      for (int b = 0; b < sp->B; ++b) total += a.Hkv * n_chunks_of(sp->req_len[b], s_av.cs);
       for (int item = blockIdx.x; item < total; item += gridDim.x) {
         int b, hk, c;
-        if (decode_item(sp, a.Hkv, item, b, hk, c)) attn_item_cta<DPL>(&s_av, l, sp, b, hk, c, att_area);
+        if (decode_item(sp, a.Hkv, s_av.cs, item, b, hk, c)) attn_item_cta<DPL>(&s_av, l, sp, b, hk, c, att_area);
+      }
+      // merges, when CTAs take several items: (b, hk) goes to the CTA that
+      // took its last chunk
+      for (int b = 0, base = 0; !s_av.last_merges && b < sp->B; ++b) {
+        const int nc = n_chunks_of(sp->req_len[b], s_av.cs);
+        for (int hk = 0; hk < a.Hkv; ++hk)
+          if ((base + hk * nc + nc - 1) % gridDim.x == blockIdx.x) attn_merge_cta<DPL>(&s_av, sp, b, hk, a.status);
+        base += a.Hkv * nc;
       }
     }
     grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
