@@ -386,7 +386,7 @@ def run_gpu(args, rank: int, world: int):
     for i, name in enumerate(PHASES):
         v = np.array(lay[i::len(PHASES)])
         phases[name] = {"avg_us_per_layer": float(v.mean()), "total_us_per_step": float(v.sum())}
-    for name, kind in (("qkv", "qkv"), ("o", "o"), ("gate_up", "gate_up"), ("down", "down")):
+    for name, kind in (("o", "o"), ("gate_up", "gate_up"), ("down", "down")):
         t_us = phases[name]["avg_us_per_layer"]
         if t_us > 0:
             phases[name]["achieved_gbs"] = pplan.kind_bytes(kind) / (t_us * 1e3)

@@ -41,8 +41,8 @@ int shard_debug_gemv(shard_t shard, int layer, int op, const uint16_t* x, int M,
 /* Phase durations of the last completed shard_step, from the GPU's global
  * timer read by one thread at each grid barrier of the step kernel: us[i] is
  * the time between barrier i and barrier i+1 (barrier 0 = kernel start;
- * order: prologue, then per layer: RMSNorm + q|k|v, attention (partials
- * and merge), o, RMSNorm + gate|up, down; the last layer's down phase
+ * order: prologue, then per layer: RMSNorm + q|k|v + attention, o,
+ * RMSNorm + gate|up, down; the last layer's down phase
  * ends with the kernel and is not reported).  Returns the number of values
  * written (at most n), or a negative error.  Synchronises the device. */
 int shard_debug_phase_times(shard_t shard, double* us, int n);

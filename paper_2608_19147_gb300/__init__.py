@@ -28,7 +28,8 @@ EXPORTS = ("shard_create", "shard_destroy", "kv_state_alloc", "kv_state_free", "
            "kv_state_read", "kv_state_length", "kv_trim", "shard_step", "shard_step_host", "shard_sync_status",
            "shard_last_error", "shard_debug_op_info", "shard_debug_unpack", "shard_debug_gemv",
            "shard_debug_phase_times", "shard_gemv_noalloc")
-PHASES = ("qkv", "attention", "o", "gate_up", "down")  # qkv and gate_up include their RMSNorm
+# per layer, between grid barriers: RMSNorm + q|k|v + attention, o, RMSNorm + gate|up, down
+PHASES = ("qkv_attention", "o", "gate_up", "down")
 
 
 class ShardError(RuntimeError):

@@ -332,6 +332,8 @@ struct GemvPhase {
   int* status;
   const StepParams* sp;
   EpiArgs ep;
+  unsigned* done_flags;  // nullptr, or row-block flags this projection publishes (release of the epoch
+                         // after the row-block's epilogue)
 };
 
 // Floats of one stored piece: [token][64 rows] for up to kMaxTokens tokens.
@@ -368,7 +370,7 @@ __device__ __forceinline__ void load_act(uint4 (&act)[NT][2][2], const uint16_t*
 // if its run started before the row-block.  When T < nw some runs are empty
 // and each non-empty run is a single unit.
 static __device__ __noinline__ void finish_rowblock(const GemvPhase* pp, int layer, int rb, int g_first, int g_last,
-                                                    int T, int nw, int upr, int lane) {
+                                                    int T, int nw, int upr, int lane, unsigned epoch) {
   const GemvPhase& p = *pp;
   constexpr int kPerLane = 8;  // pieces per lane and batch (32 per batch over the 4 piece groups)
   const int rb_begin = rb * upr;
@@ -425,6 +427,10 @@ static __device__ __noinline__ void finish_rowblock(const GemvPhase* pp, int lay
       if (lane == 0) p.ep.ss[rb * kMaxTokens + m] = ss;
     }
   }
+  if (p.done_flags) {
+    __syncwarp();
+    if (lane == 0) st_release_u32(p.done_flags + rb, epoch);
+  }
 }
 
 // Merge of split row-block rb by the warp owning its last unit: wait until
@@ -452,7 +458,7 @@ static __device__ __noinline__ void merge_rowblock(const GemvPhase* pp, int laye
     }
   }
   __syncwarp();
-  finish_rowblock(pp, layer, rb, g_first, g_last, T, nw, upr, lane);
+  finish_rowblock(pp, layer, rb, g_first, g_last, T, nw, upr, lane, epoch);
 }
 
 // End of one row-block segment of a warp's run: store the piece (slot 0:
@@ -481,7 +487,7 @@ __device__ __forceinline__ void piece_end(const GemvPhase* pp, int layer, const 
       }
   __syncwarp();
   if (whole) {
-    finish_rowblock(pp, layer, rb, g, g, T, nw, upr, lane);
+    finish_rowblock(pp, layer, rb, g, g, T, nw, upr, lane, epoch);
     return;
   }
   // The warp barrier above orders every lane's piece stores before lane 0's

@@ -204,6 +204,7 @@ struct StepKernelArgs {
   int cap, n_chunks;         // items per row at kAttnChunkMin entries (the partials layout)
   float* attn_part;          // [B][Hkv][n_chunks][16*G][d+4]
   int* attn_cnt;             // [16][Hkv] finished chunks per (request, kv head); zero, self-resetting
+  unsigned* rb_done;         // [max row-blocks] epoch of each q|k|v row-block's finish
   int* status;
   unsigned long long* barrier;         // grid-barrier counter (monotonic)
   unsigned long long barrier_base;     // its value when this launch starts

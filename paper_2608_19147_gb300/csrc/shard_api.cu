@@ -80,6 +80,7 @@ struct shard_s {
   float* x = nullptr;              // [16][H]
   float* ss = nullptr;             // [n_rb_H][16] per 64-row block sums of squares of x
   int* attn_cnt = nullptr;         // [16][Hkv] attention chunks finished per (request, kv head)
+  unsigned* rb_done = nullptr;     // [max_rb] epoch of each q|k|v row-block's last finish
   uint16_t* act_h = nullptr;       // [16][Kp_H]
   uint16_t* act_attn = nullptr;    // [16][Kp_dq]
   uint16_t* act_f = nullptr;       // [16][Kp_F]
@@ -188,6 +189,7 @@ unsigned next_epochs(shard_s* sh, unsigned n) {
   if (sh->epoch > 0xFFFFFFFFu - n) {
     cudaDeviceSynchronize();
     cudaMemset(sh->flags, 0, sizeof(unsigned) * gemv_flags_count(std::max(std::max(sh->grid[1], sh->grid[2]), sh->num_sms)));
+    cudaMemset(sh->rb_done, 0, sizeof(unsigned) * sh->max_rb);
     cudaDeviceSynchronize();
     sh->epoch = 1;
   }
@@ -370,6 +372,8 @@ int shard_create(const shard_config* cfg, const shard_weights_host* w, shard_t* 
   CUDA_TRY(cudaMalloc(&sh->ss, sizeof(float) * kMaxTokens * ((sh->H + kRowsPerBlock - 1) / kRowsPerBlock)));
   CUDA_TRY(cudaMalloc(&sh->attn_cnt, sizeof(int) * kMaxRequests * sh->Hkv));
   CUDA_TRY(cudaMemset(sh->attn_cnt, 0, sizeof(int) * kMaxRequests * sh->Hkv));
+  CUDA_TRY(cudaMalloc(&sh->rb_done, sizeof(unsigned) * sh->max_rb));
+  CUDA_TRY(cudaMemset(sh->rb_done, 0, sizeof(unsigned) * sh->max_rb));
   CUDA_TRY(cudaMalloc(&sh->act_h, sizeof(uint16_t) * kMaxTokens * sh->Kp_H));
   CUDA_TRY(cudaMalloc(&sh->act_attn, sizeof(uint16_t) * kMaxTokens * sh->Kp_dq));
   CUDA_TRY(cudaMalloc(&sh->act_f, sizeof(uint16_t) * kMaxTokens * sh->Kp_F));
@@ -421,6 +425,7 @@ int shard_destroy(shard_t sh) {
   cudaFree(sh->x);
   cudaFree(sh->ss);
   cudaFree(sh->attn_cnt);
+  cudaFree(sh->rb_done);
   cudaFree(sh->act_h);
   cudaFree(sh->act_attn);
   cudaFree(sh->act_f);
@@ -699,6 +704,7 @@ int shard_step(shard_t sh, kvstate_t st, const uint16_t* hidden_in, const int32_
   ka.n_chunks = st->n_chunks;
   ka.attn_part = st->attn_part;
   ka.attn_cnt = sh->attn_cnt;
+  ka.rb_done = sh->rb_done;
   ka.status = sh->status;
   ka.barrier = sh->barrier;
   ka.barrier_base = sh->barrier_base;

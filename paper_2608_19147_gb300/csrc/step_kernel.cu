@@ -1,11 +1,16 @@
 // The whole decode step of a shard as one persistent, cooperative kernel.
 //
 // One CTA per SM, kCtaWarps warps.  The step runs as a sequence of phases separated
-// by grid-wide barriers:
+// by grid-wide barriers ('|'):
 //   prologue (CTA 0) | for each layer: RMSNorm + q|k|v projection (+RoPE,
-//   K/V append) | attention (chunk partials; the last chunk's CTA merges) |
-//   o projection (+residual) | RMSNorm + gate|up projection (+SwiGLU) |
-//   down projection (+residual; the last layer writes hidden_out).
+//   K/V append) -> attention (chunk partials and merges) | o projection
+//   (+residual) | RMSNorm + gate|up projection (+SwiGLU) | down projection
+//   (+residual; the last layer writes hidden_out).
+// '->' is dataflow instead of a barrier: each q|k|v row-block's finisher
+// release-stores the launch's epoch of that projection into the row-block's
+// flag, and an attention item waits (acquire loads, bounded) only for the
+// row-blocks of its kv head.  Flags are never cleared: an epoch is unique per
+// launch and op.
 // Each RMSNorm is computed by every CTA at the start of the projection that
 // consumes it, from per-row-block sums of squares left by the residual's
 // producer, so it needs no barrier of its own.
@@ -288,6 +293,8 @@ struct AttnView {
   int cap, Hq, Hkv, d, n_chunks, qmax;
   float* part;
   int* cnt;  // finished chunks per (request, kv head)
+  const unsigned* rb_done;  // q|k|v row-block flags the items wait for
+  int rb_k0, rb_v0;         // first k and v row-block of the q|k|v projection
   int cs;    // entries per item this step: kAttnChunkMin, or kChunk when that gives more items than CTAs
   int last_merges;  // at most one item per CTA: the CTA finishing the last chunk merges at once
   uint16_t* out;
@@ -447,8 +454,9 @@ __device__ __noinline__ void attn_merge_warp(const AttnView* ap, const StepParam
 
 // One item, processed by the whole CTA:
 //   1. the chunk's slots (beam table) and mask bits;
-//   2. its K and V rows and the first query group into shared memory, every
-//      load of a thread in flight at once;
+//   2. its K and V rows -- those of earlier steps before waiting for this
+//      step's q|k|v row-blocks, the appended ones after -- and the first query
+//      group into shared memory, every load of a thread in flight at once;
 //   3. scores: warp w takes queries w, w + kWarps, ...; lane = entry; the
 //      softmax pieces (max, sum of exp) per query across the lanes;
 //   4. values: thread = (query, pair of head dims), sum over the entries;
@@ -457,7 +465,7 @@ __device__ __noinline__ void attn_merge_warp(const AttnView* ap, const StepParam
 //      merges at once.
 template <int DPL>
 __device__ __noinline__ void attn_item_cta(const AttnView* ap, int layer, const StepParams* sp, int b, int hk, int c,
-                                           uint8_t* area) {
+                                           uint8_t* area, unsigned qkv_epoch, int* status) {
   const AttnView& a = *ap;
   const uint16_t* kpool = a.kpool + (size_t)layer * a.layer_stride;
   const uint16_t* vpool = a.vpool + (size_t)layer * a.layer_stride;
@@ -479,6 +487,7 @@ __device__ __noinline__ void attn_item_cta(const AttnView* ap, int layer, const 
   // query qi of the item is head hk * G + qi % G of token tok0 + qi / G
   auto q_src = [&](int qi) { return a.q + (size_t)(tok0 + qi / G) * a.Hq * d + (hk * G + qi % G) * d; };
 
+  // 1. the chunk's slots and mask bits (independent of this step's projections)
   if (tid < kChunk) {
     int slot = 0, vis = 0;
     if (tid < nj) {
@@ -497,15 +506,43 @@ __device__ __noinline__ void attn_item_cta(const AttnView* ap, int layer, const 
     const int qn0 = min(S::kQg, Q);
     uint4 v[kPer];
     float4 qv[kQPer];
+    auto load_row_piece = [&](int pi, int r) {
+      const int sl = slot_s[r];
+      const size_t row = (((size_t)(sl / a.cap) * a.Hkv + hk) * a.cap + sl % a.cap) * d;
+      return __ldcg(reinterpret_cast<const uint4*>((pi >= kRowPieces ? vpool : kpool) + row) + pi % KP);
+    };
+    // 2. K/V rows of entries from earlier steps: in flight during the wait
 #pragma unroll
     for (int i = 0; i < kPer; ++i) {
       const int pi = tid + i * kThreads, r = (pi % kRowPieces) / KP;
       v[i] = make_uint4(0, 0, 0, 0);
-      if (pi < 2 * kRowPieces && r < nj) {
-        const int sl = slot_s[r];
-        const size_t row = (((size_t)(sl / a.cap) * a.Hkv + hk) * a.cap + sl % a.cap) * d;
-        v[i] = __ldcg(reinterpret_cast<const uint4*>((pi >= kRowPieces ? vpool : kpool) + row) + pi % KP);
+      if (pi < 2 * kRowPieces && r < nj && j0 + r < P) v[i] = load_row_piece(pi, r);
+    }
+    // 3. wait (bounded) for this kv head's q|k|v row-blocks: its G q heads,
+    //    its k and its v
+    {
+      const int per_head = d / kRowsPerBlock > 0 ? d / kRowsPerBlock : 1;
+      const int nq = G * d / kRowsPerBlock, n = nq + 2 * per_head;
+      if (tid < n) {
+        const int r = tid < nq ? hk * G * d / kRowsPerBlock + tid
+                               : (tid < nq + per_head ? a.rb_k0 + hk * per_head + (tid - nq)
+                                                      : a.rb_v0 + hk * per_head + (tid - nq - per_head));
+        uint32_t it = 0;
+        while (ld_acquire_u32(a.rb_done + r) != qkv_epoch) {
+          if (++it > (1u << 22)) {
+            atomicOr(status, ST_WAIT_TIMEOUT);
+            break;
+          }
+          __nanosleep(64);
+        }
       }
+      __syncthreads();
+    }
+    // 4. the rows this step appended, and the queries
+#pragma unroll
+    for (int i = 0; i < kPer; ++i) {
+      const int pi = tid + i * kThreads, r = (pi % kRowPieces) / KP;
+      if (pi < 2 * kRowPieces && r < nj && j0 + r >= P) v[i] = load_row_piece(pi, r);
     }
 #pragma unroll
     for (int i = 0; i < kQPer; ++i) {
@@ -676,6 +713,7 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
     gp.ep.out_layer = k == 3 ? a.L - 1 : -1;
     gp.ep.h = a.act_f;
     gp.ep.h_ld = a.Kp_F;
+    gp.done_flags = k == 0 ? a.rb_done : nullptr;
     s_gp[k] = gp;
   }
   if (threadIdx.x == 32) {
@@ -692,6 +730,9 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
     av.qmax = kMaxTokens * (a.Hq / a.Hkv);
     av.part = a.attn_part;
     av.cnt = a.attn_cnt;
+    av.rb_done = a.rb_done;
+    av.rb_k0 = a.Hq * a.d / kRowsPerBlock;
+    av.rb_v0 = (a.Hq + a.Hkv) * a.d / kRowsPerBlock;
     int items = 0;
     for (int b = 0; b < sp->B; ++b) items += a.Hkv * n_chunks_of(sp->req_len[b], kAttnChunkMin);
     av.cs = items > (int)gridDim.x ? kChunk : kAttnChunkMin;
@@ -708,13 +749,12 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
     // attention block
     if (!skip) rmsnorm_cta(a.x, a.H, nrm, a.eps, a.ss, a.act_h, a.Kp_H, M);
     gemv(4 * l + 0, l);
-    grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
     if (!skip) {
       int total = 0;
       for (int b = 0; b < sp->B; ++b) total += a.Hkv * n_chunks_of(sp->req_len[b], s_av.cs);
       for (int item = blockIdx.x; item < total; item += gridDim.x) {
         int b, hk, c;
-        if (decode_item(sp, a.Hkv, s_av.cs, item, b, hk, c)) attn_item_cta<DPL>(&s_av, l, sp, b, hk, c, att_area);
+        if (decode_item(sp, a.Hkv, s_av.cs, item, b, hk, c)) attn_item_cta<DPL>(&s_av, l, sp, b, hk, c, att_area, a.epoch_base + 4 * l, a.status);
       }
       // merges, when CTAs take several items: (b, hk) goes to the CTA that
       // took its last chunk
@@ -762,7 +802,7 @@ cudaError_t setup_t() {
 
 }  // namespace
 
-int step_barriers(int n_layers) { return 5 * n_layers; }
+int step_barriers(int n_layers) { return 4 * n_layers; }
 
 size_t step_attention_part_floats(int B, int Hkv, int n_chunks, int G, int d) {
   return (size_t)B * Hkv * n_chunks * (kMaxTokens * G) * part_stride(d);
