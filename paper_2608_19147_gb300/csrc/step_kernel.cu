@@ -31,14 +31,14 @@ namespace {
 
 constexpr int kWarps = kCtaWarps;
 constexpr int kThreads = kWarps * 32;
-constexpr int kChunk = kAttnChunk;  // most cache entries per attention item (two per lane)
+constexpr int kChunk = kAttnChunk;  // most cache entries per attention item (four per lane)
 
 template <int GPU>
 struct StepSmem {
   static constexpr size_t kRing = (size_t)kWarps * kRingSlots * Geom<GPU>::kUnitBytes;
   static constexpr size_t kBars = (size_t)kWarps * kRingSlots * sizeof(uint64_t);
   // attention item area (AttnSmem)
-  static constexpr size_t kQ = 48 * 1024;
+  static constexpr size_t kQ = 96 * 1024;
   static constexpr size_t kFixed = kRing + kBars + kQ;  // + the op table (4L entries)
   static size_t total(int n_layers) { return kFixed + (size_t)4 * n_layers * sizeof(OpDesc); }
 };
@@ -271,9 +271,9 @@ __device__ __noinline__ void rmsnorm_cta(const float* x, int H, const uint16_t* 
 
 // ---------------------------------------------------------------------------
 // Attention.  Item = (request b, kv head hk, chunk c of cs entries); one CTA
-// per item, items dealt round-robin.  cs is 32 when that gives no more items
-// than CTAs (short caches: more parallel items), else 64 (long caches: fewer
-// rounds and merges).  Each item writes (max, sum of exp,
+// per item, items dealt round-robin.  cs is the smallest of 32, 64, 128 that
+// gives no more items than CTAs (short caches: more parallel items), else 128
+// (long caches: fewer rounds and merges).  Each item writes (max, sum of exp,
 // unnormalised output) per query (the request's new tokens x the kv head's
 // query heads).  With several items per CTA, after its items the CTA that
 // took the last chunk of (b, hk) waits for the chunk count and combines the
@@ -295,7 +295,7 @@ struct AttnView {
   int* cnt;  // finished chunks per (request, kv head)
   const unsigned* rb_done;  // q|k|v row-block flags the items wait for
   int rb_k0, rb_v0;         // first k and v row-block of the q|k|v projection
-  int cs;    // entries per item this step: kAttnChunkMin, or kChunk when that gives more items than CTAs
+  int cs;    // entries per item this step: 32, 64 or 128 (kChunk)
   int last_merges;  // at most one item per CTA: the CTA finishing the last chunk merges at once
   uint16_t* out;
   int out_ld;
@@ -575,26 +575,39 @@ __device__ __noinline__ void attn_item_cta(const AttnView* ap, int layer, const 
     __syncthreads();
     for (int qi = warp; qi < qn; qi += kWarps) {
       const float* qq = qsm + qi * d;
-      float s0, s1 = 0.f;
-      if (a.cs > 32) {
-        s0 = dot_q_k2(qq, Ks + lane * S::kKld, Ks + (lane + 32) * S::kKld, s1, KP);
+      // lane scores entries lane, lane + 32, ... (cs / 32 of them)
+      float sc[kChunk / 32];
+#pragma unroll
+      for (int k = 0; k < kChunk / 32; ++k) sc[k] = 0.f;
+      if (a.cs == 32) {
+        sc[0] = dot_q_k(qq, Ks + lane * S::kKld, KP);
       } else {
-        s0 = dot_q_k(qq, Ks + lane * S::kKld, KP);
+#pragma unroll
+        for (int k = 0; k < kChunk / 32; k += 2)
+          if (32 * k < a.cs) sc[k] = dot_q_k2(qq, Ks + (lane + 32 * k) * S::kKld, Ks + (lane + 32 * k + 32) * S::kKld, sc[k + 1], KP);
       }
       const int q = q0 + qi;
       const int lim = P + q / G;  // causal limit of this query's token
-      const bool vis0 = lane < nj && vis_s[lane] && j0 + lane <= lim;
-      const bool vis1 = lane + 32 < nj && vis_s[lane + 32] && j0 + lane + 32 <= lim;
-      const float v0 = vis0 ? s0 * scale : -INFINITY, v1 = vis1 ? s1 * scale : -INFINITY;
-      float mx = fmaxf(v0, v1);
+      float mx = -INFINITY;
+      bool vis[kChunk / 32];
+#pragma unroll
+      for (int k = 0; k < kChunk / 32; ++k) {
+        const int e = lane + 32 * k;
+        vis[k] = e < nj && vis_s[e] && j0 + e <= lim;
+        sc[k] = vis[k] ? sc[k] * scale : -INFINITY;
+        mx = fmaxf(mx, sc[k]);
+      }
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-      const float e0 = vis0 ? expf(v0 - mx) : 0.f, e1 = vis1 ? expf(v1 - mx) : 0.f;
-      float l = e0 + e1;
+      float l = 0.f;
+#pragma unroll
+      for (int k = 0; k < kChunk / 32; ++k) {
+        const float e = vis[k] ? expf(sc[k] - mx) : 0.f;
+        l += e;
+        if (32 * k < a.cs) ps[qi * kChunk + lane + 32 * k] = e;
+      }
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
-      ps[qi * kChunk + lane] = e0;
-      ps[qi * kChunk + lane + 32] = e1;
       if (lane == 0) {
         part[(size_t)q * part_stride(d)] = mx;
         part[(size_t)q * part_stride(d) + 1] = l;
@@ -735,7 +748,13 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
     av.rb_v0 = (a.Hq + a.Hkv) * a.d / kRowsPerBlock;
     int items = 0;
     for (int b = 0; b < sp->B; ++b) items += a.Hkv * n_chunks_of(sp->req_len[b], kAttnChunkMin);
-    av.cs = items > (int)gridDim.x ? kChunk : kAttnChunkMin;
+    // the smallest item size that needs one round of CTAs, else the largest
+    av.cs = kAttnChunkMin;
+    while (av.cs < kChunk && items > (int)gridDim.x) {
+      av.cs *= 2;
+      items = 0;
+      for (int b = 0; b < sp->B; ++b) items += a.Hkv * n_chunks_of(sp->req_len[b], av.cs);
+    }
     av.last_merges = items <= (int)gridDim.x;
     av.out = a.act_attn;
     av.out_ld = a.Kp_dq;
