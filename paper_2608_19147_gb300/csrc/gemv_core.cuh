@@ -326,6 +326,8 @@ __device__ __forceinline__ float epilogue_pair(const EpiArgs& e, const StepParam
 struct GemvPhase {
   const uint16_t* act;  // fp16 [M][act_ld]
   int act_ld, M;
+  uint32_t act_s;       // 0, or the shared-memory address of this CTA's own copy of the activations,
+  int act_s_ld;         // fp16 [M][act_s_ld], read instead of act
   bool skip;            // consume the weights but compute nothing (aborted step)
   float* partials;      // [n_cta * kCtaWarps][2][kPieceFloats] pieces of split row-blocks
   unsigned* flags;      // [n_cta * kCtaWarps][2] epoch of the piece last published in each slot
@@ -341,8 +343,8 @@ constexpr int kPieceFloats = kMaxTokens * kRowsPerBlock;
 
 // Loads the B fragments of input unit ku for tokens gid (and gid + 8).
 template <int NT>
-__device__ __forceinline__ void load_act(uint4 (&act)[NT][2][2], const uint16_t* actp, int act_ld, int M, bool skip,
-                                         int ku, int lane) {
+__device__ __forceinline__ void load_act(uint4 (&act)[NT][2][2], const uint16_t* actp, uint32_t acts, int act_ld,
+                                         int M, bool skip, int ku, int lane) {
   const int gid = lane >> 2, tig = lane & 3;
 #pragma unroll
   for (int nt = 0; nt < NT; ++nt) {
@@ -350,10 +352,19 @@ __device__ __forceinline__ void load_act(uint4 (&act)[NT][2][2], const uint16_t*
 #pragma unroll
     for (int kc = 0; kc < 2; ++kc)
 #pragma unroll
-      for (int h = 0; h < 2; ++h)
-        act[nt][kc][h] = (n < M && !skip) ? __ldcg(reinterpret_cast<const uint4*>(
-                                                actp + (size_t)n * act_ld + ku * kUnitK + kc * 64 + h * 32 + tig * 8))
-                                          : make_uint4(0, 0, 0, 0);
+      for (int h = 0; h < 2; ++h) {
+        const int off = n * act_ld + ku * kUnitK + kc * 64 + h * 32 + tig * 8;
+        uint4 v = make_uint4(0, 0, 0, 0);
+        if (n < M && !skip) {
+          if (acts)
+            asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+                         : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                         : "r"(acts + 2u * (uint32_t)off));
+          else
+            v = __ldcg(reinterpret_cast<const uint4*>(actp + off));
+        }
+        act[nt][kc][h] = v;
+      }
   }
 }
 
@@ -517,12 +528,13 @@ __device__ __noinline__ void gemv_phase(WarpStream<GPU>* ws_io, int op, const Ge
   const int T = ws.ops[op].n_rb * upr;
   const int g = ws.cta * kCtaWarps + ws.warp, nw = ws.n_cta * kCtaWarps;
   const uint16_t* actp = p.act;
-  const int act_ld = p.act_ld, M = p.M;
+  const uint32_t acts = p.act_s;
+  const int act_ld = acts ? p.act_s_ld : p.act_ld, M = p.M;
   const bool skip = p.skip;
   int rb = wb / upr;
   int ku = wb - rb * upr;
   uint4 nxt[NT][2][2];
-  load_act<NT>(nxt, actp, act_ld, M, skip, ku, lane);
+  load_act<NT>(nxt, actp, acts, act_ld, M, skip, ku, lane);
   for (int u = wb; u < we; ++rb) {
     const int seg_begin = u, rb_end = (rb + 1) * upr;
     const int seg_end = we < rb_end ? we : rb_end;
@@ -542,7 +554,7 @@ __device__ __noinline__ void gemv_phase(WarpStream<GPU>* ws_io, int op, const Ge
 #pragma unroll
           for (int h = 0; h < 2; ++h) cur[nt][kc][h] = nxt[nt][kc][h];
       if (++ku == upr) ku = 0;
-      if (u + 1 < we) load_act<NT>(nxt, actp, act_ld, M, skip, ku, lane);
+      if (u + 1 < we) load_act<NT>(nxt, actp, acts, act_ld, M, skip, ku, lane);
       const uint8_t* U = ws.acquire();
       if (!skip && !ws.timed_out) mma_unit<NT, GPU>(U, cur, tot, lane);
       ws.release(lane);

@@ -32,6 +32,8 @@ namespace {
 constexpr int kWarps = kCtaWarps;
 constexpr int kThreads = kWarps * 32;
 constexpr int kChunk = kAttnChunk;  // most cache entries per attention item (four per lane)
+constexpr bool kNormInSmem = true;   // normalised activations in shared memory when they fit
+constexpr bool kNormPrefetch = true; // RMSNorm: first x loads issued with the sums-of-squares loads
 
 template <int GPU>
 struct StepSmem {
@@ -61,6 +63,11 @@ __device__ __forceinline__ float2 h2f2(uint32_t u) {
   __half2 h;
   memcpy(&h, &u, sizeof(h));
   return __half22float2(h);
+}
+
+// two floats rounded to fp16 (to nearest even), lo in the low half
+__device__ __forceinline__ uint32_t pack_h2(float lo, float hi) {
+  return (uint32_t)f2h(lo) | ((uint32_t)f2h(hi) << 16);
 }
 
 __device__ __forceinline__ void red_release_add_s32(int* p, int v) {
@@ -230,19 +237,11 @@ __device__ __noinline__ void rmsnorm_cta(const float* x, int H, const uint16_t* 
   __shared__ float s_r[kMaxTokens];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int n_rb = (H + kRowsPerBlock - 1) / kRowsPerBlock;
-  for (int m = warp; m < M; m += kWarps) {
-    float t = 0.f;
-    for (int rb = lane; rb < n_rb; rb += 32) t += __ldcg(ss + rb * kMaxTokens + m);
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
-    if (lane == 0) s_r[m] = rsqrtf(t / H + eps);
-  }
-  __syncthreads();
   constexpr int kBatch = 4;  // float4 pieces per thread in flight
   const int H4 = H / 4, n4 = M * H4;
-  for (int i0 = tid; i0 < n4; i0 += kBatch * kThreads) {
-    float4 xv[kBatch];
-    uint2 wv[kBatch];
+  float4 xv[kBatch];
+  uint2 wv[kBatch];
+  auto load = [&](int i0) {
 #pragma unroll
     for (int j = 0; j < kBatch; ++j) {
       const int i = i0 + j * kThreads;
@@ -251,6 +250,8 @@ __device__ __noinline__ void rmsnorm_cta(const float* x, int H, const uint16_t* 
         wv[j] = *reinterpret_cast<const uint2*>(w + 4 * (i % H4));
       }
     }
+  };
+  auto store = [&](int i0) {
 #pragma unroll
     for (int j = 0; j < kBatch; ++j) {
       const int i = i0 + j * kThreads;
@@ -258,13 +259,27 @@ __device__ __noinline__ void rmsnorm_cta(const float* x, int H, const uint16_t* 
         const int m = i / H4, k = 4 * (i % H4);
         const float r = s_r[m];
         const float2 w01 = h2f2(wv[j].x), w23 = h2f2(wv[j].y);
-        uint16_t* o = out + (size_t)m * out_ld + k;
-        o[0] = f2h(xv[j].x * r * w01.x);
-        o[1] = f2h(xv[j].y * r * w01.y);
-        o[2] = f2h(xv[j].z * r * w23.x);
-        o[3] = f2h(xv[j].w * r * w23.y);
+        uint2 o;
+        o.x = pack_h2(xv[j].x * r * w01.x, xv[j].y * r * w01.y);
+        o.y = pack_h2(xv[j].z * r * w23.x, xv[j].w * r * w23.y);
+        *reinterpret_cast<uint2*>(out + (size_t)m * out_ld + k) = o;
       }
     }
+  };
+  // the first batch of x and weights is in flight with the sums of squares
+  if (kNormPrefetch) load(tid);
+  for (int m = warp; m < M; m += kWarps) {
+    float t = 0.f;
+    for (int rb = lane; rb < n_rb; rb += 32) t += __ldcg(ss + rb * kMaxTokens + m);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+    if (lane == 0) s_r[m] = rsqrtf(t / H + eps);
+  }
+  __syncthreads();
+  if (kNormPrefetch) store(tid);
+  for (int i0 = tid + (kNormPrefetch ? kBatch * kThreads : 0); i0 < n4; i0 += kBatch * kThreads) {
+    load(i0);
+    store(i0);
   }
   __syncthreads();
 }
@@ -702,12 +717,23 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
   const StepParams* sp = a.pro.sp;
   const bool skip = __ldcg(&sp->abort_step) != 0;
   const int M = a.pro.M;
+  // Each CTA normalises the whole hidden state for itself; when the M rows
+  // fit, it keeps them in the attention area (idle during the q|k|v and
+  // gate|up projections) and the projections read them from there.  Rows are
+  // padded by 32 halves so that the two token rows a fragment load touches in
+  // one phase fall on different banks.
+  const int xn_ld = a.H + 32;
+  const bool xn_smem = kNormInSmem && a.Kp_H == a.H && (size_t)M * xn_ld * 2 <= SS::kQ;
+  uint16_t* xn = xn_smem ? reinterpret_cast<uint16_t*>(att_area) : a.act_h;
+  const int xn_out_ld = xn_smem ? xn_ld : a.Kp_H;
   if (threadIdx.x < 4) {
     const int k = threadIdx.x;
     GemvPhase gp{};
     gp.act = k == 0 || k == 2 ? a.act_h : k == 1 ? a.act_attn : a.act_f;
     gp.act_ld = k == 0 || k == 2 ? a.Kp_H : k == 1 ? a.Kp_dq : a.Kp_F;
     gp.M = M;
+    gp.act_s = (k == 0 || k == 2) && xn_smem ? smem_addr(att_area) : 0u;
+    gp.act_s_ld = xn_ld;
     gp.skip = skip;
     gp.partials = a.partials;
     gp.flags = a.flags;
@@ -766,9 +792,10 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
   for (int l = 0; l < a.L; ++l) {
     const uint16_t* nrm = a.norms + (size_t)l * 2 * a.H;
     // attention block
-    if (!skip) rmsnorm_cta(a.x, a.H, nrm, a.eps, a.ss, a.act_h, a.Kp_H, M);
+    if (!skip) rmsnorm_cta(a.x, a.H, nrm, a.eps, a.ss, xn, xn_out_ld, M);
     gemv(4 * l + 0, l);
     if (!skip) {
+      if (xn_smem) __syncthreads();  // the attention items reuse the normalised rows' space
       int total = 0;
       for (int b = 0; b < sp->B; ++b) total += a.Hkv * n_chunks_of(sp->req_len[b], s_av.cs);
       for (int item = blockIdx.x; item < total; item += gridDim.x) {
@@ -788,7 +815,7 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
     gemv(4 * l + 1, l);
     grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
     // MLP block
-    if (!skip) rmsnorm_cta(a.x, a.H, nrm + a.H, a.eps, a.ss, a.act_h, a.Kp_H, M);
+    if (!skip) rmsnorm_cta(a.x, a.H, nrm + a.H, a.eps, a.ss, xn, xn_out_ld, M);
     gemv(4 * l + 2, l);
     grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
     gemv(4 * l + 3, l);
