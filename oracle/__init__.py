@@ -95,6 +95,7 @@ def _load():
             lib.or_step.argtypes = [vp, vp, vp, vp, vp, ip, vp, vp, ip, vp, ip, vp, vp]
             lib.or_step.restype = ip
             lib.or_logits.argtypes = [vp, ip, ip, vp, ip, dp, vp]
+            lib.or_head_top1.argtypes = [vp, ip, ip, vp, dp, ctypes.POINTER(_Matrix), ip, ip, ip, vp, vp, vp, vp]
             _lib = lib
     return _lib
 
@@ -188,6 +189,26 @@ def logits(h: np.ndarray, embedding: np.ndarray, eps: float) -> np.ndarray:
     out = np.empty((M, E.shape[0]), dtype=np.float64)
     _load().or_logits(_p(h), M, H, _p(E), E.shape[0], eps, _p(out))
     return out
+
+
+def head_top1(h16: np.ndarray, norm16: np.ndarray, w, eps: float, round_points: bool = True):
+    """LM head with the top-1 epilogue (Section 6.7): fp16 hidden rows
+    [M][H] -> (token [M] int32, p_max [M], margin [M], logits [M][V]), all
+    fp64 but the token; w is the [V][H] packed INT4 lm_head (.codes,
+    .scales, .zeros, .rows, .cols, .group)."""
+    h16 = np.ascontiguousarray(h16, dtype=np.uint16)
+    M, H = h16.shape
+    assert w.cols == H
+    V = w.rows
+    norm16 = np.ascontiguousarray(norm16, dtype=np.uint16)
+    tok = np.empty(M, np.int32)
+    p = np.empty(M, np.float64)
+    margin = np.empty(M, np.float64)
+    lg = np.empty((M, V), np.float64)
+    m = _matrix_struct(w)
+    _load().or_head_top1(_p(h16), M, H, _p(norm16), eps, ctypes.byref(m), V, w.group, int(round_points), _p(tok),
+                         _p(p), _p(margin), _p(lg))
+    return tok, p, margin, lg
 
 
 # ---------------------------------------------------------------------------

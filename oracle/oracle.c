@@ -26,6 +26,9 @@
  *    rotary tables): RMSNorm, q/k/v projections, rotate-half RoPE at
  *    theta^(-2i/d) frequencies, grouped-query softmax attention with scale
  *    1/sqrt(d), output projection + residual, RMSNorm, SwiGLU MLP + residual.
+ *  - The final stage's LM head with top-1 compression [Section 6.7]: final
+ *    RMSNorm, the INT4 lm_head projection to vocabulary logits, and only the
+ *    greedy token (argmax) with its softmax probability leave the stage.
  *
  * Precision: everything is fp64.  With round_points = 1 the result is
  * rounded to fp16 (round to nearest even) at the points where the W4A16 path
@@ -496,4 +499,51 @@ void or_logits(const double* h, int M, int H, const uint16_t* E, int V, double e
         }
     }
     free(hn);
+}
+
+/* ------------------------------------------------------------------------- */
+/* LM head of a final stage with the top-1 epilogue [Section 6.7]            */
+/* ------------------------------------------------------------------------- */
+
+/* For each fp16 hidden row h[t] (t < M):
+     x          = rmsnorm(h[t]) * w_norm, rounded to fp16 when round_points
+                  (the projection's 16-bit activation operand),
+     logits[v]  = sum_i W[v][i] * x[i]   (W the INT4 lm_head, [V][H]),
+     token[t]   = the v with the largest logit (the lowest such v on ties),
+     p_max[t]   = its softmax probability, 1 / sum_v exp(logits[v] - max),
+     margin[t]  = max minus the second largest logit (0 on a tie; for V = 1,
+                  +inf).
+   Only (token, p_max) are what the final stage sends back in the paper's
+   top-1 compression; margin is for tolerance gating in tests.  logits_out
+   (nullable) receives [M][V]. */
+void or_head_top1(const uint16_t* h16, int M, int H, const uint16_t* w_norm, double eps, const or_matrix* W, int V,
+                  int group, int round_points, int32_t* token, double* p_max, double* margin, double* logits_out) {
+    double* hx = (double*)malloc(sizeof(double) * (size_t)H);
+    double* x = (double*)malloc(sizeof(double) * (size_t)M * H);
+    double* lg = (double*)malloc(sizeof(double) * (size_t)M * V);
+    for (int t = 0; t < M; ++t) {
+        for (int i = 0; i < H; ++i) hx[i] = or_f16_to_f64(h16[(size_t)t * H + i]);
+        or_rmsnorm(hx, H, w_norm, eps, x + (size_t)t * H);
+        if (round_points)
+            for (int i = 0; i < H; ++i) x[(size_t)t * H + i] = or_round_f16(x[(size_t)t * H + i]);
+    }
+    or_gemv(W, V, H, group, x, M, lg);
+    for (int t = 0; t < M; ++t) {
+        const double* l = lg + (size_t)t * V;
+        int best = 0;
+        for (int v = 1; v < V; ++v)
+            if (l[v] > l[best]) best = v;
+        double second = -INFINITY;
+        for (int v = 0; v < V; ++v)
+            if (v != best && l[v] > second) second = l[v];
+        double den = 0.0;
+        for (int v = 0; v < V; ++v) den += exp(l[v] - l[best]);
+        token[t] = best;
+        p_max[t] = 1.0 / den;
+        margin[t] = l[best] - second;
+    }
+    if (logits_out) memcpy(logits_out, lg, sizeof(double) * (size_t)M * V);
+    free(hx);
+    free(x);
+    free(lg);
 }

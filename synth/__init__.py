@@ -180,6 +180,7 @@ def quant_matrix(rows: int, cols: int, group: int, sigma: float, *, seed: int, s
 MATRIX_NAMES = ("q", "k", "v", "o", "gate", "up", "down")
 
 TAG_WEIGHT, TAG_NORM, TAG_EMBED, TAG_KV, TAG_HIDDEN, TAG_TOKENS, TAG_ACCEPT, TAG_BEAM, TAG_LENGTHS, TAG_DRAFT = range(1, 11)
+TAG_HEAD = 11
 
 
 @dataclass(frozen=True)
@@ -265,6 +266,29 @@ def make_weights(shape: ShardShape, seed: int, threads: Optional[int] = None, n_
         sw.embedding = normal(shape.vocab * shape.hidden, seed=seed, stream=0, tag=TAG_EMBED,
                               dtype=np.uint16, threads=threads).reshape(shape.vocab, shape.hidden)
     return sw
+
+
+@dataclass
+class HeadWeights:
+    """The final stage's LM head: final RMSNorm weight and the [V][H] lm_head."""
+    hidden: int
+    vocab: int
+    group: int
+    lm_head: PackedMatrix          # [vocab][hidden]
+    norm: np.ndarray               # uint16 fp16 bits [hidden]
+    rms_eps: float = 1e-5
+
+    def packed_bytes(self) -> int:
+        return self.lm_head.nbytes()
+
+
+def make_head(hidden: int, vocab: int, group: int, seed: int, sigma: float = 0.02, rms_eps: float = 1e-5,
+              threads: Optional[int] = None) -> HeadWeights:
+    """Seeded LM head: lm_head ~ N(0, sigma^2) quantised to uint4 like the
+    layer matrices; final norm weight fp16(1 + 0.1 N(0,1))."""
+    w = quant_matrix(vocab, hidden, group, sigma, seed=seed, stream=0, tag=TAG_HEAD, threads=threads)
+    norm = normal(hidden, seed=seed, stream=1, tag=TAG_HEAD, mean=1.0, sigma=0.1, dtype=np.uint16)
+    return HeadWeights(hidden, vocab, group, w, norm, rms_eps)
 
 
 # ---------------------------------------------------------------------------
