@@ -1,4 +1,5 @@
-"""Python binding of libshard (include/shard.h, include/shard_debug.h).
+"""Python binding of libshard (include/shard.h, include/shard_debug.h,
+include/head.h).
 
 Argument marshalling only: every function forwards to the C ABI function of
 the same name, which runs the work in the library's CUDA kernels.  Device
@@ -27,7 +28,8 @@ OP_QKV, OP_O, OP_GU, OP_DOWN = 0, 1, 2, 3
 EXPORTS = ("shard_create", "shard_destroy", "kv_state_alloc", "kv_state_free", "kv_state_reset", "kv_state_load",
            "kv_state_read", "kv_state_length", "kv_trim", "shard_step", "shard_step_host", "shard_sync_status",
            "shard_last_error", "shard_debug_op_info", "shard_debug_unpack", "shard_debug_gemv",
-           "shard_debug_phase_times", "shard_gemv_noalloc")
+           "shard_debug_phase_times", "shard_gemv_noalloc", "head_create", "head_destroy", "head_top1",
+           "head_top1_host", "head_debug_logits")
 # per layer, between grid barriers: RMSNorm + q|k|v + attention, o, RMSNorm + gate|up, down
 PHASES = ("qkv_attention", "o", "gate_up", "down")
 
@@ -55,6 +57,15 @@ class shard_layer_host(ctypes.Structure):
 
 class shard_weights_host(ctypes.Structure):
     _fields_ = [("layers", ctypes.POINTER(shard_layer_host)), ("embedding", ctypes.c_void_p)]
+
+
+class head_config(ctypes.Structure):
+    _fields_ = [("hidden", ctypes.c_int32), ("vocab", ctypes.c_int32), ("group", ctypes.c_int32),
+                ("reserved", ctypes.c_int32), ("rms_eps", ctypes.c_double)]
+
+
+class head_weights_host(ctypes.Structure):
+    _fields_ = [("lm_head", shard_matrix_host), ("norm", ctypes.c_void_p)]
 
 
 _lib = None
@@ -90,6 +101,11 @@ def load_library(path: str = LIB_PATH):
         "shard_debug_gemv": ([vp, ip, ip, vp, ip, vp, ip, vp], ip),
         "shard_gemv_noalloc": ([vp, ip, ip, vp, ip, vp, ip, vp], ip),
         "shard_debug_phase_times": ([vp, ctypes.POINTER(ctypes.c_double), ip], ip),
+        "head_create": ([ctypes.POINTER(head_config), ctypes.POINTER(head_weights_host), ctypes.POINTER(vp)], ip),
+        "head_destroy": ([vp], ip),
+        "head_top1": ([vp, vp, ip, vp, vp, vp], ip),
+        "head_top1_host": ([vp, vp, ip, vp, vp, vp], ip),
+        "head_debug_logits": ([vp, vp, ip, vp, ip, vp], ip),
     }
     for name, (args, res) in sig.items():
         f = getattr(lib, name)
@@ -243,3 +259,43 @@ def shard_gemv_noalloc(shard: int, layer: int, op: int, x: int, M: int, y: int, 
     """One projection with the library's fixed scratch array (no device allocation)."""
     rc = load_library().shard_gemv_noalloc(shard, layer, op, x, M, y, y_ld, stream or None)
     return _check(rc) if check else rc
+
+
+# ---------------------------------------------------------------------------
+# LM head with the top-1 epilogue (include/head.h)
+# ---------------------------------------------------------------------------
+
+def head_create(hidden: int, vocab: int, group: int, rms_eps: float, lm_head, norm: np.ndarray) -> int:
+    """lm_head: packed [vocab][hidden] matrix (.codes/.scales/.zeros arrays);
+    norm: fp16 bits [hidden]."""
+    cfg = head_config(hidden, vocab, group, 0, float(rms_eps))
+    w = head_weights_host(shard_matrix_host(_np(lm_head.codes, np.uint8), _np(lm_head.scales, np.uint16),
+                                            _np(lm_head.zeros, np.uint8)), _np(norm, np.uint16))
+    out = ctypes.c_void_p()
+    _check(load_library().head_create(ctypes.byref(cfg), ctypes.byref(w), ctypes.byref(out)))
+    return out.value
+
+
+def head_destroy(head: int) -> None:
+    _check(load_library().head_destroy(head))
+
+
+def head_top1(head: int, hidden: int, M: int, token: int, p_max: Optional[int], stream: int = 0,
+              check: bool = True) -> int:
+    """Device pointers as ints: hidden fp16 [M][H], token int32 [M], p_max fp32 [M] (or None)."""
+    rc = load_library().head_top1(head, hidden, M, token, p_max or None, stream or None)
+    return _check(rc) if check else rc
+
+
+def head_top1_host(head: int, hidden: np.ndarray, stream: int = 0):
+    """Host fp16 bits [M][H] -> (token int32 [M], p_max float32 [M])."""
+    hidden = np.ascontiguousarray(hidden, dtype=np.uint16)
+    M = hidden.shape[0]
+    tok = np.empty(M, np.int32)
+    p = np.empty(M, np.float32)
+    _check(load_library().head_top1_host(head, _np(hidden), M, _np(tok), _np(p), stream or None))
+    return tok, p
+
+
+def head_debug_logits(head: int, hidden: int, M: int, logits: int, ld: int, stream: int = 0) -> None:
+    _check(load_library().head_debug_logits(head, hidden, M, logits, ld, stream or None))

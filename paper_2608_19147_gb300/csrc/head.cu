@@ -1,0 +1,476 @@
+// The final stage's LM head with the top-1 epilogue (include/head.h,
+// Section 6.7): per hidden row, the final RMSNorm, the INT4 lm_head
+// projection to fp32 logits and a top-1 reduction to (greedy token, its
+// softmax probability).  Three kernels on the caller's stream:
+//   head_norm_kernel  one CTA per row: fp16 hidden -> fp16 normalised row in
+//                     the zero-padded activation buffer;
+//   gemv_kernel       the shard's W4A16 projection (gemv_core.cuh) with the
+//                     plain store epilogue, launched with programmatic
+//                     dependent launch so its weight ring fills while the
+//                     norm finishes;
+//   head_top1_kernel  (chunk, row) CTAs: each reduces a chunk of the row's
+//                     logits to (max, lowest argmax, sum of exp relative to
+//                     the max); the CTA that finishes a row last combines the
+//                     chunks in chunk order (a fixed order: deterministic).
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <vector>
+
+#include "../../include/head.h"
+#include "common.cuh"
+
+namespace shard {
+// Sets the calling thread's last error (shard_api.cu) and returns code.
+int shard_fail_msg(int code, const char* msg);
+}  // namespace shard
+
+using namespace shard;
+
+namespace {
+
+constexpr int kNormThreads = 256;
+constexpr int kTopThreads = 256;
+constexpr int kTopChunkMin = 512;  // logits per top-1 CTA, at least
+
+int fail(int code, const char* fmt, ...) __attribute__((format(printf, 2, 3)));
+int fail(int code, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  return shard_fail_msg(code, buf);
+}
+
+#define HEAD_CUDA_TRY(expr)                                                                         \
+  do {                                                                                              \
+    cudaError_t _e = (expr);                                                                        \
+    if (_e != cudaSuccess)                                                                          \
+      return fail(_e == cudaErrorMemoryAllocation ? SHARD_ENOMEM : SHARD_ECUDA, "%s: %s (%s:%d)", #expr, \
+                  cudaGetErrorString(_e), __FILE__, __LINE__);                                      \
+  } while (0)
+
+__device__ __forceinline__ float block_sum(float v, float* red) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  if (warp == 0) {
+    float t = lane < nw ? red[lane] : 0.f;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+    if (lane == 0) red[0] = t;
+  }
+  __syncthreads();
+  const float r = red[0];
+  __syncthreads();
+  return r;
+}
+
+// x = hidden[m] / sqrt(mean(hidden[m]^2) + eps) * w, rounded to fp16.
+__global__ void __launch_bounds__(kNormThreads) head_norm_kernel(const uint16_t* __restrict__ hidden, int H,
+                                                                 const uint16_t* __restrict__ w, float eps,
+                                                                 uint16_t* __restrict__ act, int act_ld) {
+  __shared__ float red[kNormThreads / 32];
+  pdl_launch_dependents();  // the projection may start streaming its weights
+  const int m = blockIdx.x;
+  const uint16_t* h = hidden + (size_t)m * H;
+  float ss = 0.f;
+  for (int i = threadIdx.x; i < H; i += blockDim.x) {
+    const float v = h2f(h[i]);
+    ss += v * v;
+  }
+  const float r = rsqrtf(block_sum(ss, red) / H + eps);
+  for (int i = threadIdx.x; i < H; i += blockDim.x) act[(size_t)m * act_ld + i] = f2h(h2f(h[i]) * r * h2f(w[i]));
+}
+
+struct Top1Part {
+  float max, sum;  // the chunk's largest logit; sum of exp(logit - max) over the chunk
+  int idx, pad;    // the lowest id holding max
+};
+
+// a then b, where every id of a is below every id of b
+__device__ __forceinline__ void top1_merge(float& m, float& s, int& i, float m2, float s2, int i2) {
+  if (m2 > m) {
+    s = s * expf(m - m2) + s2;
+    m = m2;
+    i = i2;
+  } else {
+    s = s + s2 * expf(m2 - m);
+  }
+}
+
+// (max, lowest argmax) over a warp, then sum of exp relative to the max.
+__device__ __forceinline__ void warp_max_idx(float& m, int& i) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float m2 = __shfl_xor_sync(0xffffffffu, m, o);
+    const int i2 = __shfl_xor_sync(0xffffffffu, i, o);
+    if (m2 > m || (m2 == m && i2 < i)) {
+      m = m2;
+      i = i2;
+    }
+  }
+}
+
+__global__ void __launch_bounds__(kTopThreads) head_top1_kernel(const float* __restrict__ logits, int ld, int V,
+                                                                int chunk, Top1Part* __restrict__ parts,
+                                                                int* __restrict__ done, int32_t* __restrict__ token,
+                                                                float* __restrict__ p_max) {
+  __shared__ float s_m[kTopThreads / 32];
+  __shared__ int s_i[kTopThreads / 32];
+  __shared__ float red[kTopThreads / 32];
+  __shared__ int s_last;
+  pdl_wait();  // the projection's logits
+  const int c = blockIdx.x, m = blockIdx.y, nc = gridDim.x;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const float* l = logits + (size_t)m * ld;
+  const int b = c * chunk, e = min(V, b + chunk);
+  // 1. the chunk's max and its lowest id
+  float mx = -INFINITY;
+  int ix = 0x7fffffff;
+  for (int v = b + threadIdx.x; v < e; v += blockDim.x) {
+    const float x = __ldcg(l + v);
+    if (x > mx) {  // ids rise along a thread's walk: the first max is the lowest
+      mx = x;
+      ix = v;
+    }
+  }
+  warp_max_idx(mx, ix);
+  if (lane == 0) {
+    s_m[warp] = mx;
+    s_i[warp] = ix;
+  }
+  __syncthreads();
+  if (warp == 0) {
+    mx = lane < (kTopThreads / 32) ? s_m[lane] : -INFINITY;
+    ix = lane < (kTopThreads / 32) ? s_i[lane] : 0x7fffffff;
+    warp_max_idx(mx, ix);
+    if (lane == 0) {
+      s_m[0] = mx;
+      s_i[0] = ix;
+    }
+  }
+  __syncthreads();
+  const float cm = s_m[0];
+  // 2. sum of exp(logit - chunk max)
+  float s = 0.f;
+  for (int v = b + threadIdx.x; v < e; v += blockDim.x) s += expf(__ldcg(l + v) - cm);
+  s = block_sum(s, red);
+  if (threadIdx.x == 0) {
+    parts[(size_t)m * nc + c] = Top1Part{cm, s, s_i[0], 0};
+    __threadfence();
+    s_last = atomicAdd(done + m, 1) == nc - 1;
+  }
+  __syncthreads();
+  if (!s_last) return;
+  // 3. the row's last CTA combines the chunks (warp 0): lane L folds chunks
+  // L, L + 32, ... in order, then a butterfly in which both partners combine
+  // the lower lane's part first -- a fixed order, so every lane ends with the
+  // same bits whatever the arrival order of the CTAs
+  __threadfence();
+  if (warp != 0) return;
+  float gm = -INFINITY, gs = 0.f;
+  int gi = 0x7fffffff;
+  for (int k = lane; k < nc; k += 32) {
+    const float pm = __ldcg(&parts[(size_t)m * nc + k].max);
+    const float ps = __ldcg(&parts[(size_t)m * nc + k].sum);
+    const int pi = __ldcg(&parts[(size_t)m * nc + k].idx);
+    if (gs == 0.f && gm == -INFINITY) {
+      gm = pm;
+      gs = ps;
+      gi = pi;
+    } else {
+      top1_merge(gm, gs, gi, pm, ps, pi);
+    }
+  }
+  // butterfly over lanes: the id ranges of two lanes interleave, so the
+  // merge keeps the lowest id among equal maxima explicitly
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const float m2 = __shfl_xor_sync(0xffffffffu, gm, o);
+    const float s2 = __shfl_xor_sync(0xffffffffu, gs, o);
+    const int i2 = __shfl_xor_sync(0xffffffffu, gi, o);
+    const bool lo = (lane & o) == 0;  // combine in a lane-symmetric order: lower lane's part first
+    float am = lo ? gm : m2, as = lo ? gs : s2, bm = lo ? m2 : gm, bs = lo ? s2 : gs;
+    int ai = lo ? gi : i2, bi = lo ? i2 : gi;
+    if (bs == 0.f && bm == -INFINITY) {
+      // b is empty
+    } else if (as == 0.f && am == -INFINITY) {
+      am = bm;
+      as = bs;
+      ai = bi;
+    } else {
+      const float nm = fmaxf(am, bm);
+      as = as * expf(am - nm) + bs * expf(bm - nm);
+      ai = am > bm ? ai : (bm > am ? bi : min(ai, bi));
+      am = nm;
+    }
+    gm = am;
+    gs = as;
+    gi = ai;
+  }
+  if (lane == 0) {
+    token[m] = gi;
+    if (p_max) p_max[m] = 1.f / gs;
+    done[m] = 0;  // ready for the next call
+  }
+}
+
+}  // namespace
+
+struct head_s {
+  int device = 0;
+  head_config cfg{};
+  int num_sms = 0;
+  PackedOp op;
+  uint8_t* units = nullptr;
+  uint16_t* norm = nullptr;
+  uint16_t* act = nullptr;      // fp16 [16][Kp], padding columns zero
+  float* logits = nullptr;      // fp32 [16][ld]
+  int ld = 0;
+  float* partials = nullptr;    // projection pieces
+  unsigned* flags = nullptr;    // projection piece flags
+  unsigned epoch = 1;
+  int* status = nullptr;
+  int* status_host = nullptr;   // pinned mirror, copied after each call
+  Top1Part* parts = nullptr;    // [16][max chunks]
+  int* done = nullptr;          // [16] chunk arrivals per row (self-resetting)
+  int max_chunks = 0;
+  int grid[3] = {0, 0, 0};
+  uint16_t* hidden_dev = nullptr;  // head_top1_host staging
+  int32_t* token_dev = nullptr;
+  float* p_dev = nullptr;
+};
+
+namespace {
+
+void destroy(head_s* h) {
+  if (!h) return;
+  cudaSetDevice(h->device);
+  cudaFree(h->units);
+  cudaFree(h->norm);
+  cudaFree(h->act);
+  cudaFree(h->logits);
+  cudaFree(h->partials);
+  cudaFree(h->flags);
+  cudaFree(h->status);
+  if (h->status_host) cudaFreeHost(h->status_host);
+  cudaFree(h->parts);
+  cudaFree(h->done);
+  cudaFree(h->hidden_dev);
+  cudaFree(h->token_dev);
+  cudaFree(h->p_dev);
+  delete h;
+}
+
+int chunk_of(const head_s* h, int M, int* n_chunks) {
+  // about two CTAs per SM over the M rows, at least kTopChunkMin logits each
+  const int V = h->cfg.vocab;
+  int nc = std::max(1, (2 * h->num_sms) / M);
+  nc = std::min(nc, std::max(1, (V + kTopChunkMin - 1) / kTopChunkMin));
+  nc = std::min(nc, h->max_chunks);
+  const int chunk = (V + nc - 1) / nc;
+  *n_chunks = (V + chunk - 1) / chunk;
+  return chunk;
+}
+
+unsigned next_epoch(head_s* h) {
+  if (h->epoch >= 0xFFFFFFF0u) {  // wrap-around: no stale flag may match a reused epoch
+    cudaDeviceSynchronize();
+    cudaMemset(h->flags, 0, sizeof(unsigned) * gemv_flags_count(h->grid[0]));
+    cudaDeviceSynchronize();
+    h->epoch = 1;
+  }
+  return h->epoch++;
+}
+
+// norm -> projection -> top-1 (logits only, when token == nullptr)
+int run(head_s* h, const uint16_t* hidden, int M, int32_t* token, float* p_max, float* logits, int ld,
+        cudaStream_t s) {
+  const int bits = *reinterpret_cast<volatile int*>(h->status_host);
+  if (bits) {
+    *reinterpret_cast<volatile int*>(h->status_host) = 0;
+    return fail(SHARD_ECUDA, "an earlier head call reported a device wait timeout");
+  }
+  const head_config& c = h->cfg;
+  head_norm_kernel<<<M, kNormThreads, 0, s>>>(hidden, c.hidden, h->norm, (float)c.rms_eps, h->act, h->op.Kp);
+  HEAD_CUDA_TRY(cudaGetLastError());
+  GemvArgs g{};
+  g.units = h->op.units;
+  g.n_rb = h->op.n_rb;
+  g.upr = h->op.upr;
+  g.act = h->act;
+  g.act_ld = h->op.Kp;
+  g.M = M;
+  g.sp = nullptr;
+  g.partials = h->partials;
+  g.flags = h->flags;
+  g.epoch = next_epoch(h);
+  g.status = h->status;
+  g.ep.kind = EPI_STORE;
+  g.ep.dims = h->op.dims;
+  g.ep.y = logits;
+  g.ep.y_ld = ld;
+  const int nt = M <= 8 ? 1 : 2;
+  HEAD_CUDA_TRY(launch_gemv(g, nt, c.group, std::min<long long>(h->grid[nt], (long long)h->op.n_rb * h->op.upr), s,
+                            true));
+  if (token) {
+    int nc = 0;
+    const int chunk = chunk_of(h, M, &nc);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(nc, M);
+    cfg.blockDim = dim3(kTopThreads);
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    HEAD_CUDA_TRY(cudaLaunchKernelEx(&cfg, head_top1_kernel, (const float*)logits, ld, c.vocab, chunk, h->parts,
+                                     h->done, token, p_max));
+  }
+  HEAD_CUDA_TRY(cudaMemcpyAsync(h->status_host, h->status, sizeof(int), cudaMemcpyDeviceToHost, s));
+  return SHARD_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int head_create(const head_config* cfg, const head_weights_host* w, head_t* out) {
+  if (!cfg || !w || !out) return fail(SHARD_EINVAL, "head_create: null argument");
+  *out = nullptr;
+  const head_config c = *cfg;
+  if (c.hidden < 1 || c.vocab < 1 || !(c.rms_eps >= 0.0))
+    return fail(SHARD_EINVAL, "head_create: hidden %d / vocab %d / rms_eps out of range", c.hidden, c.vocab);
+  if (c.group != 32 && c.group != 64 && c.group != 128)
+    return fail(SHARD_EUNSUPPORTED, "head_create: group %d (supported: 32, 64, 128)", c.group);
+  if (!w->lm_head.codes || !w->lm_head.scales || !w->lm_head.zeros || !w->norm)
+    return fail(SHARD_EINVAL, "head_create: null weight pointer");
+  head_s* h = new head_s();
+  h->cfg = c;
+  auto bail = [&](int rc) {
+    destroy(h);
+    return rc;
+  };
+  int rc;
+  if ((rc = [&]() -> int {
+         HEAD_CUDA_TRY(cudaGetDevice(&h->device));
+         HEAD_CUDA_TRY(cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, h->device));
+         HEAD_CUDA_TRY(gemv_setup());
+         PackedOp& op = h->op;
+         op.rows = c.vocab;
+         op.K = c.hidden;
+         op.Kp = (c.hidden + kUnitK - 1) / kUnitK * kUnitK;
+         op.n_rb = (c.vocab + kRowsPerBlock - 1) / kRowsPerBlock;
+         op.upr = op.Kp / kUnitK;
+         op.unit_bytes = unit_bytes_for_group(c.group);
+         op.group = c.group;
+         op.bytes = (size_t)op.n_rb * op.upr * op.unit_bytes;
+         op.dims = OpDims{OP_O, 0, 0, 0, 0, c.vocab};  // natural row order, rows [0, vocab)
+         for (int nt = 1; nt <= 2; ++nt) h->grid[nt] = gemv_grid(nt, h->num_sms);
+         h->grid[0] = std::max(h->grid[1], h->grid[2]);
+         if (((uint64_t)op.n_rb * op.upr + 1) * ((uint64_t)h->grid[0] * gemv_warps_per_cta()) >= (1ull << 32))
+           return fail(SHARD_EUNSUPPORTED, "head_create: too many weight units for this GPU's warp count");
+         HEAD_CUDA_TRY(cudaMalloc(&h->units, op.bytes));
+         op.units = h->units;
+         // upload the packed matrix and repack it into the unit stream
+         const int G = (c.hidden + c.group - 1) / c.group;
+         const size_t cb = (size_t)(c.hidden + 1) / 2 * c.vocab, sb = (size_t)G * 2 * c.vocab,
+                      zb = (size_t)(G + 1) / 2 * c.vocab;
+         uint8_t* src = nullptr;
+         int* rowmap = nullptr;
+         HEAD_CUDA_TRY(cudaMalloc(&src, cb + sb + zb + 3 * 256));
+         const size_t so = (cb + 255) / 256 * 256, zo = so + (sb + 255) / 256 * 256;
+         cudaError_t e = cudaMemcpy(src, w->lm_head.codes, cb, cudaMemcpyHostToDevice);
+         if (e == cudaSuccess) e = cudaMemcpy(src + so, w->lm_head.scales, sb, cudaMemcpyHostToDevice);
+         if (e == cudaSuccess) e = cudaMemcpy(src + zo, w->lm_head.zeros, zb, cudaMemcpyHostToDevice);
+         std::vector<int> rm((size_t)op.n_rb * kRowsPerBlock, -1);
+         for (int r = 0; r < c.vocab; ++r) rm[r] = r;
+         if (e == cudaSuccess) e = cudaMalloc(&rowmap, sizeof(int) * rm.size());
+         if (e == cudaSuccess) e = cudaMemcpy(rowmap, rm.data(), sizeof(int) * rm.size(), cudaMemcpyHostToDevice);
+         if (e == cudaSuccess) {
+           RepackSrc rs{};
+           rs.codes[0] = src;
+           rs.scales[0] = reinterpret_cast<const uint16_t*>(src + so);
+           rs.zeros[0] = src + zo;
+           rs.rows[0] = c.vocab;
+           e = launch_repack(op, rowmap, rs, nullptr);
+         }
+         if (e == cudaSuccess) e = cudaDeviceSynchronize();
+         cudaFree(src);
+         cudaFree(rowmap);
+         HEAD_CUDA_TRY(e);
+         HEAD_CUDA_TRY(cudaMalloc(&h->norm, sizeof(uint16_t) * c.hidden));
+         HEAD_CUDA_TRY(cudaMemcpy(h->norm, w->norm, sizeof(uint16_t) * c.hidden, cudaMemcpyHostToDevice));
+         HEAD_CUDA_TRY(cudaMalloc(&h->act, sizeof(uint16_t) * kMaxTokens * op.Kp));
+         HEAD_CUDA_TRY(cudaMemset(h->act, 0, sizeof(uint16_t) * kMaxTokens * op.Kp));
+         h->ld = (c.vocab + 3) / 4 * 4;
+         HEAD_CUDA_TRY(cudaMalloc(&h->logits, sizeof(float) * kMaxTokens * h->ld));
+         HEAD_CUDA_TRY(cudaMalloc(&h->partials, sizeof(float) * gemv_partials_floats(h->grid[0])));
+         HEAD_CUDA_TRY(cudaMalloc(&h->flags, sizeof(unsigned) * gemv_flags_count(h->grid[0])));
+         HEAD_CUDA_TRY(cudaMemset(h->flags, 0, sizeof(unsigned) * gemv_flags_count(h->grid[0])));
+         HEAD_CUDA_TRY(cudaMalloc(&h->status, sizeof(int)));
+         HEAD_CUDA_TRY(cudaMemset(h->status, 0, sizeof(int)));
+         HEAD_CUDA_TRY(cudaHostAlloc(&h->status_host, sizeof(int), cudaHostAllocDefault));
+         *h->status_host = 0;
+         h->max_chunks = 2 * h->num_sms;
+         HEAD_CUDA_TRY(cudaMalloc(&h->parts, sizeof(Top1Part) * kMaxTokens * h->max_chunks));
+         HEAD_CUDA_TRY(cudaMalloc(&h->done, sizeof(int) * kMaxTokens));
+         HEAD_CUDA_TRY(cudaMemset(h->done, 0, sizeof(int) * kMaxTokens));
+         HEAD_CUDA_TRY(cudaMalloc(&h->hidden_dev, sizeof(uint16_t) * kMaxTokens * c.hidden));
+         HEAD_CUDA_TRY(cudaMalloc(&h->token_dev, sizeof(int32_t) * kMaxTokens));
+         HEAD_CUDA_TRY(cudaMalloc(&h->p_dev, sizeof(float) * kMaxTokens));
+         return SHARD_OK;
+       }()) != SHARD_OK)
+    return bail(rc);
+  *out = h;
+  return SHARD_OK;
+}
+
+int head_destroy(head_t h) {
+  if (!h) return fail(SHARD_EINVAL, "head_destroy: null head");
+  destroy(h);
+  return SHARD_OK;
+}
+
+int head_top1(head_t h, const uint16_t* hidden, int M, int32_t* token, float* p_max, void* cuda_stream) {
+  if (!h || !hidden || !token) return fail(SHARD_EINVAL, "head_top1: null argument");
+  if (M < 1 || M > SHARD_MAX_TOKENS) return fail(SHARD_EINVAL, "head_top1: M = %d outside [1, %d]", M, SHARD_MAX_TOKENS);
+  HEAD_CUDA_TRY(cudaSetDevice(h->device));
+  return run(h, hidden, M, token, p_max, h->logits, h->ld, static_cast<cudaStream_t>(cuda_stream));
+}
+
+int head_top1_host(head_t h, const uint16_t* hidden, int M, int32_t* token, float* p_max, void* cuda_stream) {
+  if (!h || !hidden || !token) return fail(SHARD_EINVAL, "head_top1_host: null argument");
+  if (M < 1 || M > SHARD_MAX_TOKENS)
+    return fail(SHARD_EINVAL, "head_top1_host: M = %d outside [1, %d]", M, SHARD_MAX_TOKENS);
+  HEAD_CUDA_TRY(cudaSetDevice(h->device));
+  cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+  HEAD_CUDA_TRY(cudaMemcpyAsync(h->hidden_dev, hidden, sizeof(uint16_t) * M * h->cfg.hidden, cudaMemcpyHostToDevice, s));
+  int rc = run(h, h->hidden_dev, M, h->token_dev, p_max ? h->p_dev : nullptr, h->logits, h->ld, s);
+  if (rc) return rc;
+  HEAD_CUDA_TRY(cudaMemcpyAsync(token, h->token_dev, sizeof(int32_t) * M, cudaMemcpyDeviceToHost, s));
+  if (p_max) HEAD_CUDA_TRY(cudaMemcpyAsync(p_max, h->p_dev, sizeof(float) * M, cudaMemcpyDeviceToHost, s));
+  HEAD_CUDA_TRY(cudaStreamSynchronize(s));
+  const int bits = *reinterpret_cast<volatile int*>(h->status_host);
+  if (bits) {
+    *reinterpret_cast<volatile int*>(h->status_host) = 0;
+    return fail(SHARD_ECUDA, "head_top1_host: a device wait timed out");
+  }
+  return SHARD_OK;
+}
+
+int head_debug_logits(head_t h, const uint16_t* hidden, int M, float* logits, int ld, void* cuda_stream) {
+  if (!h || !hidden || !logits) return fail(SHARD_EINVAL, "head_debug_logits: null argument");
+  if (M < 1 || M > SHARD_MAX_TOKENS) return fail(SHARD_EINVAL, "head_debug_logits: M = %d out of range", M);
+  if (ld < h->cfg.vocab) return fail(SHARD_EINVAL, "head_debug_logits: ld %d < vocab %d", ld, h->cfg.vocab);
+  HEAD_CUDA_TRY(cudaSetDevice(h->device));
+  return run(h, hidden, M, nullptr, nullptr, logits, ld, static_cast<cudaStream_t>(cuda_stream));
+}
+
+}  // extern "C"

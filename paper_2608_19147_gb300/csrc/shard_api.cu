@@ -883,6 +883,7 @@ struct NoAllocView {
 };
 
 int shard_noalloc_fail(int code, const char* msg) { return fail(code, "%s", msg); }
+int shard_fail_msg(int code, const char* msg) { return fail(code, "%s", msg); }
 
 int shard_noalloc_view(shard_t sh, int layer, int op, NoAllocView* v) {
   if (!sh || !v) return fail(SHARD_EINVAL, "shard_gemv_noalloc: null shard");

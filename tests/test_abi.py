@@ -14,7 +14,7 @@ ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 def _declared():
     names = set()
-    for h in ("shard.h", "shard_debug.h"):
+    for h in ("shard.h", "shard_debug.h", "head.h"):
         src = open(os.path.join(ROOT, "include", h)).read()
         src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
         for m in re.finditer(r"^\s*(?:const\s+)?\w+\**\s+\**(\w+)\s*\(", src, flags=re.M):
@@ -47,4 +47,7 @@ def test_no_device_call_needed_for_errors(lib):
     # argument validation happens on the host before any CUDA call
     lib.shard_destroy.argtypes = [ctypes.c_void_p]
     assert lib.shard_destroy(None) == pkg.SHARD_EINVAL
+    assert "null" in pkg.shard_last_error()
+    lib.head_destroy.argtypes = [ctypes.c_void_p]
+    assert lib.head_destroy(None) == pkg.SHARD_EINVAL
     assert "null" in pkg.shard_last_error()
