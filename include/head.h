@@ -67,7 +67,9 @@ int head_destroy(head_t head);
  *   token   dev int32 [M]: the greedy token of each row
  *   p_max   dev fp32 [M]: its softmax probability, or NULL
  * Does not synchronise.  Errors: EINVAL (M out of range, null hidden or
- * token), ECUDA. */
+ * token), ECUDA.  A bounded device wait of the projection that gave up
+ * (never expected) makes every row's token -1 and p_max NaN;
+ * head_top1_host turns that into ECUDA. */
 int head_top1(head_t head, const uint16_t* hidden, int M, int32_t* token, float* p_max, void* cuda_stream);
 
 /* head_top1 with host buffers: copies hidden (host fp16 [M][hidden]) to the

@@ -7,13 +7,18 @@
 namespace shard {
 namespace {
 
-constexpr int kW = kCtaWarps;  // warps per CTA
+constexpr int kW = kGemvWarps;  // warps per CTA
 constexpr int kCtasPerSm = 1;
 
 template <int NT, int GPU>
 constexpr size_t smem_bytes() {
-  return (size_t)kW * kRingSlots * Geom<GPU>::kUnitBytes + (size_t)kW * kRingSlots * sizeof(uint64_t);
+  return (size_t)kW * Geom<GPU>::kGemvSlots * Geom<GPU>::kUnitBytes +
+         (size_t)kW * Geom<GPU>::kGemvSlots * sizeof(uint64_t);
 }
+
+// 227 KB per CTA, less a margin for the kernel's static shared memory
+static_assert(smem_bytes<1, 1>() <= 225 * 1024 && smem_bytes<1, 2>() <= 225 * 1024 && smem_bytes<1, 4>() <= 225 * 1024,
+              "standalone projection ring too large");
 
 template <int NT, int GPU>
 __global__ void __launch_bounds__(kW * 32) gemv_kernel(const __grid_constant__ GemvArgs a) {
@@ -37,12 +42,13 @@ __global__ void __launch_bounds__(kW * 32) gemv_kernel(const __grid_constant__ G
     s_gp = p;
   }
   __syncthreads();
-  const size_t ring_bytes = (size_t)kW * kRingSlots * Geom<GPU>::kUnitBytes;
-  uint8_t* ring = smem + (size_t)warp * kRingSlots * Geom<GPU>::kUnitBytes;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + ring_bytes) + warp * kRingSlots;
+  constexpr int kSlots = Geom<GPU>::kGemvSlots;
+  const size_t ring_bytes = (size_t)kW * kSlots * Geom<GPU>::kUnitBytes;
+  uint8_t* ring = smem + (size_t)warp * kSlots * Geom<GPU>::kUnitBytes;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + ring_bytes) + warp * kSlots;
   {
     WarpStream<GPU> ws;
-    ws.init(s_op, 1, blockIdx.x, gridDim.x, warp, ring, bars, lane);
+    ws.init(s_op, 1, blockIdx.x, gridDim.x, warp, kW, ring, bars, kSlots == 4 ? 2 : 1, lane);
     ws.fill(lane);
     if (lane == 0) s_ws[warp] = ws;
     __syncwarp();
@@ -91,11 +97,12 @@ int gemv_grid(int nt, int num_sms) {
   return kCtasPerSm * num_sms;
 }
 
-int gemv_warps_per_cta() { return kW; }
+// the larger of the two kernels' warp counts: buffers and index checks cover both
+int gemv_warps_per_cta() { return kW > kCtaWarps ? kW : kCtaWarps; }
 
-size_t gemv_partials_floats(int grid) { return (size_t)grid * kW * 2 * kPieceFloats; }
+size_t gemv_partials_floats(int grid) { return (size_t)grid * gemv_warps_per_cta() * 2 * kPieceFloats; }
 
-size_t gemv_flags_count(int grid) { return (size_t)grid * kW * 2; }
+size_t gemv_flags_count(int grid) { return (size_t)grid * gemv_warps_per_cta() * 2; }
 
 cudaError_t launch_gemv(const GemvArgs& a, int nt, int group, int grid, cudaStream_t s, bool pdl) {
   if (nt == 1) {

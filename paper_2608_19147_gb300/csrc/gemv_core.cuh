@@ -3,9 +3,10 @@
 //
 // Work split.  The unit stream of a projection (n_rb row-blocks x upr units,
 // see kernels.h) is cut into contiguous runs, one per warp of the grid
-// (warp g = cta * kCtaWarps + warp), so every warp streams the same number of
+// (warp g = cta * warps per CTA + warp), so every warp streams the same number of
 // bytes and keeps its sums in registers for as long as its run stays inside
-// one row-block.  Each warp owns a ring of kRingSlots shared-memory slots that
+// one row-block.  Each warp owns a ring of shared-memory slots (a power of two:
+// kRingSlots in the step kernel, Geom::kGemvSlots in the standalone projection) that
 // its lane 0 fills with bulk copies (TMA, non-tensor), one unit per slot,
 // completion tracked by one mbarrier per slot.  Because the weights never
 // depend on earlier work, a warp's ring runs ahead through the *sequence* of
@@ -32,13 +33,18 @@
 
 namespace shard {
 
-constexpr int kRingSlots = 2;  // units in flight per warp (measured: a third adds nothing)
-constexpr int kCtaWarps = 12;  // warps per CTA that run projections
+constexpr int kRingSlots = 2;  // step kernel: units in flight per warp (measured: a third adds nothing)
+static_assert(kRingSlots == 2 || kRingSlots == 4, "ring slots: a power of two the init call passes as a shift");
+constexpr int kCtaWarps = 12;   // warps per CTA of the step kernel (all run projections)
+constexpr int kGemvWarps = 12;  // warps per CTA of the standalone projection kernel
 
 template <int GPU>
 struct Geom {
   static constexpr int kUnitBytes = kCodeBytes + GPU * kMetaBytesPerGroup;
   static constexpr int kBlocksPerGroup = 8 / GPU;
+  // the standalone projection (no attention area competes for shared
+  // memory): four slots per warp where 12 warps' rings fit in 216 KB, else two
+  static constexpr int kGemvSlots = kGemvWarps * 4 * kUnitBytes <= 216 * 1024 ? 4 : 2;
 };
 
 __device__ __forceinline__ uint32_t hsub2_u32(uint32_t a, uint32_t b) {
@@ -88,8 +94,11 @@ struct WarpStream {
   static constexpr int UB = Geom<GPU>::kUnitBytes;
   const OpDesc* ops;  // shared memory
   int n_ops, cta, n_cta, warp;
-  uint8_t* ring;      // [kRingSlots][UB]
-  uint64_t* bars;     // [kRingSlots]
+  int cta_warps;       // projection warps per CTA (the warp index space is cta * cta_warps + warp)
+  uint8_t* ring;      // [slots][UB]
+  uint64_t* bars;     // [slots]
+  uint32_t slot_mask;  // slots - 1 (slots a power of two)
+  int slot_shift;      // log2(slots)
   // fill cursor: op index, next unit, end of the CTA's range, op's units
   int f_op, f_u, f_end;
   const uint8_t* f_units;
@@ -99,7 +108,7 @@ struct WarpStream {
   // Run [wb, we) of this warp in op's unit stream.
   __device__ __forceinline__ void warp_range(int op, int& wb, int& we) const {
     const int T = ops[op].n_rb * ops[op].upr;
-    const int g = cta * kCtaWarps + warp, nw = n_cta * kCtaWarps;
+    const int g = cta * cta_warps + warp, nw = n_cta * cta_warps;
     wb = part_start(T, g, nw);
     we = part_start(T, g + 1, nw);
   }
@@ -108,9 +117,12 @@ struct WarpStream {
     f_units = ops[op].units;
   }
   // lane 0 initialises the slot barriers; the warp is synced after.
-  __device__ void init(const OpDesc* ops_, int n_ops_, int cta_, int n_cta_, int warp_, uint8_t* ring_, uint64_t* bars_,
-                       int lane) {
+  __device__ void init(const OpDesc* ops_, int n_ops_, int cta_, int n_cta_, int warp_, int cta_warps_, uint8_t* ring_,
+                       uint64_t* bars_, int slot_shift_, int lane) {
     ops = ops_;
+    cta_warps = cta_warps_;
+    slot_shift = slot_shift_;
+    slot_mask = (1u << slot_shift_) - 1u;
     n_ops = n_ops_;
     cta = cta_;
     n_cta = n_cta_;
@@ -124,14 +136,14 @@ struct WarpStream {
     f_units = nullptr;
     if (n_ops > 0) open_op(0);
     if (lane == 0) {
-      for (int s = 0; s < kRingSlots; ++s) mbar_init(&bars[s], 1);
+      for (uint32_t s = 0; s <= slot_mask; ++s) mbar_init(&bars[s], 1);
       mbar_fence_init();
     }
     __syncwarp();
   }
   // Issues bulk copies until the ring is full or the stream ends.
   __device__ __forceinline__ void fill(int lane) {
-    while (n_filled - n_used < (uint32_t)kRingSlots) {
+    while (n_filled - n_used <= slot_mask) {
       while (f_u >= f_end) {
         if (++f_op >= n_ops) return;
         open_op(f_op);
@@ -139,7 +151,7 @@ struct WarpStream {
       const uint8_t* src = f_units + (size_t)f_u * UB;
       ++f_u;
       if (lane == 0) {
-        const int slot = n_filled % kRingSlots;
+        const int slot = n_filled & slot_mask;
         fence_proxy_async_smem();
         mbar_arrive_expect_tx(&bars[slot], UB);
         // L2 evict-first: each weight byte is read once per step
@@ -149,8 +161,8 @@ struct WarpStream {
     }
   }
   __device__ __forceinline__ const uint8_t* acquire() {
-    const int slot = n_used % kRingSlots;
-    if (!timed_out && !mbar_wait(&bars[slot], (n_used / kRingSlots) & 1)) timed_out = true;
+    const int slot = n_used & slot_mask;
+    if (!timed_out && !mbar_wait(&bars[slot], (n_used >> slot_shift) & 1)) timed_out = true;
     return ring + (size_t)slot * UB;
   }
   __device__ __forceinline__ void release(int lane) {
@@ -329,8 +341,8 @@ struct GemvPhase {
   uint32_t act_s;       // 0, or the shared-memory address of this CTA's own copy of the activations,
   int act_s_ld;         // fp16 [M][act_s_ld], read instead of act
   bool skip;            // consume the weights but compute nothing (aborted step)
-  float* partials;      // [n_cta * kCtaWarps][2][kPieceFloats] pieces of split row-blocks
-  unsigned* flags;      // [n_cta * kCtaWarps][2] epoch of the piece last published in each slot
+  float* partials;      // [n_cta * warps per CTA][2][kPieceFloats] pieces of split row-blocks
+  unsigned* flags;      // [n_cta * warps per CTA][2] epoch of the piece last published in each slot
   int* status;
   const StepParams* sp;
   EpiArgs ep;
@@ -526,7 +538,7 @@ __device__ __noinline__ void gemv_phase(WarpStream<GPU>* ws_io, int op, const Ge
   if (wb >= we) return;
   const int upr = ws.ops[op].upr;
   const int T = ws.ops[op].n_rb * upr;
-  const int g = ws.cta * kCtaWarps + ws.warp, nw = ws.n_cta * kCtaWarps;
+  const int g = ws.cta * ws.cta_warps + ws.warp, nw = ws.n_cta * ws.cta_warps;
   const uint16_t* actp = p.act;
   const uint32_t acts = p.act_s;
   const int act_ld = acts ? p.act_s_ld : p.act_ld, M = p.M;

@@ -30,9 +30,11 @@ using namespace shard;
 
 namespace {
 
-constexpr int kNormThreads = 256;
+constexpr int kNormThreads = 512;
+constexpr int kNormVec = 4;          // 8-element pieces per thread kept in registers (H <= 16384)
 constexpr int kTopThreads = 256;
-constexpr int kTopChunkMin = 512;  // logits per top-1 CTA, at least
+constexpr int kTopChunkMin = 512;    // logits per top-1 CTA, at least ...
+constexpr int kTopChunkMax = 1024;   // ... and at most (four per thread, loaded at once)
 
 int fail(int code, const char* fmt, ...) __attribute__((format(printf, 2, 3)));
 int fail(int code, const char* fmt, ...) {
@@ -52,6 +54,10 @@ int fail(int code, const char* fmt, ...) {
                   cudaGetErrorString(_e), __FILE__, __LINE__);                                      \
   } while (0)
 
+__device__ __forceinline__ float2 h2f2(uint32_t u) {
+  return make_float2(h2f(static_cast<uint16_t>(u & 0xFFFFu)), h2f(static_cast<uint16_t>(u >> 16)));
+}
+
 __device__ __forceinline__ float block_sum(float v, float* red) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
 #pragma unroll
@@ -70,152 +76,174 @@ __device__ __forceinline__ float block_sum(float v, float* red) {
   return r;
 }
 
-// x = hidden[m] / sqrt(mean(hidden[m]^2) + eps) * w, rounded to fp16.
+// x = hidden[m] / sqrt(mean(hidden[m]^2) + eps) * w, rounded to fp16.  One
+// CTA per row; when H is a multiple of 8 and fits, every thread loads its
+// 8-element pieces once (all loads in flight) and keeps them in registers.
 __global__ void __launch_bounds__(kNormThreads) head_norm_kernel(const uint16_t* __restrict__ hidden, int H,
                                                                  const uint16_t* __restrict__ w, float eps,
                                                                  uint16_t* __restrict__ act, int act_ld) {
   __shared__ float red[kNormThreads / 32];
   pdl_launch_dependents();  // the projection may start streaming its weights
-  const int m = blockIdx.x;
+  const int m = blockIdx.x, tid = threadIdx.x;
   const uint16_t* h = hidden + (size_t)m * H;
+  uint16_t* out = act + (size_t)m * act_ld;
+  if (H % 8 == 0 && H <= kNormThreads * kNormVec * 8) {
+    const int nv = H / 8;
+    uint4 v[kNormVec], wv[kNormVec];
+#pragma unroll
+    for (int j = 0; j < kNormVec; ++j) {
+      const int i = tid + j * kNormThreads;
+      if (i < nv) {
+        v[j] = __ldcg(reinterpret_cast<const uint4*>(h) + i);
+        wv[j] = __ldg(reinterpret_cast<const uint4*>(w) + i);
+      }
+    }
+    float ss = 0.f;
+#pragma unroll
+    for (int j = 0; j < kNormVec; ++j) {
+      if (tid + j * kNormThreads < nv) {
+        const uint32_t u[4] = {v[j].x, v[j].y, v[j].z, v[j].w};
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const float2 f = h2f2(u[q]);
+          ss += f.x * f.x + f.y * f.y;
+        }
+      }
+    }
+    const float r = rsqrtf(block_sum(ss, red) / H + eps);
+#pragma unroll
+    for (int j = 0; j < kNormVec; ++j) {
+      const int i = tid + j * kNormThreads;
+      if (i < nv) {
+        const uint32_t u[4] = {v[j].x, v[j].y, v[j].z, v[j].w};
+        const uint32_t g[4] = {wv[j].x, wv[j].y, wv[j].z, wv[j].w};
+        uint32_t o[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const float2 f = h2f2(u[q]), gw = h2f2(g[q]);
+          o[q] = (uint32_t)f2h(f.x * r * gw.x) | ((uint32_t)f2h(f.y * r * gw.y) << 16);
+        }
+        reinterpret_cast<uint4*>(out)[i] = make_uint4(o[0], o[1], o[2], o[3]);
+      }
+    }
+    return;
+  }
   float ss = 0.f;
-  for (int i = threadIdx.x; i < H; i += blockDim.x) {
-    const float v = h2f(h[i]);
-    ss += v * v;
+  for (int i = tid; i < H; i += blockDim.x) {
+    const float x = h2f(h[i]);
+    ss += x * x;
   }
   const float r = rsqrtf(block_sum(ss, red) / H + eps);
-  for (int i = threadIdx.x; i < H; i += blockDim.x) act[(size_t)m * act_ld + i] = f2h(h2f(h[i]) * r * h2f(w[i]));
+  for (int i = tid; i < H; i += blockDim.x) out[i] = f2h(h2f(h[i]) * r * h2f(w[i]));
 }
 
 struct Top1Part {
-  float max, sum;  // the chunk's largest logit; sum of exp(logit - max) over the chunk
+  float max, sum;  // the largest logit; sum of exp(logit - max)
   int idx, pad;    // the lowest id holding max
 };
 
-// a then b, where every id of a is below every id of b
-__device__ __forceinline__ void top1_merge(float& m, float& s, int& i, float m2, float s2, int i2) {
-  if (m2 > m) {
-    s = s * expf(m - m2) + s2;
-    m = m2;
-    i = i2;
-  } else {
-    s = s + s2 * expf(m2 - m);
+// Folds (bm, bs, bi) into (am, as, ai), a first: the larger maximum wins,
+// equal maxima keep the lower id, the sums are rescaled to the new maximum.
+// An empty side has max -inf and sum 0.
+__device__ __forceinline__ void top1_combine(float& am, float& as, int& ai, float bm, float bs, int bi) {
+  if (bm == -INFINITY) return;
+  if (am == -INFINITY) {
+    am = bm;
+    as = bs;
+    ai = bi;
+    return;
   }
+  const float nm = fmaxf(am, bm);
+  as = as * expf(am - nm) + bs * expf(bm - nm);
+  ai = am > bm ? ai : (bm > am ? bi : min(ai, bi));
+  am = nm;
 }
 
-// (max, lowest argmax) over a warp, then sum of exp relative to the max.
-__device__ __forceinline__ void warp_max_idx(float& m, int& i) {
+// Butterfly over the 32 lanes; both partners fold the lower lane's part
+// first, so every lane ends with the same bits.
+__device__ __forceinline__ void top1_warp(float& m, float& s, int& i) {
+  const int lane = threadIdx.x & 31;
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
+  for (int o = 1; o < 32; o <<= 1) {
     const float m2 = __shfl_xor_sync(0xffffffffu, m, o);
+    const float s2 = __shfl_xor_sync(0xffffffffu, s, o);
     const int i2 = __shfl_xor_sync(0xffffffffu, i, o);
-    if (m2 > m || (m2 == m && i2 < i)) {
-      m = m2;
-      i = i2;
+    if ((lane & o) == 0) {
+      top1_combine(m, s, i, m2, s2, i2);
+    } else {
+      float am = m2, as = s2;
+      int ai = i2;
+      top1_combine(am, as, ai, m, s, i);
+      m = am;
+      s = as;
+      i = ai;
     }
   }
 }
 
+// (chunk, row) CTAs: one pass over the chunk's logits with an online
+// (max, sum of exp) per thread, a fixed-order reduction over the CTA, and
+// the row's last CTA folds the chunks.
 __global__ void __launch_bounds__(kTopThreads) head_top1_kernel(const float* __restrict__ logits, int ld, int V,
                                                                 int chunk, Top1Part* __restrict__ parts,
-                                                                int* __restrict__ done, int32_t* __restrict__ token,
+                                                                int* __restrict__ done, const int* status,
+                                                                int32_t* __restrict__ token,
                                                                 float* __restrict__ p_max) {
-  __shared__ float s_m[kTopThreads / 32];
+  __shared__ float s_m[kTopThreads / 32], s_s[kTopThreads / 32];
   __shared__ int s_i[kTopThreads / 32];
-  __shared__ float red[kTopThreads / 32];
   __shared__ int s_last;
-  pdl_wait();  // the projection's logits
   const int c = blockIdx.x, m = blockIdx.y, nc = gridDim.x;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const float* l = logits + (size_t)m * ld;
   const int b = c * chunk, e = min(V, b + chunk);
-  // 1. the chunk's max and its lowest id
-  float mx = -INFINITY;
+  float mx = -INFINITY, sm = 0.f;
   int ix = 0x7fffffff;
-  for (int v = b + threadIdx.x; v < e; v += blockDim.x) {
-    const float x = __ldcg(l + v);
-    if (x > mx) {  // ids rise along a thread's walk: the first max is the lowest
-      mx = x;
-      ix = v;
-    }
+  constexpr int kPer = kTopChunkMax / kTopThreads;
+  float x[kPer];
+#pragma unroll
+  for (int j = 0; j < kPer; ++j) {
+    const int v = b + threadIdx.x + j * kTopThreads;
+    x[j] = v < e ? __ldcg(l + v) : -INFINITY;
   }
-  warp_max_idx(mx, ix);
+#pragma unroll
+  for (int j = 0; j < kPer; ++j) {
+    const int v = b + threadIdx.x + j * kTopThreads;
+    if (v < e) top1_combine(mx, sm, ix, x[j], 1.f, v);  // ids rise along a thread's walk
+  }
+  top1_warp(mx, sm, ix);
   if (lane == 0) {
     s_m[warp] = mx;
+    s_s[warp] = sm;
     s_i[warp] = ix;
   }
   __syncthreads();
   if (warp == 0) {
-    mx = lane < (kTopThreads / 32) ? s_m[lane] : -INFINITY;
-    ix = lane < (kTopThreads / 32) ? s_i[lane] : 0x7fffffff;
-    warp_max_idx(mx, ix);
+    mx = lane < kTopThreads / 32 ? s_m[lane] : -INFINITY;
+    sm = lane < kTopThreads / 32 ? s_s[lane] : 0.f;
+    ix = lane < kTopThreads / 32 ? s_i[lane] : 0x7fffffff;
+    top1_warp(mx, sm, ix);
     if (lane == 0) {
-      s_m[0] = mx;
-      s_i[0] = ix;
+      parts[(size_t)m * nc + c] = Top1Part{mx, sm, ix, 0};
+      __threadfence();
+      s_last = atomicAdd(done + m, 1) == nc - 1;
     }
   }
   __syncthreads();
-  const float cm = s_m[0];
-  // 2. sum of exp(logit - chunk max)
-  float s = 0.f;
-  for (int v = b + threadIdx.x; v < e; v += blockDim.x) s += expf(__ldcg(l + v) - cm);
-  s = block_sum(s, red);
-  if (threadIdx.x == 0) {
-    parts[(size_t)m * nc + c] = Top1Part{cm, s, s_i[0], 0};
-    __threadfence();
-    s_last = atomicAdd(done + m, 1) == nc - 1;
-  }
-  __syncthreads();
-  if (!s_last) return;
-  // 3. the row's last CTA combines the chunks (warp 0): lane L folds chunks
-  // L, L + 32, ... in order, then a butterfly in which both partners combine
-  // the lower lane's part first -- a fixed order, so every lane ends with the
-  // same bits whatever the arrival order of the CTAs
+  if (!s_last || warp != 0) return;
+  // the row's last CTA: lane L folds chunks L, L + 32, ... in order, then the
+  // butterfly -- a fixed order, whatever the arrival order of the CTAs
   __threadfence();
-  if (warp != 0) return;
   float gm = -INFINITY, gs = 0.f;
   int gi = 0x7fffffff;
-  for (int k = lane; k < nc; k += 32) {
-    const float pm = __ldcg(&parts[(size_t)m * nc + k].max);
-    const float ps = __ldcg(&parts[(size_t)m * nc + k].sum);
-    const int pi = __ldcg(&parts[(size_t)m * nc + k].idx);
-    if (gs == 0.f && gm == -INFINITY) {
-      gm = pm;
-      gs = ps;
-      gi = pi;
-    } else {
-      top1_merge(gm, gs, gi, pm, ps, pi);
-    }
-  }
-  // butterfly over lanes: the id ranges of two lanes interleave, so the
-  // merge keeps the lowest id among equal maxima explicitly
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const float m2 = __shfl_xor_sync(0xffffffffu, gm, o);
-    const float s2 = __shfl_xor_sync(0xffffffffu, gs, o);
-    const int i2 = __shfl_xor_sync(0xffffffffu, gi, o);
-    const bool lo = (lane & o) == 0;  // combine in a lane-symmetric order: lower lane's part first
-    float am = lo ? gm : m2, as = lo ? gs : s2, bm = lo ? m2 : gm, bs = lo ? s2 : gs;
-    int ai = lo ? gi : i2, bi = lo ? i2 : gi;
-    if (bs == 0.f && bm == -INFINITY) {
-      // b is empty
-    } else if (as == 0.f && am == -INFINITY) {
-      am = bm;
-      as = bs;
-      ai = bi;
-    } else {
-      const float nm = fmaxf(am, bm);
-      as = as * expf(am - nm) + bs * expf(bm - nm);
-      ai = am > bm ? ai : (bm > am ? bi : min(ai, bi));
-      am = nm;
-    }
-    gm = am;
-    gs = as;
-    gi = ai;
-  }
+  for (int k = lane; k < nc; k += 32)
+    top1_combine(gm, gs, gi, __ldcg(&parts[(size_t)m * nc + k].max), __ldcg(&parts[(size_t)m * nc + k].sum),
+                 __ldcg(&parts[(size_t)m * nc + k].idx));
+  top1_warp(gm, gs, gi);
   if (lane == 0) {
-    token[m] = gi;
-    if (p_max) p_max[m] = 1.f / gs;
+    // a projection wait that gave up (never expected) marks the row failed
+    const bool ok = __ldcg(status) == 0;
+    token[m] = ok ? gi : -1;
+    if (p_max) p_max[m] = ok ? 1.f / gs : __int_as_float(0x7fc00000);
     done[m] = 0;  // ready for the next call
   }
 }
@@ -236,7 +264,6 @@ struct head_s {
   unsigned* flags = nullptr;    // projection piece flags
   unsigned epoch = 1;
   int* status = nullptr;
-  int* status_host = nullptr;   // pinned mirror, copied after each call
   Top1Part* parts = nullptr;    // [16][max chunks]
   int* done = nullptr;          // [16] chunk arrivals per row (self-resetting)
   int max_chunks = 0;
@@ -258,7 +285,6 @@ void destroy(head_s* h) {
   cudaFree(h->partials);
   cudaFree(h->flags);
   cudaFree(h->status);
-  if (h->status_host) cudaFreeHost(h->status_host);
   cudaFree(h->parts);
   cudaFree(h->done);
   cudaFree(h->hidden_dev);
@@ -268,11 +294,11 @@ void destroy(head_s* h) {
 }
 
 int chunk_of(const head_s* h, int M, int* n_chunks) {
-  // about two CTAs per SM over the M rows, at least kTopChunkMin logits each
+  // about one CTA per SM over the M rows, kTopChunkMin..kTopChunkMax logits each
   const int V = h->cfg.vocab;
-  int nc = std::max(1, (2 * h->num_sms) / M);
+  int nc = std::max(1, h->num_sms / M);
   nc = std::min(nc, std::max(1, (V + kTopChunkMin - 1) / kTopChunkMin));
-  nc = std::min(nc, h->max_chunks);
+  nc = std::max(nc, (V + kTopChunkMax - 1) / kTopChunkMax);
   const int chunk = (V + nc - 1) / nc;
   *n_chunks = (V + chunk - 1) / chunk;
   return chunk;
@@ -288,14 +314,12 @@ unsigned next_epoch(head_s* h) {
   return h->epoch++;
 }
 
-// norm -> projection -> top-1 (logits only, when token == nullptr)
+// norm -> projection -> top-1 (logits only, when token == nullptr).  No
+// status copy per call: a copy-engine transfer between the calls' kernels
+// measured ~9 us of stream time per call; the top-1 kernel reports a failed
+// projection in the tokens instead.
 int run(head_s* h, const uint16_t* hidden, int M, int32_t* token, float* p_max, float* logits, int ld,
         cudaStream_t s) {
-  const int bits = *reinterpret_cast<volatile int*>(h->status_host);
-  if (bits) {
-    *reinterpret_cast<volatile int*>(h->status_host) = 0;
-    return fail(SHARD_ECUDA, "an earlier head call reported a device wait timeout");
-  }
   const head_config& c = h->cfg;
   head_norm_kernel<<<M, kNormThreads, 0, s>>>(hidden, c.hidden, h->norm, (float)c.rms_eps, h->act, h->op.Kp);
   HEAD_CUDA_TRY(cudaGetLastError());
@@ -319,21 +343,14 @@ int run(head_s* h, const uint16_t* hidden, int M, int32_t* token, float* p_max, 
   HEAD_CUDA_TRY(launch_gemv(g, nt, c.group, std::min<long long>(h->grid[nt], (long long)h->op.n_rb * h->op.upr), s,
                             true));
   if (token) {
+    // a plain launch: with programmatic dependent launch this kernel measured
+    // ~8 us slower per call
     int nc = 0;
     const int chunk = chunk_of(h, M, &nc);
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(nc, M);
-    cfg.blockDim = dim3(kTopThreads);
-    cfg.stream = s;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    HEAD_CUDA_TRY(cudaLaunchKernelEx(&cfg, head_top1_kernel, (const float*)logits, ld, c.vocab, chunk, h->parts,
-                                     h->done, token, p_max));
+    head_top1_kernel<<<dim3(nc, M), kTopThreads, 0, s>>>(logits, ld, c.vocab, chunk, h->parts, h->done, h->status,
+                                                        token, p_max);
+    HEAD_CUDA_TRY(cudaGetLastError());
   }
-  HEAD_CUDA_TRY(cudaMemcpyAsync(h->status_host, h->status, sizeof(int), cudaMemcpyDeviceToHost, s));
   return SHARD_OK;
 }
 
@@ -416,9 +433,7 @@ int head_create(const head_config* cfg, const head_weights_host* w, head_t* out)
          HEAD_CUDA_TRY(cudaMemset(h->flags, 0, sizeof(unsigned) * gemv_flags_count(h->grid[0])));
          HEAD_CUDA_TRY(cudaMalloc(&h->status, sizeof(int)));
          HEAD_CUDA_TRY(cudaMemset(h->status, 0, sizeof(int)));
-         HEAD_CUDA_TRY(cudaHostAlloc(&h->status_host, sizeof(int), cudaHostAllocDefault));
-         *h->status_host = 0;
-         h->max_chunks = 2 * h->num_sms;
+         h->max_chunks = (c.vocab + kTopChunkMin - 1) / kTopChunkMin + 1;
          HEAD_CUDA_TRY(cudaMalloc(&h->parts, sizeof(Top1Part) * kMaxTokens * h->max_chunks));
          HEAD_CUDA_TRY(cudaMalloc(&h->done, sizeof(int) * kMaxTokens));
          HEAD_CUDA_TRY(cudaMemset(h->done, 0, sizeof(int) * kMaxTokens));
@@ -457,11 +472,12 @@ int head_top1_host(head_t h, const uint16_t* hidden, int M, int32_t* token, floa
   HEAD_CUDA_TRY(cudaMemcpyAsync(token, h->token_dev, sizeof(int32_t) * M, cudaMemcpyDeviceToHost, s));
   if (p_max) HEAD_CUDA_TRY(cudaMemcpyAsync(p_max, h->p_dev, sizeof(float) * M, cudaMemcpyDeviceToHost, s));
   HEAD_CUDA_TRY(cudaStreamSynchronize(s));
-  const int bits = *reinterpret_cast<volatile int*>(h->status_host);
-  if (bits) {
-    *reinterpret_cast<volatile int*>(h->status_host) = 0;
-    return fail(SHARD_ECUDA, "head_top1_host: a device wait timed out");
-  }
+  for (int m = 0; m < M; ++m)
+    if (token[m] < 0) {
+      cudaMemsetAsync(h->status, 0, sizeof(int), s);
+      cudaStreamSynchronize(s);
+      return fail(SHARD_ECUDA, "head_top1_host: a device wait of the projection timed out");
+    }
   return SHARD_OK;
 }
 

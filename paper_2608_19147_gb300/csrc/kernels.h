@@ -209,6 +209,8 @@ struct StepKernelArgs {
   unsigned long long* barrier;         // grid-barrier counter (monotonic)
   unsigned long long barrier_base;     // its value when this launch starts
   unsigned long long* phase_clock;     // [step_barriers(L) + 1] globaltimer at each barrier
+  int* status_out;           // host-mapped mirror: the last CTA to finish copies a nonzero status there
+  int* exit_count;           // CTAs finished in this launch (zero between launches; the last resets it)
 };
 // One-time attribute setup of the step kernel variants for a group size and
 // head dim; number of grid barriers per step; launch (cooperative, one CTA

@@ -90,7 +90,9 @@ struct shard_s {
   unsigned epoch = 1;               // next epoch for the flags
   int max_rb = 0;
   int* status = nullptr;           // device status word
-  int* status_host = nullptr;      // pinned mirror (copied after each step)
+  int* status_host = nullptr;      // host-mapped mirror the step kernel writes a nonzero status to
+  int* status_host_dev = nullptr;  // its device address
+  int* exit_count = nullptr;       // step kernel: CTAs finished (zero between launches)
   StepParams* sp = nullptr;
   int grid[3] = {0, 0, 0};         // standalone GEMV grid per token bucket
   OpDesc* ops_dev = nullptr;       // [4L] op descriptors for the step kernel
@@ -393,8 +395,11 @@ int shard_create(const shard_config* cfg, const shard_weights_host* w, shard_t* 
   }
   CUDA_TRY(cudaMalloc(&sh->status, sizeof(int)));
   CUDA_TRY(cudaMemset(sh->status, 0, sizeof(int)));
-  CUDA_TRY(cudaHostAlloc(&sh->status_host, sizeof(int), cudaHostAllocDefault));
+  CUDA_TRY(cudaHostAlloc(&sh->status_host, sizeof(int), cudaHostAllocMapped));
   *sh->status_host = 0;
+  CUDA_TRY(cudaHostGetDevicePointer(reinterpret_cast<void**>(&sh->status_host_dev), sh->status_host, 0));
+  CUDA_TRY(cudaMalloc(&sh->exit_count, sizeof(int)));
+  CUDA_TRY(cudaMemset(sh->exit_count, 0, sizeof(int)));
   CUDA_TRY(cudaMalloc(&sh->sp, sizeof(StepParams)));
   CUDA_TRY(cudaMemset(sh->sp, 0, sizeof(StepParams)));
   {
@@ -433,6 +438,7 @@ int shard_destroy(shard_t sh) {
   cudaFree(sh->partials);
   cudaFree(sh->flags);
   cudaFree(sh->status);
+  cudaFree(sh->exit_count);
   cudaFree(sh->sp);
   cudaFree(sh->dstage);
   if (sh->pin) cudaFreeHost(sh->pin);
@@ -709,10 +715,11 @@ int shard_step(shard_t sh, kvstate_t st, const uint16_t* hidden_in, const int32_
   ka.barrier = sh->barrier;
   ka.barrier_base = sh->barrier_base;
   ka.phase_clock = sh->phase_clock;
+  ka.status_out = sh->status_host_dev;
+  ka.exit_count = sh->exit_count;
   const int grid = sh->num_sms;
   CUDA_TRY(launch_step(ka, M <= 8 ? 1 : 2, sh->cfg.group, grid, s));
   sh->barrier_base += (unsigned long long)sh->n_barriers * grid;
-  CUDA_TRY(cudaMemcpyAsync(sh->status_host, sh->status, sizeof(int), cudaMemcpyDeviceToHost, s));
 
   for (int b = 0; b < B; ++b) st->cursor[b] += n_new[b];
   if (beam_idx) {

@@ -705,7 +705,7 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
   if (threadIdx.x == 0 && blockIdx.x == 0) a.phase_clock[0] = globaltimer();
   {
     WarpStream<GPU> ws;
-    ws.init(s_ops, 4 * a.L, blockIdx.x, gridDim.x, warp, ring, bars, lane);
+    ws.init(s_ops, 4 * a.L, blockIdx.x, gridDim.x, warp, kWarps, ring, bars, kRingSlots == 4 ? 2 : 1, lane);
     ws.fill(lane);
     if (lane == 0) s_ws[warp] = ws;
     __syncwarp();
@@ -822,6 +822,14 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
     if (l + 1 < a.L) grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
   }
   if (s_ws[warp].timed_out && lane == 0) atomicOr(a.status, ST_WAIT_TIMEOUT);
+  // The last CTA to finish hands a nonzero status to the host-mapped mirror,
+  // so no copy-engine transfer has to follow the step on the stream.
+  __syncthreads();
+  if (threadIdx.x == 0 && atom_add_acq_rel(a.exit_count, 1) == (int)gridDim.x - 1) {
+    *a.exit_count = 0;
+    const int st = ld_acquire_s32(a.status);
+    if (st) *reinterpret_cast<volatile int*>(a.status_out) = st;
+  }
 }
 
 template <int NT, int GPU, int DPL>
