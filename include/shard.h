@@ -139,6 +139,24 @@ int kv_state_length(kvstate_t state, int row, int* len);
  * Errors: EINVAL, EUNSUPPORTED (entries shared through a beam gather). */
 int kv_trim(kvstate_t state, int row, const uint8_t* keep, int len);
 
+/* Prefix capture (Section 8.4, KV capture and warm-resume): copies the
+ * row's cache entries j < len with keep[j] != 0 (keep host uint8 [len], or
+ * NULL for all; len must equal the row's length), in cache order and for
+ * every layer, to host k and v, each [n_layers][n_kept][Hkv][d] fp16, and
+ * returns n_kept in *n_kept.  With keep = the request's attention-mask row,
+ * the masked (rejected) entries are compacted away.  Entries are read
+ * through the beam table, so rows that share entries after a gather export
+ * correctly.  The buffers must hold the row's length.  Synchronous.
+ * Errors: EINVAL. */
+int kv_state_export(kvstate_t state, int row, const uint8_t* keep, int len, uint16_t* k, uint16_t* v, int* n_kept);
+
+/* Warm resume: sets the row to len entries from host k and v, each
+ * [n_layers][len][Hkv][d] fp16 (the layout kv_state_export writes), as
+ * kv_state_load does for every layer.  Synchronous.  Errors: EINVAL,
+ * ECAPACITY (len > capacity), EUNSUPPORTED (entries shared through a beam
+ * gather; reset all rows first). */
+int kv_state_import(kvstate_t state, int row, const uint16_t* k, const uint16_t* v, int len);
+
 /* One decode step of the shard for B requests (B == the state's n_rows).
  *   n_new        host int32 [B], n_new[b] >= 1 new tokens of request b;
  *                M = sum(n_new) <= SHARD_MAX_TOKENS.  Tokens of request b

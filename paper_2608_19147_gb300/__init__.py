@@ -26,7 +26,7 @@ OP_QKV, OP_O, OP_GU, OP_DOWN = 0, 1, 2, 3
 
 # Every symbol include/shard.h and include/shard_debug.h declare.
 EXPORTS = ("shard_create", "shard_destroy", "kv_state_alloc", "kv_state_free", "kv_state_reset", "kv_state_load",
-           "kv_state_read", "kv_state_length", "kv_trim", "shard_step", "shard_step_host", "shard_sync_status",
+           "kv_state_read", "kv_state_length", "kv_trim", "kv_state_export", "kv_state_import", "shard_step", "shard_step_host", "shard_sync_status",
            "shard_last_error", "shard_debug_op_info", "shard_debug_unpack", "shard_debug_gemv",
            "shard_debug_phase_times", "shard_gemv_noalloc", "head_create", "head_destroy", "head_top1",
            "head_top1_host", "head_debug_logits")
@@ -91,6 +91,8 @@ def load_library(path: str = LIB_PATH):
         "kv_state_read": ([vp, ip, ip, ip, ip, vp, vp], ip),
         "kv_state_length": ([vp, ip, ctypes.POINTER(ctypes.c_int)], ip),
         "kv_trim": ([vp, ip, vp, ip], ip),
+        "kv_state_export": ([vp, ip, vp, ip, vp, vp, ctypes.POINTER(ctypes.c_int)], ip),
+        "kv_state_import": ([vp, ip, vp, vp, ip], ip),
         "shard_step": ([vp, vp, vp, vp, i32p, ip, vp, vp, ip, vp, vp, vp], ip),
         "shard_step_host": ([vp, vp, vp, vp, i32p, ip, vp, vp, ip, vp, vp, vp], ip),
         "shard_sync_status": ([vp, vp], ip),
@@ -196,6 +198,27 @@ def kv_state_length(state: int, row: int) -> int:
 def kv_trim(state: int, row: int, keep: np.ndarray) -> None:
     keep = np.ascontiguousarray(keep, dtype=np.uint8)
     _check(load_library().kv_trim(state, row, _np(keep), keep.size))
+
+
+def kv_state_export(state: int, row: int, length: int, n_layers: int, n_kv_heads: int, head_dim: int,
+                    keep: Optional[np.ndarray] = None):
+    """Compacted copy of the row's entries with keep != 0 (all when None):
+    (k, v), each [n_layers][n_kept][Hkv][d] fp16 bits."""
+    per = n_kv_heads * head_dim
+    k = np.empty(n_layers * max(length, 1) * per, dtype=np.uint16)
+    v = np.empty_like(k)
+    kp = None if keep is None else np.ascontiguousarray(keep, dtype=np.uint8)
+    n = ctypes.c_int()
+    _check(load_library().kv_state_export(state, row, _np(kp), length, _np(k), _np(v), ctypes.byref(n)))
+    shape = (n_layers, n.value, n_kv_heads, head_dim)  # packed: [n_layers][n_kept][Hkv][d]
+    return k[:n_layers * n.value * per].reshape(shape).copy(), v[:n_layers * n.value * per].reshape(shape).copy()
+
+
+def kv_state_import(state: int, row: int, k: np.ndarray, v: np.ndarray) -> None:
+    """k, v: [n_layers][len][Hkv][d] fp16 bits (as kv_state_export returns)."""
+    k = np.ascontiguousarray(k, dtype=np.uint16)
+    v = np.ascontiguousarray(v, dtype=np.uint16)
+    _check(load_library().kv_state_import(state, row, _np(k), _np(v), k.shape[1]))
 
 
 def shard_step(shard: int, state: int, hidden_in: Optional[int], token_ids: Optional[int], n_new: Sequence[int],

@@ -586,6 +586,51 @@ int kv_state_read(kvstate_t st, int row, int layer, int start, int len, uint16_t
   return SHARD_OK;
 }
 
+int kv_state_export(kvstate_t st, int row, const uint8_t* keep, int len, uint16_t* k, uint16_t* v, int* n_kept) {
+  if (!st || !k || !v || !n_kept) return fail(SHARD_EINVAL, "kv_state_export: null argument");
+  shard_s* sh = st->sh;
+  if (row < 0 || row >= st->n_rows) return fail(SHARD_EINVAL, "kv_state_export: row out of range");
+  int cur = 0;
+  int rc = kv_state_length(st, row, &cur);
+  if (rc) return rc;
+  if (len != cur) return fail(SHARD_EINVAL, "kv_state_export: len %d != row length %d", len, cur);
+  *n_kept = 0;
+  if (len == 0) return SHARD_OK;
+  // the row's slots (beam table), then the kept ones in cache order
+  std::vector<int> all(len), slots;
+  CUDA_TRY(cudaMemcpy(all.data(), st->bt[st->bt_cur] + (size_t)row * st->cap, sizeof(int) * len,
+                      cudaMemcpyDeviceToHost));
+  for (int j = 0; j < len; ++j)
+    if (!keep || keep[j]) slots.push_back(all[j]);
+  const int n = static_cast<int>(slots.size());
+  if (n > 0) {
+    DevBuf<int> dslots;
+    DevBuf<uint16_t> tmp;
+    CUDA_TRY(dslots.alloc(n));
+    CUDA_TRY(cudaMemcpy(dslots.p, slots.data(), sizeof(int) * n, cudaMemcpyHostToDevice));
+    CUDA_TRY(tmp.alloc((size_t)sh->L * n * sh->Hkv * sh->d));
+    for (int which = 0; which < 2; ++which) {
+      const uint16_t* pool = which == 0 ? st->k : st->v;
+      CUDA_TRY(launch_kv_gather(pool, sh->L, st->layer_stride, sh->Hkv, st->cap, sh->d, dslots.p, n, tmp.p, nullptr));
+      CUDA_TRY(cudaMemcpy(which == 0 ? k : v, tmp.p, sizeof(uint16_t) * tmp.n, cudaMemcpyDeviceToHost));
+    }
+  }
+  *n_kept = n;
+  return SHARD_OK;
+}
+
+int kv_state_import(kvstate_t st, int row, const uint16_t* k, const uint16_t* v, int len) {
+  if (!st || ((!k || !v) && len > 0)) return fail(SHARD_EINVAL, "kv_state_import: null argument");
+  shard_s* sh = st->sh;
+  const size_t per_layer = (size_t)len * sh->Hkv * sh->d;
+  for (int l = 0; l < sh->L; ++l) {
+    int rc = kv_state_load(st, row, l, len > 0 ? k + (size_t)l * per_layer : k, len > 0 ? v + (size_t)l * per_layer : v,
+                           len);
+    if (rc) return rc;
+  }
+  return SHARD_OK;
+}
+
 int kv_trim(kvstate_t st, int row, const uint8_t* keep, int len) {
   if (!st || !keep) return fail(SHARD_EINVAL, "kv_trim: null argument");
   shard_s* sh = st->sh;
