@@ -16,7 +16,7 @@ so every step is a step of that workload.  Weights are seeded synthetic
 far larger than L2, so no L2 flush is needed between steps.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl gb300|reference]
-                  [--config 8b-decode|8b-verify|8b-microbatch|70b-decode|70b-verify|tiny]
+                  [--config 8b-decode|8b-verify|8b-microbatch|70b-decode|70b-verify|tiny|8b-head|8b-head-verify]
 
 Under torchrun each rank runs an independent replica on its own GPU
 (replicas only: the path has no exchange step) and rank 0 prints one JSON
@@ -63,7 +63,15 @@ CONFIGS = {
                                 "Bernoulli(0.6) prefix accept, 64 steps"),
     "tiny": dict(shape=synth.TINY, prefill=72, steps_per_request=256, rows=1, n=1, tokens=True,
                  workload="tiny 2L h256 decode: 72-token prefill, 1 token/step"),
+    # the final stage's LM head with top-1 compression (Section 6.7), not a shard step
+    "8b-head": dict(head=(4096, 128256, 128), rows=1,
+                    workload="llama3.1-8b final-stage LM head, top-1: RMSNorm + 128256x4096 INT4 lm_head + "
+                             "argmax/p_max, 1 hidden row per call"),
+    "8b-head-verify": dict(head=(4096, 128256, 128), rows=5,
+                           workload="llama3.1-8b final-stage LM head, top-1: RMSNorm + 128256x4096 INT4 lm_head + "
+                                    "argmax/p_max, 1+4 verify rows per call"),
 }
+HEAD_METRIC = "LM-head top-1 rows/s at 1 GB300 (final stage, Section 6.7); achieved HBM GB/s"
 
 
 def log(*a):
@@ -227,9 +235,15 @@ def measured_peaks():
         return {}
 
 
-def kernel_source_hash() -> str:
+KERNEL_SOURCES = {
+    "step": ("gemv_core.cuh", "step_kernel.cu", "common.cuh", "kernels.h"),
+    "head": ("gemv_core.cuh", "gemv.cu", "head.cu", "common.cuh", "kernels.h"),
+}
+
+
+def kernel_source_hash(kind: str = "step") -> str:
     h = hashlib.sha256()
-    for f in ("gemv_core.cuh", "step_kernel.cu", "common.cuh", "kernels.h"):
+    for f in KERNEL_SOURCES[kind]:
         h.update(open(os.path.join(ROOT, "paper_2608_19147_gb300", "csrc", f), "rb").read())
     return h.hexdigest()[:16]
 
@@ -241,7 +255,7 @@ def profiled_traffic(kind: str, cfg: str):
     try:
         data = json.load(open(path))
         ent = data.get("%s/%s" % (cfg, kind))
-        if ent and ent.get("kernel_hash") == kernel_source_hash():
+        if ent and ent.get("kernel_hash") == kernel_source_hash(kind):
             return ent.get("dram_bytes_per_launch")
     except Exception:
         pass
@@ -521,10 +535,170 @@ def cpu_baseline(cfg_name: str, weights, budget_s: float = 20.0, max_steps: int 
                       "OpenMP over output rows with %d threads, %.1f s" % (n, cfg_name, plan.M, threads, el)}
 
 
+def head_cpu_baseline(hw, M: int, budget_s: float = 20.0):
+    """The fp64 oracle head on a bounded sample: calls of M seeded rows until
+    about budget_s seconds of work."""
+    import oracle
+
+    threads = os.cpu_count() or 1
+    oracle.set_threads(threads)
+    shape = dataclasses.replace(synth.LLAMA8B_STAGE, hidden=hw.hidden)
+    n = 0
+    t0 = time.perf_counter()
+    while True:
+        oracle.head_top1(synth.hidden_in(shape, SEED, 10000 + n, M), hw.norm, hw.lm_head, hw.rms_eps)
+        n += 1
+        if time.perf_counter() - t0 > budget_s:
+            break
+    el = time.perf_counter() - t0
+    return {"value": n * M / el, "unit": "rows/s", "cores": threads, "kind": "oracle",
+            "sample": "%d calls of %d rows of the LM-head workload, fp64 oracle, OpenMP over vocabulary rows with "
+                      "%d threads, %.1f s" % (n, M, threads, el)}
+
+
+def run_head(args, rank: int, world: int):
+    """LM head with the top-1 epilogue: K calls of head_top1 on resident
+    hidden rows, CUDA-event timed; e2e through head_top1_host."""
+    import torch
+
+    import paper_2608_19147_gb300 as pkg
+
+    dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", "0")))
+    torch.cuda.set_device(dev)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.init_process_group("nccl", device_id=dev)
+    c = CONFIGS[args.config]
+    H, V, g = c["head"]
+    M = c["rows"]
+    K, W = args.steps, max(3, args.warmup)
+    hw = synth.make_head(H, V, g, SEED)
+    head = pkg.head_create(H, V, g, hw.rms_eps, hw.lm_head, hw.norm)
+    stream = torch.cuda.current_stream(dev)
+    sptr = stream.cuda_stream
+    shape = dataclasses.replace(synth.LLAMA8B_STAGE, hidden=H)
+    n_in = min(K, 64)  # distinct resident inputs, cycled
+    hid = torch.from_numpy(np.stack([synth.hidden_in(shape, SEED, t, M) for t in range(n_in)]).view(np.int16)).to(dev)
+    tok = torch.empty((K, M), dtype=torch.int32, device=dev)
+    pm = torch.empty((K, M), dtype=torch.float32, device=dev)
+    for t in range(W):
+        pkg.head_top1(head, hid[t % n_in].data_ptr(), M, tok[0].data_ptr(), pm[0].data_ptr(), sptr)
+    torch.cuda.synchronize()
+    gpu_id = ""
+    try:
+        gpu_id = str(torch.cuda.get_device_properties(dev).uuid)
+        if gpu_id and not gpu_id.startswith("GPU-"):
+            gpu_id = "GPU-" + gpu_id
+    except Exception:
+        gpu_id = ""
+    sampler = ClockSampler(gpu_id)
+    time.sleep(0.3)
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    w0 = time.time()
+    e0.record(stream)
+    for t in range(K):
+        pkg.head_top1(head, hid[t % n_in].data_ptr(), M, tok[t].data_ptr(), pm[t].data_ptr(), sptr)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    w1 = time.time()
+    if dist:
+        dist.barrier()
+    ms = e0.elapsed_time(e1)
+    sampler.stop()
+    clocks = sampler.summary(w0, w1)
+    if dist:
+        tt = torch.tensor([ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms = float(tt.item())
+    # end to end: host hidden rows in, host (token, p_max) out, every call
+    hosts = [synth.hidden_in(shape, SEED, 5000 + t, M) for t in range(min(K, 64))]
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for t in range(K):
+        pkg.head_top1_host(head, hosts[t % len(hosts)], sptr)
+    e2e_s = time.perf_counter() - t0
+    if dist:
+        tt = torch.tensor([e2e_s], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        e2e_s = float(tt.item())
+    pkg.head_destroy(head)
+    if rank != 0:
+        if dist:
+            dist.destroy_process_group()
+        return
+    peaks = measured_peaks()
+    peak = peaks.get("hbm_gbs")
+    peak_note = "of measured" if peak else "of fallback"
+    if not peak:
+        peak = 6800.0
+    call_bytes = hw.packed_bytes() + H * 2 + M * H * 2 + M * 8  # weights, norm, hidden rows, (token, p_max)
+    call_s = ms / K / 1e3
+    result = {
+        "metric": HEAD_METRIC,
+        "value": world * K * M / (ms / 1e3),
+        "unit": "rows/s",
+        "n_gpus": world,
+        "steps": K,
+        "warmup": W,
+        "ms_per_step": ms / K,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "w4a16 (uint4 weights, fp16 activations, fp32 accumulate)",
+        "data": "synthetic (seeded Gaussian lm_head quantised to uint4, fp16 N(0,1) hidden rows)",
+        "config": {"workload": c["workload"], "rows_per_call": M,
+                   "l2": "no flush: each call streams %.0f MB of packed weights, larger than the 129 MB L2" % (
+                       hw.packed_bytes() / 1e6),
+                   "parallelism": "replicas" if world > 1 else "single GPU", "seed": SEED},
+        "call_alg_bytes": call_bytes,
+        "roofline": {
+            "kernel": "head_top1 call (norm + W4A16 projection + top-1 reduction; the projection dominates)",
+            "bound": "hbm",
+            "achieved": call_bytes / call_s / 1e9,
+            "peak": peak,
+            "unit": "GB/s",
+            "frac": call_bytes / call_s / 1e9 / peak,
+            "peak_note": "%s: MEASURED_PEAKS.json hbm_gbs; achieved = algorithmic bytes per call / CUDA-event "
+                         "time per call" % peak_note,
+            "traffic": profiled_traffic("head", args.config) if M == 1 else None,
+            "traffic_note": "DRAM bytes of the projection kernel per call (ncu), M = 1",
+        },
+        "e2e": {"value": world * K * M / e2e_s, "unit": "rows/s", "h2d_bytes_per_step": M * H * 2,
+                "d2h_bytes_per_step": M * 8},
+        "gpu_launches": 3 * K,
+        "clocks": clocks,
+    }
+    if world == 1 and not args.no_cpu_baseline:
+        result["cpu_baseline"] = head_cpu_baseline(hw, M, budget_s=args.cpu_budget)
+    print(json.dumps(result), flush=True)
+    if dist:
+        dist.destroy_process_group()
+
+
 def run_reference(args, rank: int, world: int):
     if rank != 0:
         return
     c = CONFIGS[args.config]
+    if "head" in c:
+        H, V, g = c["head"]
+        hw = synth.make_head(H, V, g, SEED)
+        cb = head_cpu_baseline(hw, c["rows"], budget_s=float(os.environ.get("REFERENCE_BUDGET_S", "60")))
+        print(json.dumps({
+            "metric": HEAD_METRIC, "value": cb["value"], "unit": "rows/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": 1000.0 * c["rows"] / cb["value"], "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic (seeded Gaussian lm_head quantised to uint4)",
+            "config": {"workload": c["workload"], "rows_per_call": c["rows"]}, "impl": "reference",
+            "cpu_baseline": cb,
+            "e2e": {"value": cb["value"], "unit": "rows/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        }), flush=True)
+        return
     shape = c["shape"]
     weights = synth.make_weights(shape, SEED)
     budget = float(os.environ.get("REFERENCE_BUDGET_S", "120"))
@@ -558,6 +732,8 @@ def main():
     rank = int(os.environ.get("RANK", "0"))
     if args.impl == "reference":
         run_reference(args, rank, world)
+    elif "head" in CONFIGS[args.config]:
+        run_head(args, rank, world)
     else:
         run_gpu(args, rank, world)
 
