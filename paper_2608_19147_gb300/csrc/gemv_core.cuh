@@ -57,6 +57,12 @@ __device__ __forceinline__ uint32_t hfma2_u32(uint32_t a, uint32_t b, uint32_t c
   asm("fma.rn.f16x2 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(c));
   return d;
 }
+// bytes of (a, b) picked by the four selector nibbles of c (0..3: a, 4..7: b)
+__device__ __forceinline__ uint32_t prmt_u32(uint32_t a, uint32_t b, uint32_t c) {
+  uint32_t d;
+  asm("prmt.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(c));
+  return d;
+}
 __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
@@ -201,7 +207,9 @@ __device__ __forceinline__ void mma_unit(const uint8_t* __restrict__ U, const ui
       const uint8_t* meta = U + kCodeBytes + gi * kMetaBytesPerGroup;
       if (blk % BPG == 0) {
         // group start: clear the group sums; zero points as fp16x2
-        // (1024 + z_lo) and -(64 + z_hi)
+        // (1024 + z_lo) = bits 0x6400 | z and -(64 + z_hi) = bits 0xD400 | 16 z,
+        // each one byte permute: the unit stores the upper rows' zero
+        // points as 16 z
 #pragma unroll
         for (int rt = 0; rt < 4; ++rt)
 #pragma unroll
@@ -211,11 +219,10 @@ __device__ __forceinline__ void mma_unit(const uint8_t* __restrict__ U, const ui
         const uint2 zz = *reinterpret_cast<const uint2*>(meta + 128 + gid * 8);
 #pragma unroll
         for (int rt = 0; rt < 4; ++rt) {
-          const uint32_t zw = rt < 2 ? zz.x : zz.y;
-          const uint32_t zlo = (zw >> (16 * (rt & 1))) & 0xFFu;
-          const uint32_t zhi = (zw >> (16 * (rt & 1) + 8)) & 0xFFu;
-          zsub[rt] = (0x6400u | zlo) * 0x00010001u;
-          zfma[rt] = (0xD400u + 16u * zhi) * 0x00010001u;
+          const uint32_t zw = rt < 2 ? zz.x : zz.y;  // bytes: z_lo, 16 z_hi of tiles 2i, then 2i + 1
+          const uint32_t p = 2u * (rt & 1);
+          zsub[rt] = prmt_u32(zw, 0x64646464u, 0x4040u + p * 0x0101u);
+          zfma[rt] = prmt_u32(zw, 0xD4D4D4D4u, 0x4040u + (p + 1u) * 0x0101u);
         }
       }
       uint32_t b0[NT], b1[NT];
@@ -557,6 +564,7 @@ __device__ __noinline__ void gemv_phase(WarpStream<GPU>* ws_io, int op, const Ge
       for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
         for (int q = 0; q < 4; ++q) tot[rt][nt][q] = 0.f;
+#pragma unroll 2  // alternating activation registers instead of copies (measured ~1 % faster)
     for (; u < seg_end; ++u) {
       uint4 cur[NT][2][2];
 #pragma unroll

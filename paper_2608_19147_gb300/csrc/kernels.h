@@ -37,6 +37,9 @@ constexpr int kMaxRequests = 16;  // SHARD_MAX_REQUESTS
 //              64 fp16 scales then 64 uint8 zero points, each ordered
 //              [gid 0..7][rt 0..3][lo, hi] so one lane reads its 8 scales with
 //              one 16-byte load and its 8 zero points with one 8-byte load.
+//              The zero point z of an upper row (hi: rows 8..15 of a tile) is
+//              stored as 16 z, the low byte of the fp16 bits of -(64 + z), so
+//              the dequantisation builds both offsets with one byte permute.
 // Rows past the real ones and inputs past K carry code 0 / zero point 0 /
 // scale 0, or (inputs of a real group past K) the group's zero point, so they
 // contribute exactly 0.

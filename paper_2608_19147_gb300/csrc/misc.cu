@@ -65,7 +65,7 @@ __global__ void repack_meta_kernel(PackedOp op, const int* __restrict__ rowmap, 
     }
     uint8_t* meta = op.units + unit * op.unit_bytes + kCodeBytes + gu * kMetaBytesPerGroup;
     reinterpret_cast<uint16_t*>(meta)[idx] = s;
-    meta[128 + idx] = z;
+    meta[128 + idx] = hl ? static_cast<uint8_t>(z << 4) : z;  // upper rows: 16 z (see kernels.h)
   }
 }
 
@@ -89,7 +89,7 @@ __global__ void unpack_kernel(PackedOp op, float* out, int ld) {
     const uint8_t* meta = unit + kCodeBytes + gu * kMetaBytesPerGroup;
     const int idx = gid * 8 + rt * 2 + hl;
     const float s = h2f(reinterpret_cast<const uint16_t*>(meta)[idx]);
-    const int z = meta[128 + idx];
+    const int z = hl ? meta[128 + idx] >> 4 : meta[128 + idx];
     out[(size_t)nat * ld + k] = static_cast<float>(q - z) * s;
   }
 }
