@@ -228,6 +228,24 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(win)}
 
 
+def max_over_ranks(x: float, dist, device) -> float:
+    """The largest of every rank's value (the slowest replica's time); x
+    itself on a single process."""
+    if dist is None:
+        return x
+    import torch
+
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def replica_throughput(world: int, units_per_rank: float, seconds: float) -> float:
+    """Whole-job throughput of `world` independent replicas that each
+    processed units_per_rank units, timed by the slowest one."""
+    return world * units_per_rank / seconds
+
+
 def measured_peaks():
     try:
         return json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
@@ -374,10 +392,7 @@ def run_gpu(args, rank: int, world: int):
     sampler.stop()
     clocks = sampler.summary(w0, w1)
     pkg.shard_sync_status(sh, sptr)
-    if dist:
-        tt = torch.tensor([ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms = float(tt.item())
+    ms = max_over_ranks(ms, dist, dev)
     for st in sts + wst:
         pkg.kv_state_free(st)
 
@@ -427,10 +442,7 @@ def run_gpu(args, rank: int, world: int):
            + (s0["beam"].nbytes if s0["beam"] is not None else 0))
     d2h = out.nbytes
     e2e_s = t1 - t0
-    if dist:
-        tt = torch.tensor([e2e_s], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        e2e_s = float(tt.item())
+    e2e_s = max_over_ranks(e2e_s, dist, dev)
     for st in est:
         pkg.kv_state_free(st)
     pkg.shard_destroy(sh)
@@ -445,7 +457,7 @@ def run_gpu(args, rank: int, world: int):
     if not peak:
         peak = 6800.0
     rows_per_step = plan.M
-    value = world * K * rows_per_step / (ms / 1e3)
+    value = replica_throughput(world, K * rows_per_step, ms / 1e3)
     step_bytes = sum(plan.alg_bytes(t) for t in range(K)) / K
     launches_per_step = 1  # the whole step is one kernel
     result = {
@@ -488,7 +500,7 @@ def run_gpu(args, rank: int, world: int):
             "frac_of_8tbs_nominal": step_bytes / (ms / K * 1e6) / 8000.0,
         },
         "phases": phases,
-        "e2e": {"value": world * K * rows_per_step / e2e_s, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
+        "e2e": {"value": replica_throughput(world, K * rows_per_step, e2e_s), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
         "gpu_launches": K * launches_per_step,
         "clocks": clocks,
@@ -612,10 +624,7 @@ def run_head(args, rank: int, world: int):
     ms = e0.elapsed_time(e1)
     sampler.stop()
     clocks = sampler.summary(w0, w1)
-    if dist:
-        tt = torch.tensor([ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms = float(tt.item())
+    ms = max_over_ranks(ms, dist, dev)
     # end to end: host hidden rows in, host (token, p_max) out, every call
     hosts = [synth.hidden_in(shape, SEED, 5000 + t, M) for t in range(min(K, 64))]
     torch.cuda.synchronize()
@@ -623,10 +632,7 @@ def run_head(args, rank: int, world: int):
     for t in range(K):
         pkg.head_top1_host(head, hosts[t % len(hosts)], sptr)
     e2e_s = time.perf_counter() - t0
-    if dist:
-        tt = torch.tensor([e2e_s], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        e2e_s = float(tt.item())
+    e2e_s = max_over_ranks(e2e_s, dist, dev)
     pkg.head_destroy(head)
     if rank != 0:
         if dist:
@@ -641,7 +647,7 @@ def run_head(args, rank: int, world: int):
     call_s = ms / K / 1e3
     result = {
         "metric": HEAD_METRIC,
-        "value": world * K * M / (ms / 1e3),
+        "value": replica_throughput(world, K * M, ms / 1e3),
         "unit": "rows/s",
         "n_gpus": world,
         "steps": K,
@@ -669,7 +675,7 @@ def run_head(args, rank: int, world: int):
             "traffic": profiled_traffic("head", args.config) if M == 1 else None,
             "traffic_note": "DRAM bytes of the projection kernel per call (ncu), M = 1",
         },
-        "e2e": {"value": world * K * M / e2e_s, "unit": "rows/s", "h2d_bytes_per_step": M * H * 2,
+        "e2e": {"value": replica_throughput(world, K * M, e2e_s), "unit": "rows/s", "h2d_bytes_per_step": M * H * 2,
                 "d2h_bytes_per_step": M * 8},
         "gpu_launches": 3 * K,
         "clocks": clocks,
