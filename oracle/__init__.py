@@ -94,6 +94,8 @@ def _load():
             lib.or_trim.restype = ip
             lib.or_step.argtypes = [vp, vp, vp, vp, vp, ip, vp, vp, ip, vp, ip, vp, vp]
             lib.or_step.restype = ip
+            lib.or_step_packed.argtypes = [vp, vp, vp, vp, ip, vp, vp, ip, ip, vp, vp]
+            lib.or_step_packed.restype = ip
             lib.or_logits.argtypes = [vp, ip, ip, vp, ip, dp, vp]
             lib.or_head_top1.argtypes = [vp, ip, ip, vp, dp, ctypes.POINTER(_Matrix), ip, ip, ip, vp, vp, vp, vp]
             _lib = lib
@@ -305,4 +307,21 @@ class OracleState:
         out64 = np.zeros((M, s.hidden), dtype=np.float64) if want_f64 else None
         rc = _load().or_step(self.shard._h, self._h, _p(hid), _p(tok), _p(n), len(n), _p(pos), _p(msk),
                              msk.shape[1], _p(beam), 1 if round_points else 0, _p(out16), _p(out64))
+        return int(rc), out16, out64
+
+    def step_packed(self, position_ids: np.ndarray, mask2d: np.ndarray, *, hidden_in: Optional[np.ndarray] = None,
+                    token_ids: Optional[np.ndarray] = None, round_points: bool = True, want_f64: bool = False):
+        """Packed step (Section 8.6): S rows on cache row 0, token t seeing
+        the entries j with mask2d[t][j] != 0.  Returns (rc, out16, out64)."""
+        s = self.shard.shape
+        pos = np.ascontiguousarray(position_ids, dtype=np.int32)
+        S = int(pos.size)
+        msk = np.ascontiguousarray(mask2d, dtype=np.uint8)
+        assert msk.ndim == 2 and msk.shape[0] == S
+        hid = None if hidden_in is None else np.ascontiguousarray(hidden_in, dtype=np.uint16)
+        tok = None if token_ids is None else np.ascontiguousarray(token_ids, dtype=np.int32)
+        out16 = np.zeros((S, s.hidden), dtype=np.uint16)
+        out64 = np.zeros((S, s.hidden), dtype=np.float64) if want_f64 else None
+        rc = _load().or_step_packed(self.shard._h, self._h, _p(hid), _p(tok), S, _p(pos), _p(msk), msk.shape[1],
+                                    1 if round_points else 0, _p(out16), _p(out64))
         return int(rc), out16, out64

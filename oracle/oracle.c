@@ -20,6 +20,10 @@
  *    caller's position_ids (logical positions), not the cache index.
  *  - Physical trim [Section 5.1]: or_trim deletes entries and shifts the
  *    rest down, the operation the mask replaces.
+ *  - Packed step [Section 8.6]: or_step_packed runs S query rows over one
+ *    cache row with a mask row per query, so slots (regions of the row, an
+ *    optional shared prefix) are isolated and same-slot rows form causal
+ *    chunks -- continuous batching expressed by the mask layout alone.
  *  - INT4 weights [Section 3.2, Step 4]: W[o][i] = (q - z) * s with uint4
  *    codes q, uint4 zero point z and fp16 scale s per (row, group of inputs).
  *  - Layer math (Llama, Section 3.2 Step 2's attention with precomputed
@@ -359,9 +363,9 @@ int or_trim(or_state* st, int row, const uint8_t* keep, int len) {
  * Output: fp16 [M][H] (round_points or not) and, if out64 is given, the
  * un-rounded fp64 residual stream.
  */
-int or_step(const or_shard* sh, or_state* st, const uint16_t* hidden_in, const int32_t* token_ids,
-            const int32_t* n_new, int B, const int32_t* position_ids, const uint8_t* mask, int mask_stride,
-            const int32_t* beam_idx, int round_points, uint16_t* out16, double* out64) {
+static int step_core(const or_shard* sh, or_state* st, const uint16_t* hidden_in, const int32_t* token_ids,
+                     const int32_t* n_new, int B, const int32_t* position_ids, const uint8_t* mask, int mask_stride,
+                     const int32_t* beam_idx, int round_points, uint16_t* out16, double* out64, int packed) {
     if (!sh || !st || !n_new || !position_ids || !mask || B < 1 || B > st->n_rows) return OR_EINVAL;
     const or_config* c = &sh->cfg;
     const int H = c->hidden, Hq = c->n_heads, Hkv = c->n_kv_heads, d = c->head_dim, F = c->ffn;
@@ -399,13 +403,16 @@ int or_step(const or_shard* sh, or_state* st, const uint16_t* hidden_in, const i
         free(tk); free(tv); free(tl);
     }
 
-    /* Validate capacity and the mask on the new entries. */
+    /* Validate capacity and the mask on the new entries (packed: the mask
+       has one row per token, and each token must open its own entry). */
     for (int b = 0; b < B; ++b) {
         int P = st->len[b];
         if (P + n_new[b] > st->capacity) { free(req); free(idx); return OR_ECAP; }
         if (P + n_new[b] > mask_stride) { free(req); free(idx); return OR_EINVAL; }
-        for (int i = 0; i < n_new[b]; ++i)
-            if (!mask[(size_t)b * mask_stride + P + i]) { free(req); free(idx); return OR_EINVAL; }
+        for (int i = 0; i < n_new[b]; ++i) {
+            const size_t r = packed ? (size_t)i : (size_t)b;
+            if (!mask[r * mask_stride + P + i]) { free(req); free(idx); return OR_EINVAL; }
+        }
     }
 
     double* x = (double*)malloc(sizeof(double) * (size_t)M * H);      /* residual stream */
@@ -450,8 +457,11 @@ int or_step(const or_shard* sh, or_state* st, const uint16_t* hidden_in, const i
             }
         }
         for (int t = 0; t < M; ++t) {
-            int b = req[t], last = P0[b] + idx[t]; /* attends to j <= last */
-            for (int j = 0; j <= last; ++j) vis[j] = mask[(size_t)b * mask_stride + j] ? 1 : 0;
+            /* per request: entries j <= P_b + i with mask[b][j] = 1;
+               packed: every entry of the row (old and new) with mask[t][j] = 1 */
+            int b = req[t], last = packed ? P0[b] + n_new[b] - 1 : P0[b] + idx[t];
+            for (int j = 0; j <= last; ++j)
+                vis[j] = mask[(size_t)(packed ? t : b) * mask_stride + j] ? 1 : 0;
             for (int h = 0; h < Hq; ++h) {
                 int hk = h / grp;
                 const double* K = st->k + kv_off(st, b, l, 0) + hk * d;
@@ -482,6 +492,36 @@ int or_step(const or_shard* sh, or_state* st, const uint16_t* hidden_in, const i
     free(x); free(xn); free(q); free(kk); free(vv); free(att); free(y); free(g); free(u);
     free(vis); free(P0); free(req); free(idx);
     return OR_OK;
+}
+
+int or_step(const or_shard* sh, or_state* st, const uint16_t* hidden_in, const int32_t* token_ids,
+            const int32_t* n_new, int B, const int32_t* position_ids, const uint8_t* mask, int mask_stride,
+            const int32_t* beam_idx, int round_points, uint16_t* out16, double* out64) {
+    return step_core(sh, st, hidden_in, token_ids, n_new, B, position_ids, mask, mask_stride, beam_idx, round_points,
+                     out16, out64, 0);
+}
+
+/*
+ * Packed step (Section 8.6, continuous batching through the mask layout):
+ * S query rows share ONE cache row (row 0 of the state), whose entries the
+ * host has partitioned into regions -- an optional shared prefix, then one
+ * region per slot.  The S new entries are appended after the existing ones,
+ * token t at index P + t, and token t attends to exactly the entries j < P + S
+ * with mask2d[t][j] != 0 (mask2d [S][mask_stride]): its own slot's region,
+ * the shared prefix, and the new entries of its own slot at or before it, so
+ * that several rows of one slot form a causal chunk and rows of different
+ * slots are isolated.  Every token must open its own new entry (an idle row
+ * opens only that one; a fully masked row would have no softmax).  RoPE uses
+ * position_ids, each slot's absolute positions.  Otherwise the layer math is
+ * that of or_step.
+ */
+int or_step_packed(const or_shard* sh, or_state* st, const uint16_t* hidden_in, const int32_t* token_ids, int S,
+                   const int32_t* position_ids, const uint8_t* mask2d, int mask_stride, int round_points,
+                   uint16_t* out16, double* out64) {
+    if (S < 1) return OR_EINVAL;
+    const int32_t n_new[1] = {S};
+    return step_core(sh, st, hidden_in, token_ids, n_new, 1, position_ids, mask2d, mask_stride, NULL, round_points,
+                     out16, out64, 1);
 }
 
 /* Test head for greedy-token checks (not part of the shard): logits of the
