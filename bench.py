@@ -516,7 +516,7 @@ def run_gpu(args, rank: int, world: int):
 # CPU oracle arm
 # ---------------------------------------------------------------------------
 
-def cpu_baseline(cfg_name: str, weights, budget_s: float = 20.0, max_steps: int = 256):
+def cpu_baseline(cfg_name: str, weights, budget_s: float = 20.0, max_steps: int = 256, one_thread: bool = True):
     """The fp64 CPU oracle, as it stands, on a bounded sample of the workload:
     the first steps of one request, until about budget_s seconds of work."""
     import oracle
@@ -548,7 +548,7 @@ def cpu_baseline(cfg_name: str, weights, budget_s: float = 20.0, max_steps: int 
     # the same oracle on one thread: the next steps of the request, when one
     # step fits in the budget
     est = el / max(n, 1) * threads
-    if threads > 1 and n < min(max_steps, plan.spr) and est <= 1.5 * budget_s:
+    if one_thread and threads > 1 and n < min(max_steps, plan.spr) and est <= 1.5 * budget_s:
         oracle.set_threads(1)
         n1 = 0
         t1 = time.perf_counter()
@@ -728,7 +728,7 @@ def run_reference(args, rank: int, world: int):
     shape = c["shape"]
     weights = synth.make_weights(shape, SEED)
     budget = float(os.environ.get("REFERENCE_BUDGET_S", "120"))
-    cb = cpu_baseline(args.config, weights, budget_s=budget, max_steps=args.steps)
+    cb = cpu_baseline(args.config, weights, budget_s=budget, max_steps=args.steps, one_thread=False)
     result = {
         "metric": METRIC, "value": cb["value"], "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": 1000.0 * CONFIGS[args.config]["rows"] * c["n"] / cb["value"],
