@@ -247,6 +247,25 @@ class ShardWeights:
         return sum(m.nbytes() for lw in self.layers for m in lw.matrices)
 
 
+def layer_weights(shape: ShardShape, seed: int, layer: int, threads: Optional[int] = None) -> LayerWeights:
+    """The seeded weights of one layer of a shard (its own streams: the same
+    values whether the layer is made alone or as part of the whole shard)."""
+    mats = []
+    for mi, name in enumerate(MATRIX_NAMES):
+        r, c = shape.matrix_shape(name)
+        mats.append(quant_matrix(r, c, shape.group, shape.weight_sigma, seed=seed,
+                                 stream=layer * 16 + mi, tag=TAG_WEIGHT, threads=threads))
+    an = normal(shape.hidden, seed=seed, stream=layer * 2, tag=TAG_NORM, mean=1.0, sigma=0.1, dtype=np.uint16)
+    fn = normal(shape.hidden, seed=seed, stream=layer * 2 + 1, tag=TAG_NORM, mean=1.0, sigma=0.1, dtype=np.uint16)
+    return LayerWeights(mats, an, fn)
+
+
+def embedding(shape: ShardShape, seed: int, threads: Optional[int] = None) -> np.ndarray:
+    """The seeded token embedding of a first-stage shard (fp16 N(0,1) bits [V][H])."""
+    return normal(shape.vocab * shape.hidden, seed=seed, stream=0, tag=TAG_EMBED,
+                  dtype=np.uint16, threads=threads).reshape(shape.vocab, shape.hidden)
+
+
 def make_weights(shape: ShardShape, seed: int, threads: Optional[int] = None, n_layers: Optional[int] = None) -> ShardWeights:
     """Seeded weights for a shard: per layer q,k,v,o,gate,up,down ~ N(0, sigma^2)
     quantised to uint4 (group = shape.group); norm weights fp16(1 + 0.1 N(0,1));
@@ -254,17 +273,9 @@ def make_weights(shape: ShardShape, seed: int, threads: Optional[int] = None, n_
     sw = ShardWeights(shape, seed)
     L = shape.n_layers if n_layers is None else n_layers
     for layer in range(L):
-        mats = []
-        for mi, name in enumerate(MATRIX_NAMES):
-            r, c = shape.matrix_shape(name)
-            mats.append(quant_matrix(r, c, shape.group, shape.weight_sigma, seed=seed,
-                                     stream=layer * 16 + mi, tag=TAG_WEIGHT, threads=threads))
-        an = normal(shape.hidden, seed=seed, stream=layer * 2, tag=TAG_NORM, mean=1.0, sigma=0.1, dtype=np.uint16)
-        fn = normal(shape.hidden, seed=seed, stream=layer * 2 + 1, tag=TAG_NORM, mean=1.0, sigma=0.1, dtype=np.uint16)
-        sw.layers.append(LayerWeights(mats, an, fn))
+        sw.layers.append(layer_weights(shape, seed, layer, threads))
     if shape.vocab > 0:
-        sw.embedding = normal(shape.vocab * shape.hidden, seed=seed, stream=0, tag=TAG_EMBED,
-                              dtype=np.uint16, threads=threads).reshape(shape.vocab, shape.hidden)
+        sw.embedding = embedding(shape, seed, threads)
     return sw
 
 
