@@ -16,7 +16,7 @@ so every step is a step of that workload.  Weights are seeded synthetic
 far larger than L2, so no L2 flush is needed between steps.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl gb300|reference]
-                  [--config 8b-decode|8b-verify|8b-microbatch|70b-decode|70b-verify|tiny|8b-head|8b-head-verify]
+                  [--config 8b-decode|8b-verify|8b-microbatch|70b-decode|70b-verify|tiny|8b-head|8b-head-verify|8b-prefill]
 
 Under torchrun each rank runs an independent replica on its own GPU
 (replicas only: the path has no exchange step) and rank 0 prints one JSON
@@ -70,8 +70,13 @@ CONFIGS = {
     "8b-head-verify": dict(head=(4096, 128256, 128), rows=5,
                            workload="llama3.1-8b final-stage LM head, top-1: RMSNorm + 128256x4096 INT4 lm_head + "
                                     "argmax/p_max, 1+4 verify rows per call"),
+    # prefill of a prompt through the stage (Section 3.4), projections on the tensor cores
+    "8b-prefill": dict(prefill_tokens=512, shape=synth.LLAMA8B_STAGE, rows=512,
+                       workload="llama3.1-8b-stage1of2 16L prefill: one 512-token prompt (token ids) onto an empty "
+                                "row per call, chunks of 256 tokens, projections as tcgen05 GEMMs"),
 }
 HEAD_METRIC = "LM-head top-1 rows/s at 1 GB300 (final stage, Section 6.7); achieved HBM GB/s"
+PREFILL_METRIC = "INT4 shard prefill tokens/s at 1 GB300; achieved tensor TFLOP/s of the projections"
 
 
 def log(*a):
@@ -402,16 +407,17 @@ def run_gpu(args, rank: int, world: int):
     pplan = Plan(args.config, prof_K, SEED + 2, shape=shape)
     pst, pd = load_states(pplan), stage(pplan)
     PHASES = list(pkg.PHASES)
-    n_ph = len(PHASES) * shape.n_layers
+    n_ph = len(PHASES) * shape.n_layers + 1
     acc = np.zeros(n_ph)
     for t in range(prof_K):
         run_steps_one(pplan, pst, pd, t)
         acc += np.array(pkg.shard_debug_phase_times(sh, shape.n_layers))
     acc /= prof_K
-    # times[0] is the prologue, then the phases of every layer (the last
-    # layer's down phase ends with the kernel, not at a barrier)
-    phases = {"prologue": {"total_us_per_step": float(acc[0])}}
-    lay = acc[1:].tolist() + [0.0]
+    # times[0]: the prologue with the first RMSNorm and q|k|v projection;
+    # then per layer: attention (after the first layer, with that layer's
+    # RMSNorm and q|k|v projection in front), o, RMSNorm + gate|up, down
+    phases = {"prologue_norm_qkv0": {"total_us_per_step": float(acc[0])}}
+    lay = acc[1:].tolist()
     for i, name in enumerate(PHASES):
         v = np.array(lay[i::len(PHASES)])
         phases[name] = {"avg_us_per_layer": float(v.mean()), "total_us_per_step": float(v.sum())}
@@ -483,6 +489,9 @@ def run_gpu(args, rank: int, world: int):
             "requests_chained": plan.R,
             "l2": "no flush: each step streams %.2f GB of packed weights, far larger than the 129 MB L2" % (
                 plan.weight_bytes() / 1e9),
+            "inputs": "value: every step's inputs (token ids or hidden rows, positions, mask rows, beam_idx) are "
+                      "resident in HBM before the timed region, which holds only the step launches; e2e times "
+                      "the same steps through shard_step_host with each step's uploads and the output read-back",
             "parallelism": "replicas" if world > 1 else "single GPU",
             "seed": SEED,
         },
@@ -707,6 +716,221 @@ def run_head(args, rank: int, world: int):
         dist.destroy_process_group()
 
 
+def run_prefill(args, rank: int, world: int):
+    """Prefill throughput (shard_prefill) and the tensor-core projection
+    against the decode path's GEMV at small token counts."""
+    import torch
+
+    import paper_2608_19147_gb300 as pkg
+
+    dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", "0")))
+    torch.cuda.set_device(dev)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.init_process_group("nccl", device_id=dev)
+    c = CONFIGS[args.config]
+    shape = c["shape"]
+    if args.layers:
+        shape = dataclasses.replace(shape, n_layers=args.layers)
+    S = c["prefill_tokens"]
+    K, W = args.steps, max(3, args.warmup)
+    t0 = time.time()
+    weights = synth.make_weights(shape, SEED)
+    log("weights generated in %.1fs" % (time.time() - t0))
+    sh = pkg.shard_create(pkg.make_config(shape), weights.layers, weights.embedding)
+    stream = torch.cuda.current_stream(dev)
+    sptr = stream.cuda_stream
+    n_st = min(K + W, 16)  # states cycled (each call prefills an empty row; reset outside the timed region)
+    sts = [pkg.kv_state_alloc(sh, 1, S + 8) for _ in range(n_st)]
+    tok = torch.from_numpy(synth.token_ids(shape, SEED, 0, S).astype(np.int32)).to(dev)
+    pos = torch.arange(S, dtype=torch.int32, device=dev)
+    mask = torch.ones(S, dtype=torch.uint8, device=dev)
+    out = torch.empty((S, shape.hidden), dtype=torch.int16, device=dev)
+
+    def call(st):
+        pkg.shard_prefill(sh, st, 0, None, tok.data_ptr(), S, pos.data_ptr(), mask.data_ptr(), S, out.data_ptr(), sptr)
+
+    for i in range(W):
+        call(sts[i % n_st])
+    torch.cuda.synchronize()
+    for st in sts:
+        pkg.kv_state_reset(st, -1)
+    gpu_id = ""
+    try:
+        gpu_id = str(torch.cuda.get_device_properties(dev).uuid)
+        if gpu_id and not gpu_id.startswith("GPU-"):
+            gpu_id = "GPU-" + gpu_id
+    except Exception:
+        gpu_id = ""
+    ms_total, done = 0.0, 0
+    clocks = None
+    while done < K:
+        n = min(n_st, K - done)
+        sampler = ClockSampler(gpu_id)
+        time.sleep(0.2)
+        torch.cuda.synchronize()
+        if dist:
+            dist.barrier()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        w0 = time.time()
+        e0.record(stream)
+        for i in range(n):
+            call(sts[i])
+        e1.record(stream)
+        torch.cuda.synchronize()
+        w1 = time.time()
+        sampler.stop()
+        clocks = clocks or sampler.summary(w0, w1)
+        ms_total += e0.elapsed_time(e1)
+        done += n
+        for st in sts[:n]:
+            pkg.kv_state_reset(st, -1)
+    pkg.shard_sync_status(sh, sptr)
+    ms = max_over_ranks(ms_total, dist, dev)
+    # the dominant kernel, the tensor-core projection, timed alone per 256-token chunk on layer 0
+    chunk = 256
+    proj = {}
+    flops_chunk, ms_chunk = 0.0, 0.0
+    for k, name in ((pkg.OP_QKV, "qkv"), (pkg.OP_O, "o"), (pkg.OP_GU, "gate_up"), (pkg.OP_DOWN, "down")):
+        rows, Kin, _ = pkg.shard_debug_op_info(sh, 0, k)
+        ld = (Kin + 127) // 128 * 128
+        x = torch.zeros((chunk, ld), dtype=torch.int16, device=dev)
+        x[:, :Kin] = torch.from_numpy(synth.hidden_in(dataclasses.replace(shape, hidden=Kin), SEED, 9, chunk).view(np.int16))
+        y = torch.empty((chunk, rows), dtype=torch.float32, device=dev)
+        for _ in range(3):
+            pkg.shard_debug_gemm(sh, 0, k, x.data_ptr(), ld, chunk, y.data_ptr(), rows, sptr)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        reps = 20
+        torch.cuda.synchronize()
+        e0.record(stream)
+        for _ in range(reps):
+            pkg.shard_debug_gemm(sh, 0, k, x.data_ptr(), ld, chunk, y.data_ptr(), rows, sptr)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        t_ms = e0.elapsed_time(e1) / reps
+        fl = 2.0 * rows * Kin * chunk
+        proj[name] = {"us_per_call": t_ms * 1e3, "tflops": fl / (t_ms * 1e9)}
+        flops_chunk += fl
+        ms_chunk += t_ms
+    # the same projection at decode-sized token counts: the decode step's
+    # mma.sync GEMV against the tcgen05 GEMM (gate|up of layer 0)
+    rows, Kin, nbytes = pkg.shard_debug_op_info(sh, 0, pkg.OP_GU)
+    ld = (Kin + 127) // 128 * 128
+    cmp_m = {}
+    for M in (1, 5, 8, 16):
+        x = torch.zeros((M, ld), dtype=torch.int16, device=dev)
+        x[:, :Kin] = torch.from_numpy(synth.hidden_in(shape, SEED, 11, M).view(np.int16))
+        y = torch.empty((M, rows), dtype=torch.float32, device=dev)
+        xk = x[:, :Kin].contiguous()
+        res = {}
+        for nm, fn in (("mma_sync_gemv", lambda: pkg.shard_debug_gemv(sh, 0, pkg.OP_GU, xk.data_ptr(), M, y.data_ptr(),
+                                                                        rows, sptr)),
+                       ("tcgen05_gemm", lambda: pkg.shard_debug_gemm(sh, 0, pkg.OP_GU, x.data_ptr(), ld, M,
+                                                                       y.data_ptr(), rows, sptr))):
+            for _ in range(3):
+                fn()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            torch.cuda.synchronize()
+            e0.record(stream)
+            for _ in range(20):
+                fn()
+            e1.record(stream)
+            torch.cuda.synchronize()
+            t_ms = e0.elapsed_time(e1) / 20
+            res[nm] = {"us_per_call": t_ms * 1e3, "weight_gbs": nbytes / (t_ms * 1e6)}
+        cmp_m["M=%d" % M] = res
+    for st in sts:
+        pkg.kv_state_free(st)
+    # end to end: token ids from pinned host memory in, hidden states out, every call
+    htok = torch.from_numpy(synth.token_ids(shape, SEED, 0, S).astype(np.int32)).pin_memory()
+    hout = torch.empty((S, shape.hidden), dtype=torch.int16).pin_memory()
+    st = pkg.kv_state_alloc(sh, 1, S + 8)
+    n_e2e = min(K, 4)
+    e2e_s = 0.0
+    for i in range(n_e2e):
+        torch.cuda.synchronize()
+        a = time.perf_counter()
+        tok.copy_(htok, non_blocking=True)
+        call(st)
+        hout.copy_(out, non_blocking=True)
+        torch.cuda.synchronize()
+        e2e_s += time.perf_counter() - a
+        pkg.kv_state_reset(st, -1)
+    pkg.kv_state_free(st)
+    pkg.shard_destroy(sh)
+    if rank != 0:
+        if dist:
+            dist.destroy_process_group()
+        return
+    peaks = measured_peaks()
+    peak = peaks.get("bf16_tflops")
+    peak_note = "of measured (MEASURED_PEAKS.json bf16_tflops, burst; fp16 has the same dense rate)"
+    if not peak:
+        peak, peak_note = 1900.0, "of fallback (1.9 PFLOP/s bf16 burst)"
+    result = {
+        "metric": PREFILL_METRIC,
+        "value": replica_throughput(world, K * S, ms / 1e3),
+        "unit": "tokens/s",
+        "n_gpus": world,
+        "steps": K,
+        "warmup": W,
+        "ms_per_step": ms / K,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "w4a16 (uint4 weights, fp16 activations, fp32 accumulate)",
+        "data": "synthetic (seeded Gaussian weights quantised to uint4; seeded token ids)",
+        "config": {"workload": c["workload"], "tokens_per_call": S,
+                   "shard": "%s: %d layers" % (shape.name, shape.n_layers),
+                   "l2": "no flush: each call streams the %.2f GB of packed weights twice (two chunks)" % (
+                       shape.packed_bytes_per_layer() * shape.n_layers / 1e9),
+                   "parallelism": "replicas" if world > 1 else "single GPU", "seed": SEED},
+        "roofline": {
+            "kernel": "gemm_tc (W4A16 projection, tcgen05.mma kind::f16 M=128, N=128 tokens, accumulator in TMEM), "
+                      "one 256-token chunk of each projection of layer 0, timed alone",
+            "bound": "tensor",
+            "achieved": flops_chunk / (ms_chunk * 1e9),
+            "peak": peak,
+            "unit": "TFLOP/s",
+            "frac": flops_chunk / (ms_chunk * 1e9) / peak,
+            "peak_note": peak_note,
+            "traffic": None,
+            "per_projection": proj,
+        },
+        "projection_gate_up_small_m": cmp_m,
+        "e2e": {"value": replica_throughput(world, n_e2e * S, e2e_s), "unit": "tokens/s", "h2d_bytes_per_step": S * 4,
+                "d2h_bytes_per_step": S * shape.hidden * 2},
+        "gpu_launches": K * (2 + shape.n_layers * 11 * 2 + 1),
+        "clocks": clocks,
+    }
+    if world == 1 and not args.no_cpu_baseline:
+        result["cpu_baseline"] = prefill_cpu_baseline(shape, weights, budget_s=args.cpu_budget)
+    print(json.dumps(result), flush=True)
+    if dist:
+        dist.destroy_process_group()
+
+
+def prefill_cpu_baseline(shape, weights, budget_s: float = 20.0):
+    """The oracle's step with a prompt of tokens as the new tokens of one
+    request, on the host cores: a bounded prompt length, scaled to tokens/s."""
+    import oracle
+    oracle.build()
+    oracle.set_threads(os.cpu_count() or 1)
+    shard = oracle.OracleShard(shape, weights)
+    n = 8
+    st = shard.state(1, n + 8)
+    tok = synth.token_ids(shape, SEED, 0, n)
+    t0 = time.perf_counter()
+    st.step([n], np.arange(n, dtype=np.int32), np.ones(n, np.uint8), token_ids=tok)
+    dt = time.perf_counter() - t0
+    return {"value": n / dt, "unit": "tokens/s", "cores": os.cpu_count() or 1, "kind": "oracle",
+            "sample": "one %d-token prompt through the %d-layer stage (fp64 oracle, OpenMP over output rows), "
+                      "%.1f s" % (n, shape.n_layers, dt)}
+
+
 def run_reference(args, rank: int, world: int):
     if rank != 0:
         return
@@ -727,6 +951,18 @@ def run_reference(args, rank: int, world: int):
         return
     shape = c["shape"]
     weights = synth.make_weights(shape, SEED)
+    if "prefill_tokens" in c:
+        cb = prefill_cpu_baseline(shape, weights)
+        print(json.dumps({
+            "metric": PREFILL_METRIC, "value": cb["value"], "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": 1000.0 * c["prefill_tokens"] / cb["value"], "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic (seeded Gaussian weights quantised to uint4; seeded token ids)",
+            "config": {"workload": c["workload"], "tokens_per_call": c["prefill_tokens"]}, "impl": "reference",
+            "cpu_baseline": cb,
+            "e2e": {"value": cb["value"], "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        }), flush=True)
+        return
     budget = float(os.environ.get("REFERENCE_BUDGET_S", "120"))
     cb = cpu_baseline(args.config, weights, budget_s=budget, max_steps=args.steps, one_thread=False)
     result = {
@@ -760,6 +996,8 @@ def main():
         run_reference(args, rank, world)
     elif "head" in CONFIGS[args.config]:
         run_head(args, rank, world)
+    elif "prefill_tokens" in CONFIGS[args.config]:
+        run_prefill(args, rank, world)
     else:
         run_gpu(args, rank, world)
 

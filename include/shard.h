@@ -111,25 +111,30 @@ int shard_destroy(shard_t shard);
 int kv_state_alloc(shard_t shard, int n_rows, int capacity, kvstate_t* out);
 int kv_state_free(kvstate_t state);
 
-/* Empties one row (row >= 0) or all rows (row == -1).  A single row can only
- * be reset while no other row shares its cache entries, i.e. before any step
- * with a non-NULL beam_idx since the last full reset (else EUNSUPPORTED). */
+/* Empties one row (row >= 0) or all rows (row == -1): the stateful cache of
+ * Section 3.4 starts a new sequence.  Also clears a state that a rejected
+ * step left unusable.  A single row can only be reset while no other row
+ * shares its cache entries, i.e. before any step with a non-NULL beam_idx
+ * since the last full reset (else EUNSUPPORTED).  Synchronous.  Errors:
+ * EINVAL (row out of range), EUNSUPPORTED. */
 int kv_state_reset(kvstate_t state, int row);
 
 /* Sets one layer of one row to `len` cache entries from host fp16 K and V,
- * each [len][Hkv][d]; the row's length becomes len (load every layer with the
- * same len).  Synchronous.  Errors: EINVAL, ECAPACITY (len > capacity),
+ * each [len][Hkv][d] (a prefilled cache, Section 3.4); the row's length
+ * becomes len (load every layer with the same len).  Synchronous.  Errors: EINVAL, ECAPACITY (len > capacity),
  * EUNSUPPORTED (row entries shared through a beam gather; reset first). */
 int kv_state_load(kvstate_t state, int row, int layer, const uint16_t* k, const uint16_t* v, int len);
 
 /* Copies cache entries [start, start+len) of one row and layer, in the row's
- * own (logical) order, into host fp16 K and V [len][Hkv][d].  Synchronous
+ * own (logical) order -- through the beam table, as the step's attention
+ * reads them (Section 4) -- into host fp16 K and V [len][Hkv][d]; what a
+ * masked-rewind run is compared with against a physical trim (Section 5.2).  Synchronous
  * (waits for all work on the legacy default stream and the shard's streams
  * to finish by synchronising the device).  Errors: EINVAL. */
 int kv_state_read(kvstate_t state, int row, int layer, int start, int len, uint16_t* k, uint16_t* v);
 
-/* The row's current cache length (entries, including masked ones).
- * Synchronous.  Errors: EINVAL. */
+/* The row's current cache length (entries, including masked ones: mask-based
+ * rewind, Section 5.2, never shortens a row).  Synchronous.  Errors: EINVAL. */
 int kv_state_length(kvstate_t state, int row, int* len);
 
 /* Physical trim (Section 5.1): removes the entries j < len with keep[j] == 0
@@ -161,8 +166,8 @@ int kv_state_import(kvstate_t state, int row, const uint16_t* k, const uint16_t*
  *   n_new        host int32 [B], n_new[b] >= 1 new tokens of request b;
  *                M = sum(n_new) <= SHARD_MAX_TOKENS.  Tokens of request b
  *                are consecutive, request 0 first.
- *   hidden_in    dev fp16 [M][H] input hidden states, or NULL when token_ids
- *                is given (exactly one of the two)
+ *   hidden_in    dev fp16 [M][H] input hidden states, 16-byte aligned, or
+ *                NULL when token_ids is given (exactly one of the two)
  *   token_ids    dev int32 [M], ids < vocab, looked up in the embedding
  *                (shards with vocab > 0 only; else EUNSUPPORTED)
  *   position_ids dev int32 [M], the RoPE positions (logical positions,
@@ -189,6 +194,44 @@ int shard_step(shard_t shard, kvstate_t state, const uint16_t* hidden_in, const 
                const int32_t* n_new, int B, const int32_t* position_ids, const uint8_t* attention_mask,
                int mask_stride, const int32_t* beam_idx, uint16_t* hidden_out, void* cuda_stream);
 
+/* Packed step (Section 8.6, continuous batching by the mask layout): S new
+ * tokens (1 <= S <= SHARD_MAX_TOKENS) on the single row of `state` (a state
+ * with n_rows == 1), whose entries the caller partitions into regions -- for
+ * example a shared prefix and one region per slot.  Token t is appended at
+ * entry P + t (P the row's length before the step) and attends to exactly the
+ * entries j < P + S with mask2d[t][j] != 0 (dev uint8 [S][mask_stride],
+ * mask_stride >= P + S); it must open its own entry P + t (else the device
+ * guard rejects the step, EINVAL).  Rows of one slot that open each other's
+ * earlier entries form a causal chunk; rows of different slots are isolated;
+ * an idle row opened only on its own entry affects nobody.  Other arguments
+ * as shard_step (position_ids are each row's absolute RoPE positions).
+ * Errors as shard_step. */
+int shard_step_packed(shard_t shard, kvstate_t state, const uint16_t* hidden_in, const int32_t* token_ids, int S,
+                      const int32_t* position_ids, const uint8_t* mask2d, int mask_stride, uint16_t* hidden_out,
+                      void* cuda_stream);
+
+/* Prefill of one row (Section 3.4: the prompt runs through the stage and
+ * fills its stateful cache): S >= 1 new tokens of request `row`, any number,
+ * appended at the row's entries P .. P + S - 1 (P its length).  The result
+ * is the one shard_step gives for S tokens of one request -- the same
+ * rounding points, causal attention among the new tokens and over the row's
+ * entries with mask != 0 -- computed with the projections as dense
+ * contractions on the tensor cores, in chunks of up to 256 tokens.
+ *   hidden_in / token_ids  as shard_step (exactly one), [S] rows
+ *   position_ids           dev int32 [S]
+ *   attention_mask         dev uint8 [mask_len], the row's mask, mask_len >=
+ *                          P + S, 1 at the new entries
+ *   hidden_out             dev fp16 [S][H]
+ * The row must hold its entries contiguously (no beam gather since the last
+ * full reset; else EUNSUPPORTED).  The first call allocates the library's
+ * prefill work buffers.  Device-side values (token ids, positions, the mask at
+ * the new entries) are checked on the device; a violation is reported by
+ * shard_sync_status or the next call as EINVAL.  Asynchronous on cuda_stream.
+ * Errors: EINVAL, ECAPACITY, EUNSUPPORTED, ENOMEM, ECUDA. */
+int shard_prefill(shard_t shard, kvstate_t state, int row, const uint16_t* hidden_in, const int32_t* token_ids, int S,
+                  const int32_t* position_ids, const uint8_t* attention_mask, int mask_len, uint16_t* hidden_out,
+                  void* cuda_stream);
+
 /* shard_step on HOST buffers: copies the inputs to the device (through
  * library-owned pinned staging buffers), runs the step on `cuda_stream`,
  * copies hidden_out back and waits for it.  Arguments as in shard_step, but
@@ -208,8 +251,9 @@ int shard_sync_status(shard_t shard, void* cuda_stream);
  * and forbids outside cudaMalloc, a thread that may not take the allocator's
  * lock, or a loop where an allocation's implicit synchronisation is not
  * allowed).  It runs the same kernel as the step's projections; the kernel's
- * scratch (cross-CTA partial sums, arrival counters, a zero-padded copy of x)
- * lives in one fixed 4 MiB device array inside the library, which every GPU
+ * scratch (the row sums of row-blocks split between warps, in 64-bit fixed
+ * point, the per-row-block counts of units added, and a zero-padded copy of
+ * x) lives in one fixed 4 MiB device array inside the library, which every GPU
  * that loads the library holds until the process exits.  The paper has no
  * counterpart; this is a deployment convenience.
  *   op      0 = q|k|v, 1 = o, 2 = gate|up, 3 = down (row order as in
@@ -217,11 +261,14 @@ int shard_sync_status(shard_t shard, void* cuda_stream);
  *   x       dev fp16 [M][K], K the op's input width, 1 <= M <= 16
  *   y       dev fp32 [M][y_ld], y_ld >= the op's natural row count
  * Calls larger than the fixed array (scratch for M tokens of K inputs and
- * the op's row-blocks) fail with ECAPACITY and a message giving the sizes.
+ * of the op's rows) fail with ECAPACITY and a message giving the sizes.  The
+ * kernel's own waits are bounded: one that runs out (never expected) sets the
+ * shard's status word, which shard_sync_status then reports as EINVAL.
  * The first call on each device resolves the array's device address (with
  * that device made current); make that first call before any stream capture.
  * Every call on a device shares the one array and it keeps the last call's
- * contents (the call zeroes what must start at zero): calls whose work
+ * contents (each call clears the counts, sums and padding on its stream before
+ * its kernel runs): calls whose work
  * overlaps on the GPU -- different streams, or different host threads --
  * race and corrupt each other's results.  Asynchronous on cuda_stream; it
  * does not synchronise. */

@@ -26,12 +26,15 @@ OP_QKV, OP_O, OP_GU, OP_DOWN = 0, 1, 2, 3
 
 # Every symbol include/shard.h and include/shard_debug.h declare.
 EXPORTS = ("shard_create", "shard_destroy", "kv_state_alloc", "kv_state_free", "kv_state_reset", "kv_state_load",
-           "kv_state_read", "kv_state_length", "kv_trim", "kv_state_export", "kv_state_import", "shard_step", "shard_step_host", "shard_sync_status",
-           "shard_last_error", "shard_debug_op_info", "shard_debug_unpack", "shard_debug_gemv",
-           "shard_debug_phase_times", "shard_gemv_noalloc", "head_create", "head_destroy", "head_top1",
+           "kv_state_read", "kv_state_length", "kv_trim", "kv_state_export", "kv_state_import", "shard_step", "shard_step_packed", "shard_prefill", "shard_step_host", "shard_sync_status",
+           "shard_last_error", "shard_debug_op_info", "shard_debug_unpack", "shard_debug_gemv", "shard_debug_gemm",
+           "shard_debug_phase_times", "shard_debug_set_wait", "shard_gemv_noalloc", "head_create", "head_destroy", "head_top1",
            "head_top1_host", "head_debug_logits")
-# per layer, between grid barriers: RMSNorm + q|k|v + attention, o, RMSNorm + gate|up, down
-PHASES = ("qkv_attention", "o", "gate_up", "down")
+# per layer, between the ends of grid-barrier waits: attention (with the next
+# layer's RMSNorm + q|k|v projection in front of it after the first layer), o,
+# RMSNorm + gate|up, down; before them the prologue with the first RMSNorm and
+# q|k|v projection
+PHASES = ("attention", "o", "gate_up", "down")
 
 
 class ShardError(RuntimeError):
@@ -95,6 +98,8 @@ def load_library(path: str = LIB_PATH):
         "kv_state_import": ([vp, ip, vp, vp, ip], ip),
         "shard_step": ([vp, vp, vp, vp, i32p, ip, vp, vp, ip, vp, vp, vp], ip),
         "shard_step_host": ([vp, vp, vp, vp, i32p, ip, vp, vp, ip, vp, vp, vp], ip),
+        "shard_step_packed": ([vp, vp, vp, vp, ip, vp, vp, ip, vp, vp], ip),
+        "shard_prefill": ([vp, vp, ip, vp, vp, ip, vp, vp, ip, vp, vp], ip),
         "shard_sync_status": ([vp, vp], ip),
         "shard_last_error": ([], ctypes.c_char_p),
         "shard_debug_op_info": ([vp, ip, ip, ctypes.POINTER(ctypes.c_int), ctypes.POINTER(ctypes.c_int),
@@ -103,6 +108,8 @@ def load_library(path: str = LIB_PATH):
         "shard_debug_gemv": ([vp, ip, ip, vp, ip, vp, ip, vp], ip),
         "shard_gemv_noalloc": ([vp, ip, ip, vp, ip, vp, ip, vp], ip),
         "shard_debug_phase_times": ([vp, ctypes.POINTER(ctypes.c_double), ip], ip),
+        "shard_debug_gemm": ([vp, ip, ip, vp, ip, ip, vp, ip, vp], ip),
+        "shard_debug_set_wait": ([vp, ctypes.c_uint, ip], ip),
         "head_create": ([ctypes.POINTER(head_config), ctypes.POINTER(head_weights_host), ctypes.POINTER(vp)], ip),
         "head_destroy": ([vp], ip),
         "head_top1": ([vp, vp, ip, vp, vp, vp], ip),
@@ -231,6 +238,24 @@ def shard_step(shard: int, state: int, hidden_in: Optional[int], token_ids: Opti
     return _check(rc) if check else rc
 
 
+def shard_step_packed(shard: int, state: int, hidden_in: Optional[int], token_ids: Optional[int], S: int,
+                      position_ids: int, mask2d: int, mask_stride: int, hidden_out: int, stream: int = 0,
+                      check: bool = True) -> int:
+    """Packed step (Section 8.6): device pointers as ints; mask2d [S][mask_stride]."""
+    rc = load_library().shard_step_packed(shard, state, hidden_in or None, token_ids or None, S, position_ids, mask2d,
+                                          mask_stride, hidden_out, stream or None)
+    return _check(rc) if check else rc
+
+
+def shard_prefill(shard: int, state: int, row: int, hidden_in: Optional[int], token_ids: Optional[int], S: int,
+                  position_ids: int, attention_mask: int, mask_len: int, hidden_out: int, stream: int = 0,
+                  check: bool = True) -> int:
+    """Prefill of one row (device pointers as ints)."""
+    rc = load_library().shard_prefill(shard, state, row, hidden_in or None, token_ids or None, S, position_ids,
+                                      attention_mask, mask_len, hidden_out, stream or None)
+    return _check(rc) if check else rc
+
+
 def shard_step_host(shard: int, state: int, hidden_in: Optional[np.ndarray], token_ids: Optional[np.ndarray],
                     n_new: Sequence[int], position_ids: np.ndarray, attention_mask: np.ndarray,
                     beam_idx: Optional[np.ndarray], hidden_out: np.ndarray, stream: int = 0,
@@ -265,16 +290,27 @@ def shard_debug_gemv(shard: int, layer: int, op: int, x: int, M: int, y: int, y_
     _check(load_library().shard_debug_gemv(shard, layer, op, x, M, y, y_ld, stream or None))
 
 
+def shard_debug_gemm(shard: int, layer: int, op: int, x: int, x_ld: int, S: int, y: int, y_ld: int,
+                     stream: int = 0) -> None:
+    """Many-token tensor-core projection (device pointers as ints; x padded to x_ld)."""
+    _check(load_library().shard_debug_gemm(shard, layer, op, x, x_ld, S, y, y_ld, stream or None))
+
+
 def shard_debug_phase_times(shard: int, n_layers: int):
-    """Durations (microseconds) of the last step's phases: the prologue, then
-    per layer the phases named in PHASES (the last layer's last phase ends
-    with the kernel, not at a barrier, and is not included)."""
-    n = len(PHASES) * n_layers
+    """Durations (microseconds) of the last step's phases: the prologue (with
+    the first RMSNorm and q|k|v projection), then per layer the phases named
+    in PHASES."""
+    n = len(PHASES) * n_layers + 1
     buf = (ctypes.c_double * n)()
     k = load_library().shard_debug_phase_times(shard, buf, n)
     if k < 0:
         _check(k)
     return list(buf)[:k]
+
+
+def shard_debug_set_wait(shard: int, limit: int, skip_arrival: int = -1) -> None:
+    """Test knob of the step kernel's bounded waits (include/shard_debug.h)."""
+    _check(load_library().shard_debug_set_wait(shard, int(limit), int(skip_arrival)))
 
 
 def shard_gemv_noalloc(shard: int, layer: int, op: int, x: int, M: int, y: int, y_ld: int, stream: int = 0,

@@ -15,7 +15,7 @@ PKG = os.path.dirname(os.path.abspath(__file__))
 ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 LIB = os.path.join(PKG, "libshard.so")
-SOURCES = ["gemv.cu", "step_kernel.cu", "misc.cu", "shard_api.cu", "noalloc.cu", "head.cu"]
+SOURCES = ["gemv.cu", "step_kernel.cu", "misc.cu", "shard_api.cu", "noalloc.cu", "head.cu", "gemm_tc.cu", "prefill.cu"]
 HEADERS = ["common.cuh", "kernels.h", "gemv_core.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC,-O2", "--expt-relaxed-constexpr"]

@@ -1,70 +1,78 @@
 // Standalone launch of one W4A16 projection (the test export
-// shard_debug_gemv and the allocation-free entry point use it).  The device
-// code is the warp-level projection of gemv_core.cuh, the same code the
-// whole-step kernel runs.
+// shard_debug_gemv, the allocation-free entry point and the LM head use it).
+// The device code is the warp-level projection of gemv_core.cuh, the same
+// code the whole-step kernel runs: kGemvWarps consumer warps and one producer
+// warp per CTA, one CTA per SM.
 #include "gemv_core.cuh"
 
 namespace shard {
 namespace {
 
-constexpr int kW = kGemvWarps;  // warps per CTA
+constexpr int kW = kGemvWarps;  // consumer warps per CTA
 constexpr int kCtasPerSm = 1;
 
-template <int NT, int GPU>
+template <int GPU>
 constexpr size_t smem_bytes() {
   return (size_t)kW * Geom<GPU>::kGemvSlots * Geom<GPU>::kUnitBytes +
-         (size_t)kW * Geom<GPU>::kGemvSlots * sizeof(uint64_t);
+         (size_t)2 * kW * Geom<GPU>::kGemvSlots * sizeof(uint64_t);
 }
 
 // 227 KB per CTA, less a margin for the kernel's static shared memory
-static_assert(smem_bytes<1, 1>() <= 225 * 1024 && smem_bytes<1, 2>() <= 225 * 1024 && smem_bytes<1, 4>() <= 225 * 1024,
+static_assert(smem_bytes<1>() <= 225 * 1024 && smem_bytes<2>() <= 225 * 1024 && smem_bytes<4>() <= 225 * 1024,
               "standalone projection ring too large");
 
 template <int NT, int GPU>
-__global__ void __launch_bounds__(kW * 32) gemv_kernel(const __grid_constant__ GemvArgs a) {
+__global__ void __launch_bounds__((kW + 1) * 32, 1) gemv_kernel(const __grid_constant__ GemvArgs a) {
   extern __shared__ __align__(128) uint8_t smem[];
   __shared__ OpDesc s_op[1];
   __shared__ GemvPhase s_gp;
-  __shared__ WarpStream<GPU> s_ws[kW];
+  __shared__ WarpRing<GPU> s_ring[kW];
+  constexpr int kSlots = Geom<GPU>::kGemvSlots;
+  constexpr int kShift = kSlots == 4 ? 2 : 1;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  uint8_t* rings = smem;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + (size_t)kW * kSlots * Geom<GPU>::kUnitBytes);
+  uint64_t* empty = full + kW * kSlots;
   if (threadIdx.x == 0) {
     s_op[0] = OpDesc{a.units, a.n_rb, a.upr};
     GemvPhase p{};
     p.act = a.act;
     p.act_ld = a.act_ld;
-    p.M = a.sp ? a.sp->M : a.M;
-    p.skip = a.sp ? (a.sp->abort_step != 0) : false;
-    p.partials = a.partials;
-    p.flags = a.flags;
+    p.M = a.M;
     p.status = a.status;
-    p.sp = a.sp;
     p.ep = a.ep;
     s_gp = p;
+    ring_init_barriers(full, empty, kW * kSlots);
+  }
+  if (lane == 0 && warp < kW) {
+    WarpRing<GPU> r;
+    r.ring = rings + (size_t)warp * kSlots * Geom<GPU>::kUnitBytes;
+    r.full = full + warp * kSlots;
+    r.empty = empty + warp * kSlots;
+    r.slot_mask = kSlots - 1;
+    r.slot_shift = kShift;
+    r.n_used = 0;
+    r.timed_out = false;
+    s_ring[warp] = r;
   }
   __syncthreads();
-  constexpr int kSlots = Geom<GPU>::kGemvSlots;
-  const size_t ring_bytes = (size_t)kW * kSlots * Geom<GPU>::kUnitBytes;
-  uint8_t* ring = smem + (size_t)warp * kSlots * Geom<GPU>::kUnitBytes;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + ring_bytes) + warp * kSlots;
-  {
-    WarpStream<GPU> ws;
-    ws.init(s_op, 1, blockIdx.x, gridDim.x, warp, kW, ring, bars, kSlots == 4 ? 2 : 1, lane);
-    ws.fill(lane);
-    if (lane == 0) s_ws[warp] = ws;
-    __syncwarp();
+  if (warp == kW) {
+    // the weights do not depend on the preceding kernel: start streaming them
+    ring_producer<GPU>(s_op, 1, blockIdx.x, gridDim.x, kW, rings, full, empty, kShift, a.status, 1u << 22, lane);
+    return;
   }
   pdl_launch_dependents();
   pdl_wait();
-  gemv_phase<NT, GPU>(&s_ws[warp], 0, &s_gp, 0, a.epoch, lane);
-  if (s_ws[warp].timed_out && lane == 0) atomicOr(a.status, ST_WAIT_TIMEOUT);
+  gemv_phase<NT, GPU>(&s_ring[warp], &s_op[0], &s_gp, blockIdx.x * kW + warp, gridDim.x * kW, lane);
+  if (s_ring[warp].timed_out && lane == 0) atomicOr(a.status, ST_WAIT_TIMEOUT);
 }
 
 template <int NT, int GPU>
 cudaError_t launch_t(const GemvArgs& a, int grid, cudaStream_t s, bool pdl) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
-  cfg.blockDim = dim3(kW * 32);
-  cfg.dynamicSmemBytes = smem_bytes<NT, GPU>();
+  cfg.blockDim = dim3((kW + 1) * 32);
+  cfg.dynamicSmemBytes = smem_bytes<GPU>();
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -77,7 +85,7 @@ cudaError_t launch_t(const GemvArgs& a, int grid, cudaStream_t s, bool pdl) {
 template <int NT, int GPU>
 cudaError_t setup_t() {
   return cudaFuncSetAttribute(gemv_kernel<NT, GPU>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              (int)smem_bytes<NT, GPU>());
+                              (int)smem_bytes<GPU>());
 }
 
 }  // namespace
@@ -97,12 +105,8 @@ int gemv_grid(int nt, int num_sms) {
   return kCtasPerSm * num_sms;
 }
 
-// the larger of the two kernels' warp counts: buffers and index checks cover both
+// the larger of the two kernels' consumer warp counts: index checks cover both
 int gemv_warps_per_cta() { return kW > kCtaWarps ? kW : kCtaWarps; }
-
-size_t gemv_partials_floats(int grid) { return (size_t)grid * gemv_warps_per_cta() * 2 * kPieceFloats; }
-
-size_t gemv_flags_count(int grid) { return (size_t)grid * gemv_warps_per_cta() * 2; }
 
 cudaError_t launch_gemv(const GemvArgs& a, int nt, int group, int grid, cudaStream_t s, bool pdl) {
   if (nt == 1) {

@@ -2,41 +2,45 @@
 // kernel and the standalone projection kernel.
 //
 // Work split.  The unit stream of a projection (n_rb row-blocks x upr units,
-// see kernels.h) is cut into contiguous runs, one per warp of the grid
-// (warp g = cta * warps per CTA + warp), so every warp streams the same number of
-// bytes and keeps its sums in registers for as long as its run stays inside
-// one row-block.  Each warp owns a ring of shared-memory slots (a power of two:
-// kRingSlots in the step kernel, Geom::kGemvSlots in the standalone projection) that
-// its lane 0 fills with bulk copies (TMA, non-tensor), one unit per slot,
-// completion tracked by one mbarrier per slot.  Because the weights never
-// depend on earlier work, a warp's ring runs ahead through the *sequence* of
-// projections it will process (the step's q|k|v, o, gate|up, down of every
-// layer): while the warp waits for other work, its next projection's weights
-// are already in flight.
+// see kernels.h) is cut into contiguous runs, one per consumer warp of the
+// grid (warp g = cta * warps per CTA + warp), so every warp streams the same
+// number of bytes and keeps its sums in registers for as long as its run
+// stays inside one row-block.
+//
+// Weight streaming.  Every consumer warp owns a ring of shared-memory slots
+// (a power of two).  One producer warp per CTA fills them: its lane w walks
+// consumer warp w's runs of every projection of the launch in order and
+// issues one bulk copy (TMA, non-tensor) per unit into the next free slot,
+// completion signalled on the slot's "full" mbarrier; the consumer releases
+// the slot on its "empty" mbarrier after the unit's fragments are in
+// registers.  Because the weights never depend on earlier work, the rings run
+// ahead across projections: while consumers wait at a barrier or work on
+// norms and attention, their next projection's first units are already
+// arriving, and consumers execute no stream bookkeeping at all.
 //
 // Per unit, a lane turns each 32-bit code word into the four registers of its
-// m16n8k16 A fragment -- (q - z) exactly, in fp16 -- and multiplies them with
-// the activations (the B fragment) on the tensor cores, accumulating in fp32;
-// the fp16 group scale multiplies the fp32 group sum.
+// m16n8k16 A fragment with one AND per register (the codes as fp16
+// subnormals) and multiplies them with the activations (the B fragment) on
+// the tensor cores, accumulating in fp32; per group, the zero point is
+// applied through the activations' group sum and the fp16 scale multiplies
+// the result (mma_unit).
 //
-// Reduction.  A row-block lying wholly inside one warp's run is finished by
-// that warp.  A row-block split between warps gets one piece per warp; each
-// contributor stores its piece and publishes it with a release-store of the
-// launch's epoch into its flag, never waiting.  The warp that owns the
-// row-block's last unit, after its own run, waits (acquire loads, all
-// contributors polled at once, bounded) for the other flags, adds the pieces
-// in warp order and runs the epilogue.  Waits only ever point to lower warp
-// indices, so they cannot form a cycle; the fixed order makes results
-// deterministic and independent of the token count M.
+// Reduction.  At the end of each row-block segment of its run, a warp adds
+// its fp32 sums, converted to 64-bit fixed point, to the projection's
+// accumulator with integer atomics (kernels.h: EpiArgs).  Nothing waits:
+// the residual projections add straight into the residual stream; q|k|v
+// contributors count finished units per kv head for the attention items; for
+// gate|up (and the standalone store) the contributor whose unit count
+// completes a row-block finishes it.  Integer sums make every result
+// independent of arrival order.
 #pragma once
 #include "common.cuh"
 
 namespace shard {
 
-constexpr int kRingSlots = 2;  // step kernel: units in flight per warp (measured: a third adds nothing)
-static_assert(kRingSlots == 2 || kRingSlots == 4, "ring slots: a power of two the init call passes as a shift");
-constexpr int kCtaWarps = 12;   // warps per CTA of the step kernel (all run projections)
-constexpr int kGemvWarps = 12;  // warps per CTA of the standalone projection kernel
+constexpr int kRingSlots = 2;  // step kernel: units in flight per consumer warp (measured: a third adds nothing)
+constexpr int kCtaWarps = 11;   // consumer warps per CTA of the step kernel (+ 1 producer: 3 warps per SM sub-partition)
+constexpr int kGemvWarps = 11;  // consumer warps per CTA of the standalone projection kernel (+ 1 producer)
 
 template <int GPU>
 struct Geom {
@@ -63,19 +67,11 @@ __device__ __forceinline__ uint32_t prmt_u32(uint32_t a, uint32_t b, uint32_t c)
   asm("prmt.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(c));
   return d;
 }
-__device__ __forceinline__ void fence_proxy_async_smem() {
-  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-}
 
 // Start of part i of n of a stream of T units.  32-bit arithmetic: the host
 // checks (T + 1) * n < 2^32 for every projection when a shard is created.
 __device__ __forceinline__ int part_start(int T, int i, int n) {
   return static_cast<int>(static_cast<uint32_t>(T) * static_cast<uint32_t>(i) / static_cast<uint32_t>(n));
-}
-// The part owning unit x: the largest i with part_start(T, i, n) <= x.
-__device__ __forceinline__ int part_of(int T, int x, int n) {
-  return static_cast<int>((static_cast<uint32_t>(x + 1) * static_cast<uint32_t>(n) + static_cast<uint32_t>(T) - 1u) /
-                          static_cast<uint32_t>(T)) - 1;
 }
 
 __device__ __forceinline__ int atom_add_acq_rel(int* p, int v) {
@@ -83,118 +79,139 @@ __device__ __forceinline__ int atom_add_acq_rel(int* p, int v) {
   asm volatile("atom.add.acq_rel.gpu.global.s32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
   return old;
 }
-__device__ __forceinline__ void st_release_u32(unsigned* p, unsigned v) {
-  asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+__device__ __forceinline__ void red_release_add_s32(int* p, int v) {
+  asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
 }
-__device__ __forceinline__ unsigned ld_acquire_u32(const unsigned* p) {
-  unsigned v;
-  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+__device__ __forceinline__ int ld_acquire_s32(const int* p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
   return v;
 }
+__device__ __forceinline__ void red_add_s64(long long* p, long long v) {
+  asm volatile("red.relaxed.gpu.global.add.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
+}
+__device__ __forceinline__ long long to_fixed(float v) { return __float2ll_rn(v * kFixOne); }
+// int64 -> fp32 rounds once; the power-of-two scale is exact
+__device__ __forceinline__ float fixed_to_f32(long long v) { return __ll2float_rn(v) * 2.3283064365386963e-10f; }
 
 // ---------------------------------------------------------------------------
-// Per-warp weight stream over a table of ops (in shared memory).
+// Weight rings.
 // ---------------------------------------------------------------------------
+__device__ __forceinline__ bool mbar_test_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(smem_addr(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Consumer side of one warp's ring.
 template <int GPU>
-struct WarpStream {
+struct WarpRing {
   static constexpr int UB = Geom<GPU>::kUnitBytes;
-  const OpDesc* ops;  // shared memory
-  int n_ops, cta, n_cta, warp;
-  int cta_warps;       // projection warps per CTA (the warp index space is cta * cta_warps + warp)
-  uint8_t* ring;      // [slots][UB]
-  uint64_t* bars;     // [slots]
-  uint32_t slot_mask;  // slots - 1 (slots a power of two)
+  uint8_t* ring;       // [slots][UB]
+  uint64_t* full;      // [slots]
+  uint64_t* empty;     // [slots]
+  uint32_t slot_mask;  // slots - 1
   int slot_shift;      // log2(slots)
-  // fill cursor: op index, next unit, end of the CTA's range, op's units
-  int f_op, f_u, f_end;
-  const uint8_t* f_units;
-  uint32_t n_filled, n_used;
+  uint32_t n_used;
   bool timed_out;
 
-  // Run [wb, we) of this warp in op's unit stream.
-  __device__ __forceinline__ void warp_range(int op, int& wb, int& we) const {
-    const int T = ops[op].n_rb * ops[op].upr;
-    const int g = cta * cta_warps + warp, nw = n_cta * cta_warps;
-    wb = part_start(T, g, nw);
-    we = part_start(T, g + 1, nw);
-  }
-  __device__ __forceinline__ void open_op(int op) {
-    warp_range(op, f_u, f_end);
-    f_units = ops[op].units;
-  }
-  // lane 0 initialises the slot barriers; the warp is synced after.
-  __device__ void init(const OpDesc* ops_, int n_ops_, int cta_, int n_cta_, int warp_, int cta_warps_, uint8_t* ring_,
-                       uint64_t* bars_, int slot_shift_, int lane) {
-    ops = ops_;
-    cta_warps = cta_warps_;
-    slot_shift = slot_shift_;
-    slot_mask = (1u << slot_shift_) - 1u;
-    n_ops = n_ops_;
-    cta = cta_;
-    n_cta = n_cta_;
-    warp = warp_;
-    ring = ring_;
-    bars = bars_;
-    n_filled = n_used = 0;
-    timed_out = false;
-    f_op = 0;
-    f_u = f_end = 0;
-    f_units = nullptr;
-    if (n_ops > 0) open_op(0);
-    if (lane == 0) {
-      for (uint32_t s = 0; s <= slot_mask; ++s) mbar_init(&bars[s], 1);
-      mbar_fence_init();
-    }
-    __syncwarp();
-  }
-  // Issues bulk copies until the ring is full or the stream ends.
-  __device__ __forceinline__ void fill(int lane) {
-    while (n_filled - n_used <= slot_mask) {
-      while (f_u >= f_end) {
-        if (++f_op >= n_ops) return;
-        open_op(f_op);
-      }
-      const uint8_t* src = f_units + (size_t)f_u * UB;
-      ++f_u;
-      if (lane == 0) {
-        const int slot = n_filled & slot_mask;
-        fence_proxy_async_smem();
-        mbar_arrive_expect_tx(&bars[slot], UB);
-        // L2 evict-first: each weight byte is read once per step
-        bulk_g2s_hint(ring + (size_t)slot * UB, src, UB, &bars[slot], l2_policy_evict_first());
-      }
-      ++n_filled;
-    }
-  }
+  // Waits (bounded) for the next unit; returns its slot.
   __device__ __forceinline__ const uint8_t* acquire() {
-    const int slot = n_used & slot_mask;
-    if (!timed_out && !mbar_wait(&bars[slot], (n_used >> slot_shift) & 1)) timed_out = true;
+    const uint32_t slot = n_used & slot_mask;
+    if (!timed_out && !mbar_wait(&full[slot], (n_used >> slot_shift) & 1)) timed_out = true;
     return ring + (size_t)slot * UB;
   }
+  // The unit's fragments are in registers: hand the slot back.
   __device__ __forceinline__ void release(int lane) {
     __syncwarp();
+    if (lane == 0) mbar_arrive(&empty[n_used & slot_mask]);
     ++n_used;
-    fill(lane);
   }
 };
+
+// Initialises the full/empty barriers of all rings of the CTA (one thread).
+__device__ __forceinline__ void ring_init_barriers(uint64_t* full, uint64_t* empty, int n) {
+  for (int i = 0; i < n; ++i) {
+    mbar_init(&full[i], 1);
+    mbar_init(&empty[i], 1);
+  }
+  mbar_fence_init();
+}
+
+// Producer: lane w < n_warps fills consumer warp w's ring with the warp's
+// runs of ops[0 .. n_ops), in order.  A slot is refilled once its previous
+// unit was released.  Bounded: a slot that stays busy for `limit` polls sets
+// ST_WAIT_TIMEOUT and ends the producer (the consumers' own bounded waits
+// then give up too).
+template <int GPU>
+__device__ __noinline__ void ring_producer(const OpDesc* ops, int n_ops, int cta, int n_cta, int n_warps, uint8_t* rings,
+                                           uint64_t* full, uint64_t* empty, int slot_shift, int* status,
+                                           uint32_t limit, int lane) {
+  constexpr int UB = Geom<GPU>::kUnitBytes;
+  if (lane >= n_warps) return;
+  const uint32_t S = 1u << slot_shift, mask = S - 1;
+  uint8_t* ring = rings + (size_t)lane * S * UB;
+  uint64_t* f = full + lane * S;
+  uint64_t* e = empty + lane * S;
+  const int g = cta * n_warps + lane, nw = n_cta * n_warps;
+  const uint64_t policy = l2_policy_evict_first();  // each weight byte is read once per launch
+  uint32_t n = 0, spins = 0;
+  for (int op = 0; op < n_ops; ++op) {
+    const int T = ops[op].n_rb * ops[op].upr;
+    const int ub = part_start(T, g, nw), ue = part_start(T, g + 1, nw);
+    const uint8_t* src = ops[op].units + (size_t)ub * UB;
+    for (int u = ub; u < ue; ++u, ++n, src += UB) {
+      const uint32_t slot = n & mask;
+      if (n >= S) {
+        while (!mbar_test_wait(&e[slot], ((n >> slot_shift) - 1) & 1)) {
+          if (++spins > limit) {
+            atomicOr(status, ST_WAIT_TIMEOUT);
+            return;
+          }
+          __nanosleep(32);
+        }
+        spins = 0;
+      }
+      mbar_arrive_expect_tx(&f[slot], UB);
+      bulk_g2s_hint(ring + (size_t)slot * UB, src, UB, &f[slot], policy);
+    }
+  }
+}
 
 // ---------------------------------------------------------------------------
 // One unit (64 rows x 128 inputs) of one warp.
 //
-// Dequantisation of a code word w: (w & 0x000F000F) | 0x64006400 is the fp16
-// pair (1024 + q_lo, 1024 + q_hi) of the nibbles at bits 0 and 16; subtracting
-// (1024 + z) leaves q - z exactly.  The nibbles at bits 4 and 20 give
-// 1024 + 16 q; one fma with 1/16 and -(64 + z) leaves q - z exactly.  Bits
-// 8..15 / 24..31 are handled the same way after a shift by 8.
+// Codes enter the tensor cores as fp16 subnormals: the nibbles at bits 0..3
+// (and 16..19) of a code word w are, read as fp16 bit patterns, exactly
+// q * 2^-24, and the nibbles at bits 4..7 are 16 q * 2^-24, so each A
+// register is one AND of w (or of w >> 8): a0 = w & 0x000F000F, a1 = w &
+// 0x00F000F0 (rows gid + 8 of the tile, scaled by 16), a2 and a3 likewise
+// from w >> 8.  The zero point is applied once per group instead of once per
+// weight: sum_k (q - z) a = sum_k q a - z sum_k a, where sum_k a, the group
+// sum of each token's activations, comes from one more MMA per k-block with
+// an all-ones A.  The unit stores z (rows gid) and 16 z (rows gid + 8) as
+// bytes, so one byte permute gives (-z * 2^-24, -16 z * 2^-24) as fp16
+// subnormals in the same scale as the sums.  Per group and row:
+//   tot += s * (acc + zs * sum_a)
+// in units of 2^-24 (rows gid) and 2^-20 (rows gid + 8); segment_end applies
+// the powers of two when it converts to fixed point.  Products are exact and
+// accumulate in fp32.
 // ---------------------------------------------------------------------------
+constexpr float kTotScaleLo = 72057594037927936.0f;  // 2^56 = 2^32 (fixed point) * 2^24
+constexpr float kTotScaleHi = 4503599627370496.0f;   // 2^52 = 2^32 * 2^20
+
 template <int NT, int GPU>
 __device__ __forceinline__ void mma_unit(const uint8_t* __restrict__ U, const uint4 (&act)[NT][2][2],
                                          float (&tot)[4][NT][4], int lane) {
   constexpr int BPG = Geom<GPU>::kBlocksPerGroup;
-  constexpr uint32_t kSixteenth = 0x2C002C00u;  // fp16x2 1/16
+  constexpr uint32_t kOnes = 0x3C003C00u;  // fp16x2 (1, 1)
   const int gid = lane >> 2;
   float accg[4][NT][4];
-  uint32_t zsub[4], zfma[4];
+  float sa[NT][4];  // group sums of the activations: tokens 2 tig, 2 tig + 1 (twice)
 #pragma unroll
   for (int kc = 0; kc < 2; ++kc) {
     uint4 A[4];
@@ -206,23 +223,14 @@ __device__ __forceinline__ void mma_unit(const uint8_t* __restrict__ U, const ui
       const int gi = blk / BPG;
       const uint8_t* meta = U + kCodeBytes + gi * kMetaBytesPerGroup;
       if (blk % BPG == 0) {
-        // group start: clear the group sums; zero points as fp16x2
-        // (1024 + z_lo) = bits 0x6400 | z and -(64 + z_hi) = bits 0xD400 | 16 z,
-        // each one byte permute: the unit stores the upper rows' zero
-        // points as 16 z
 #pragma unroll
-        for (int rt = 0; rt < 4; ++rt)
+        for (int nt = 0; nt < NT; ++nt) {
 #pragma unroll
-          for (int nt = 0; nt < NT; ++nt)
+          for (int e = 0; e < 4; ++e) sa[nt][e] = 0.f;
+#pragma unroll
+          for (int rt = 0; rt < 4; ++rt)
 #pragma unroll
             for (int e = 0; e < 4; ++e) accg[rt][nt][e] = 0.f;
-        const uint2 zz = *reinterpret_cast<const uint2*>(meta + 128 + gid * 8);
-#pragma unroll
-        for (int rt = 0; rt < 4; ++rt) {
-          const uint32_t zw = rt < 2 ? zz.x : zz.y;  // bytes: z_lo, 16 z_hi of tiles 2i, then 2i + 1
-          const uint32_t p = 2u * (rt & 1);
-          zsub[rt] = prmt_u32(zw, 0x64646464u, 0x4040u + p * 0x0101u);
-          zfma[rt] = prmt_u32(zw, 0xD4D4D4D4u, 0x4040u + (p + 1u) * 0x0101u);
         }
       }
       uint32_t b0[NT], b1[NT];
@@ -231,31 +239,38 @@ __device__ __forceinline__ void mma_unit(const uint8_t* __restrict__ U, const ui
         const uint4 v = act[nt][kc][j >> 1];
         b0[nt] = (j & 1) ? v.z : v.x;
         b1[nt] = (j & 1) ? v.w : v.y;
+        mma_16816(sa[nt], kOnes, kOnes, kOnes, kOnes, b0[nt], b1[nt]);
       }
 #pragma unroll
       for (int rt = 0; rt < 4; ++rt) {
         const uint32_t w = (j == 0) ? A[rt].x : (j == 1) ? A[rt].y : (j == 2) ? A[rt].z : A[rt].w;
         const uint32_t w2 = w >> 8;
-        const uint32_t a0 = hsub2_u32(lop3_and_or(w, 0x000F000Fu, 0x64006400u), zsub[rt]);
-        const uint32_t a1 = hfma2_u32(lop3_and_or(w, 0x00F000F0u, 0x64006400u), kSixteenth, zfma[rt]);
-        const uint32_t a2 = hsub2_u32(lop3_and_or(w2, 0x000F000Fu, 0x64006400u), zsub[rt]);
-        const uint32_t a3 = hfma2_u32(lop3_and_or(w2, 0x00F000F0u, 0x64006400u), kSixteenth, zfma[rt]);
+        const uint32_t a0 = w & 0x000F000Fu, a1 = w & 0x00F000F0u;
+        const uint32_t a2 = w2 & 0x000F000Fu, a3 = w2 & 0x00F000F0u;
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt) mma_16816(accg[rt][nt], a0, a1, a2, a3, b0[nt], b1[nt]);
       }
       if (blk % BPG == BPG - 1) {
+        // group end: zero-point correction and scale
+        const uint2 zz = *reinterpret_cast<const uint2*>(meta + 128 + gid * 8);
         const uint4 sc = *reinterpret_cast<const uint4*>(meta + gid * 16);
         const uint32_t scw[4] = {sc.x, sc.y, sc.z, sc.w};
 #pragma unroll
         for (int rt = 0; rt < 4; ++rt) {
+          const uint32_t zw = rt < 2 ? zz.x : zz.y;  // bytes: z_lo, 16 z_hi of tiles 2i, then 2i + 1
+          const uint32_t p = 2u * (rt & 1);
+          // fp16 bits 0x8000 | z and 0x8000 | 16 z: -z * 2^-24 and -16 z * 2^-24
+          const uint32_t zp = prmt_u32(zw, 0x80u, p | (4u << 4) | ((p + 1u) << 8) | (4u << 12));
+          const float zlo = h2f(static_cast<uint16_t>(zp & 0xFFFFu));
+          const float zhi = h2f(static_cast<uint16_t>(zp >> 16));
           const float slo = h2f(static_cast<uint16_t>(scw[rt] & 0xFFFFu));
           const float shi = h2f(static_cast<uint16_t>(scw[rt] >> 16));
 #pragma unroll
           for (int nt = 0; nt < NT; ++nt) {
-            tot[rt][nt][0] = fmaf(slo, accg[rt][nt][0], tot[rt][nt][0]);
-            tot[rt][nt][1] = fmaf(slo, accg[rt][nt][1], tot[rt][nt][1]);
-            tot[rt][nt][2] = fmaf(shi, accg[rt][nt][2], tot[rt][nt][2]);
-            tot[rt][nt][3] = fmaf(shi, accg[rt][nt][3], tot[rt][nt][3]);
+            tot[rt][nt][0] = fmaf(slo, fmaf(zlo, sa[nt][0], accg[rt][nt][0]), tot[rt][nt][0]);
+            tot[rt][nt][1] = fmaf(slo, fmaf(zlo, sa[nt][1], accg[rt][nt][1]), tot[rt][nt][1]);
+            tot[rt][nt][2] = fmaf(shi, fmaf(zhi, sa[nt][0], accg[rt][nt][2]), tot[rt][nt][2]);
+            tot[rt][nt][3] = fmaf(shi, fmaf(zhi, sa[nt][1], accg[rt][nt][3]), tot[rt][nt][3]);
           }
         }
       }
@@ -265,105 +280,21 @@ __device__ __forceinline__ void mma_unit(const uint8_t* __restrict__ U, const ui
 
 __device__ __forceinline__ float silu(float v) { return v / (1.f + expf(-v)); }
 
-// Epilogue of one (row R_lo, row R_lo + 8, token m) pair of a finished
-// row-block: rotary pairs and gate/up pairs sit on these two rows.  Returns
-// the sum of squares of the residual values written (EPI_RESID), else 0.
-// xlo, xhi: the residual's current values at the two rows (EPI_RESID).
-__device__ __forceinline__ float epilogue_pair(const EpiArgs& e, const StepParams* sp, int layer, int Rlo, int m,
-                                               float vlo, float vhi, float xlo, float xhi) {
-  float ss = 0.f;
-  const OpDims& o = e.dims;
-  const int Rhi = Rlo + 8;
-  switch (e.kind) {
-    case EPI_STORE: {
-      const int n1 = natural_row(o, Rlo), n2 = natural_row(o, Rhi);
-      if (n1 >= 0) e.y[(size_t)m * e.y_ld + n1] = vlo;
-      if (n2 >= 0) e.y[(size_t)m * e.y_ld + n2] = vhi;
-      break;
-    }
-    case EPI_QKV: {
-      const int tph = o.d >> 4, nq = o.Hq * tph, nk = o.Hkv * tph, half = o.d >> 1;
-      const int T = Rlo >> 4;
-      const int slot = sp->tok_slot[m];
-      const int prow = slot / e.cap, ppos = slot % e.cap;
-      if (T < nq + nk) {
-        const int t = T < nq ? T : T - nq;
-        const int head = t / tph, i = 8 * (t % tph) + (Rlo & 7);
-        const float2 cs = e.rope[(size_t)sp->tok_pos[m] * half + i];
-        const float olo = vlo * cs.x - vhi * cs.y;
-        const float ohi = vhi * cs.x + vlo * cs.y;
-        if (T < nq) {
-          float* q = e.q + (size_t)m * o.Hq * o.d + head * o.d;
-          q[i] = olo;
-          q[half + i] = ohi;
-        } else {
-          uint16_t* k = e.kpool + (size_t)layer * e.layer_stride + (((size_t)prow * o.Hkv + head) * e.cap + ppos) * o.d;
-          k[i] = f2h(olo);
-          k[half + i] = f2h(ohi);
-        }
-      } else {
-        const int base = (o.Hq + o.Hkv) * o.d;
-        const int rv[2] = {Rlo - base, Rhi - base};
-        const float vv[2] = {vlo, vhi};
-#pragma unroll
-        for (int u = 0; u < 2; ++u) {
-          if (rv[u] < o.Hkv * o.d) {
-            const int head = rv[u] / o.d, dim = rv[u] % o.d;
-            e.vpool[(size_t)layer * e.layer_stride + (((size_t)prow * o.Hkv + head) * e.cap + ppos) * o.d + dim] =
-                f2h(vv[u]);
-          }
-        }
-      }
-      break;
-    }
-    case EPI_RESID: {
-      const int rr[2] = {Rlo, Rhi};
-      const float vv[2] = {vlo, vhi}, xv[2] = {xlo, xhi};
-#pragma unroll
-      for (int u = 0; u < 2; ++u) {
-        if (rr[u] < o.H) {
-          float* xp = e.x + (size_t)m * o.H + rr[u];
-          const float nx = xv[u] + vv[u];
-          *xp = nx;
-          ss = fmaf(nx, nx, ss);
-          if (e.out_layer == layer) sp->hidden_out[(size_t)m * o.H + rr[u]] = f2h(nx);
-        }
-      }
-      break;
-    }
-    case EPI_SWIGLU: {
-      const int j = 8 * (Rlo >> 4) + (Rlo & 7);
-      if (j < o.F) e.h[(size_t)m * e.h_ld + j] = f2h(silu(vlo) * vhi);
-      break;
-    }
-    default:
-      break;
-  }
-  return ss;
-}
-
 struct GemvPhase {
   const uint16_t* act;  // fp16 [M][act_ld]
   int act_ld, M;
   uint32_t act_s;       // 0, or the shared-memory address of this CTA's own copy of the activations,
   int act_s_ld;         // fp16 [M][act_s_ld], read instead of act
-  bool skip;            // consume the weights but compute nothing (aborted step)
-  float* partials;      // [n_cta * warps per CTA][2][kPieceFloats] pieces of split row-blocks
-  unsigned* flags;      // [n_cta * warps per CTA][2] epoch of the piece last published in each slot
   int* status;
-  const StepParams* sp;
   EpiArgs ep;
-  unsigned* done_flags;  // nullptr, or row-block flags this projection publishes (release of the epoch
-                         // after the row-block's epilogue)
+  int kv_rb_q, kv_rb_k;  // EPI_QKV: row-blocks per q head group, first k and v row-block (see kv_head_of)
+  int kv_rb_v, kv_rb_per_head;
 };
-
-// Floats of one stored piece: [token][64 rows] for up to kMaxTokens tokens.
-constexpr int kPieceFloats = kMaxTokens * kRowsPerBlock;
 
 // Loads the B fragments of input unit ku for tokens gid (and gid + 8).
 template <int NT>
 __device__ __forceinline__ void load_act(uint4 (&act)[NT][2][2], const uint16_t* actp, uint32_t acts, int act_ld,
-                                         int M, bool skip, int ku, int lane) {
+                                         int M, int ku, int lane) {
   const int gid = lane >> 2, tig = lane & 3;
 #pragma unroll
   for (int nt = 0; nt < NT; ++nt) {
@@ -374,7 +305,7 @@ __device__ __forceinline__ void load_act(uint4 (&act)[NT][2][2], const uint16_t*
       for (int h = 0; h < 2; ++h) {
         const int off = n * act_ld + ku * kUnitK + kc * 64 + h * 32 + tig * 8;
         uint4 v = make_uint4(0, 0, 0, 0);
-        if (n < M && !skip) {
+        if (n < M) {
           if (acts)
             asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
                          : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
@@ -387,122 +318,58 @@ __device__ __forceinline__ void load_act(uint4 (&act)[NT][2][2], const uint16_t*
   }
 }
 
-// Finishes row-block rb from the stored pieces of warps g_first..g_last (the
-// cold path), then runs the epilogue.  Lane L = rg + 8 * pg loads, as
-// float4s, the four row pairs (R0 + i, R0 + 8 + i), R0 = 16 * (rg / 2) +
-// 4 * (rg % 2), of the pieces g_first + pg, + pg + 4, ... and adds them in
-// that order; two butterfly levels over pg then give every lane of the row
-// group the same totals, and lane L finishes the pair R0 + pg (a rotary or
-// gate/up pair).  The order is fixed, so the result is deterministic.
-//
-// Which slot holds a warp's piece: every contributor after the first started
-// its run inside the row-block (slot 0); the first contributor used slot 1
-// if its run started before the row-block.  When T < nw some runs are empty
-// and each non-empty run is a single unit.
-static __device__ __noinline__ void finish_rowblock(const GemvPhase* pp, int layer, int rb, int g_first, int g_last,
-                                                    int T, int nw, int upr, int lane, unsigned epoch) {
+// kv head of q|k|v row-block rb (each row-block lies inside one head: d is a
+// multiple of 64).
+__device__ __forceinline__ int kv_head_of(const GemvPhase& p, int rb) {
+  if (rb < p.kv_rb_k) return rb / p.kv_rb_q;
+  if (rb < p.kv_rb_v) return (rb - p.kv_rb_k) / p.kv_rb_per_head;
+  return (rb - p.kv_rb_v) / p.kv_rb_per_head;
+}
+
+// The contributor that completed row-block rb of a gate|up projection: lane
+// = (tile t, row r) pair; gate is row 16 t + r, up row 16 t + r + 8, and h
+// index j = 32 rb + 8 t + r.  Clears the sums and the count for the next use.
+static __device__ __noinline__ void finish_swiglu(const GemvPhase* pp, int rb, int lane) {
   const GemvPhase& p = *pp;
-  constexpr int kPerLane = 8;  // pieces per lane and batch (32 per batch over the 4 piece groups)
-  const int rb_begin = rb * upr;
-  const int rg = lane & 7, pg = lane >> 3;
-  const int R0 = 16 * (rg >> 1) + 4 * (rg & 1);
-  const int R = rb * kRowsPerBlock + R0 + pg;
-  const bool dense = T >= nw;
-  const size_t first_off = ((size_t)g_first * 2 + (part_start(T, g_first, nw) < rb_begin ? 1 : 0)) * kPieceFloats;
+  const int t = lane >> 3, r = lane & 7;
+  const int Rg = rb * kRowsPerBlock + 16 * t + r, Ru = Rg + 8;
+  const int j = 32 * rb + 8 * t + r;
   for (int m = 0; m < p.M; ++m) {
-    // the residual's current values, loaded with the pieces
-    float xlo = 0.f, xhi = 0.f;
-    if (p.ep.kind == EPI_RESID) {
-      if (R < p.ep.dims.H) xlo = __ldcg(p.ep.x + (size_t)m * p.ep.dims.H + R);
-      if (R + 8 < p.ep.dims.H) xhi = __ldcg(p.ep.x + (size_t)m * p.ep.dims.H + R + 8);
-    }
-    float4 slo = make_float4(0.f, 0.f, 0.f, 0.f), shi = slo;
-    for (int g0 = g_first + pg; g0 <= g_last; g0 += 4 * kPerLane) {
-      float4 a[kPerLane], b[kPerLane];
-#pragma unroll
-      for (int i = 0; i < kPerLane; ++i) {
-        const int gg = g0 + 4 * i;
-        a[i] = b[i] = make_float4(0.f, 0.f, 0.f, 0.f);
-        bool live = gg <= g_last;
-        if (live && !dense) live = part_start(T, gg + 1, nw) > part_start(T, gg, nw);
-        if (live) {
-          const float* pc = p.partials + (gg == g_first ? first_off : (size_t)gg * 2 * kPieceFloats) + m * kRowsPerBlock;
-          a[i] = __ldcg(reinterpret_cast<const float4*>(pc + R0));
-          b[i] = __ldcg(reinterpret_cast<const float4*>(pc + R0 + 8));
-        }
-      }
-#pragma unroll
-      for (int i = 0; i < kPerLane; ++i) {
-        slo.x += a[i].x; slo.y += a[i].y; slo.z += a[i].z; slo.w += a[i].w;
-        shi.x += b[i].x; shi.y += b[i].y; shi.z += b[i].z; shi.w += b[i].w;
-      }
-    }
-#pragma unroll
-    for (int o = 8; o <= 16; o <<= 1) {
-      slo.x += __shfl_xor_sync(0xffffffffu, slo.x, o);
-      slo.y += __shfl_xor_sync(0xffffffffu, slo.y, o);
-      slo.z += __shfl_xor_sync(0xffffffffu, slo.z, o);
-      slo.w += __shfl_xor_sync(0xffffffffu, slo.w, o);
-      shi.x += __shfl_xor_sync(0xffffffffu, shi.x, o);
-      shi.y += __shfl_xor_sync(0xffffffffu, shi.y, o);
-      shi.z += __shfl_xor_sync(0xffffffffu, shi.z, o);
-      shi.w += __shfl_xor_sync(0xffffffffu, shi.w, o);
-    }
-    const float vlo = pg == 0 ? slo.x : pg == 1 ? slo.y : pg == 2 ? slo.z : slo.w;
-    const float vhi = pg == 0 ? shi.x : pg == 1 ? shi.y : pg == 2 ? shi.z : shi.w;
-    float ss = epilogue_pair(p.ep, p.sp, layer, R, m, vlo, vhi, xlo, xhi);
-    if (p.ep.ss) {  // the row-block's sum of squares of the new residual, for the next RMSNorm
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
-      if (lane == 0) p.ep.ss[rb * kMaxTokens + m] = ss;
-    }
+    long long* a = p.ep.acc + (size_t)m * p.ep.acc_ld;
+    const float g = fixed_to_f32(__ldcg(a + Rg)), u = fixed_to_f32(__ldcg(a + Ru));
+    if (j < p.ep.dims.F) p.ep.h[(size_t)m * p.ep.h_ld + j] = f2h(silu(g) * u);
+    __stcg(a + Rg, 0LL);
+    __stcg(a + Ru, 0LL);
   }
-  if (p.done_flags) {
-    __syncwarp();
-    if (lane == 0) st_release_u32(p.done_flags + rb, epoch);
-  }
+  if (lane == 0) __stcg(p.ep.cnt + rb, 0);
 }
 
-// Merge of split row-block rb by the warp owning its last unit: wait until
-// every other contributor (g_first .. g_last - 1, non-empty runs) has
-// published its piece for this epoch, then finish the row-block.
-static __device__ __noinline__ void merge_rowblock(const GemvPhase* pp, int layer, int rb, int g_first, int g_last,
-                                                   int T, int nw, int upr, unsigned epoch, int lane) {
+// The contributor that completed row-block rb of a stored projection: lane
+// takes rows lane and lane + 32 of the row-block.
+static __device__ __noinline__ void finish_store(const GemvPhase* pp, int rb, int lane) {
   const GemvPhase& p = *pp;
-  const int rb_begin = rb * upr;
-  for (int g0 = g_first; g0 < g_last; g0 += 32) {
-    const int gg = g0 + lane;
-    if (gg < g_last) {
-      const int s0 = part_start(T, gg, nw);
-      if (part_start(T, gg + 1, nw) > s0) {  // non-empty run
-        const unsigned* f = p.flags + (size_t)gg * 2 + (gg == g_first && s0 < rb_begin ? 1 : 0);
-        uint32_t it = 0;
-        while (ld_acquire_u32(f) != epoch) {
-          if (++it > (1u << 22)) {
-            atomicOr(p.status, ST_WAIT_TIMEOUT);
-            break;
-          }
-          __nanosleep(32);
-        }
-      }
+  for (int m = 0; m < p.M; ++m) {
+    long long* a = p.ep.acc + (size_t)m * p.ep.acc_ld;
+#pragma unroll
+    for (int hh = 0; hh < 2; ++hh) {
+      const int R = rb * kRowsPerBlock + lane + 32 * hh;
+      const int nat = natural_row(p.ep.dims, R);
+      if (nat >= 0) p.ep.y[(size_t)m * p.ep.y_ld + nat] = fixed_to_f32(__ldcg(a + R));
+      __stcg(a + R, 0LL);
     }
   }
-  __syncwarp();
-  finish_rowblock(pp, layer, rb, g_first, g_last, T, nw, upr, lane, epoch);
+  if (lane == 0) __stcg(p.ep.cnt + rb, 0);
 }
 
-// End of one row-block segment of a warp's run: store the piece (slot 0:
-// the run's first segment, slot 1: a later one) and publish it.  A whole
-// row-block is finished at once; a split one is merged by the owner of its
-// last unit after that warp's run (gemv_phase) -- the owner itself (owner
-// set) publishes nothing.
+// End of one row-block segment (units of row-block rb) of a warp's run: add
+// the sums to the accumulator, then count the units (see EpiArgs).
 template <int NT>
-__device__ __forceinline__ void piece_end(const GemvPhase* pp, int layer, const float (&tot)[4][NT][4], int rb, bool whole,
-                                          bool owner, int slot, int g, int nw, int T, int upr, unsigned epoch,
-                                          int lane) {
+__device__ __forceinline__ void segment_end(const GemvPhase* pp, const float (&tot)[4][NT][4], int rb, int units,
+                                            int upr, int lane) {
   const GemvPhase& p = *pp;
   const int gid = lane >> 2, tig = lane & 3;
-  float* mine = p.partials + ((size_t)g * 2 + slot) * kPieceFloats;
+  const int kind = p.ep.kind;
+  const int rows = kind == EPI_RESID ? p.ep.dims.H : 0x7FFFFFFF;
 #pragma unroll
   for (int rt = 0; rt < 4; ++rt)
 #pragma unroll
@@ -511,49 +378,56 @@ __device__ __forceinline__ void piece_end(const GemvPhase* pp, int layer, const 
       for (int c = 0; c < 2; ++c) {
         const int m = nt * 8 + 2 * tig + c;
         if (m < p.M) {
-          __stcg(mine + m * kRowsPerBlock + rt * 16 + gid, tot[rt][nt][c]);
-          __stcg(mine + m * kRowsPerBlock + rt * 16 + gid + 8, tot[rt][nt][2 + c]);
+          long long* a = p.ep.acc + (size_t)m * p.ep.acc_ld + rb * kRowsPerBlock + rt * 16 + gid;
+          if (rb * kRowsPerBlock + rt * 16 + gid < rows) red_add_s64(a, __float2ll_rn(tot[rt][nt][c] * kTotScaleLo));
+          if (rb * kRowsPerBlock + rt * 16 + gid + 8 < rows)
+            red_add_s64(a + 8, __float2ll_rn(tot[rt][nt][2 + c] * kTotScaleHi));
         }
       }
+  if (kind == EPI_RESID) return;
+  // The warp barrier orders every lane's additions before lane 0's release
+  // (and lane 0's acquire before the finisher's loads).
   __syncwarp();
-  if (whole) {
-    finish_rowblock(pp, layer, rb, g, g, T, nw, upr, lane, epoch);
+  if (kind == EPI_QKV) {
+    if (lane == 0) red_release_add_s32(p.ep.cnt + kv_head_of(p, rb), units);
     return;
   }
-  // The warp barrier above orders every lane's piece stores before lane 0's
-  // release; the merging warp's acquire loads pair with it.
-  if (!owner && lane == 0) st_release_u32(p.flags + (size_t)g * 2 + slot, epoch);
+  int last = 0;
+  if (lane == 0) last = atom_add_acq_rel(p.ep.cnt + rb, units) + units == upr;
+  last = __shfl_sync(0xffffffffu, last, 0);
+  __syncwarp();
+  if (!last) return;
+  if (kind == EPI_SWIGLU)
+    finish_swiglu(pp, rb, lane);
+  else
+    finish_store(pp, rb, lane);
 }
 
-// One projection for one warp: consume the warp's run of units from the
-// stream (which must be positioned at this op) and finish or hand on each
-// row-block segment of it.
+// One projection for one warp: consume the warp's run of units from its ring
+// (which the producer fills in the same order) and hand on each row-block
+// segment of it.
 //
 // Not inlined: the step's four projections run this one copy of the code, so
-// it stays in the instruction cache.  The stream state and the phase
-// arguments live in shared memory (ws_io, pp): nothing crosses the call
-// through the stack, whose local memory would miss the small L1 left next to
-// the weight rings.  The stream state is worked on in registers and written
-// back at the end.
+// it stays in the instruction cache.  The ring state and the phase arguments
+// live in shared memory (ring_io, pp): nothing crosses the call through the
+// stack, whose local memory would miss the small L1 left next to the weight
+// rings.
 template <int NT, int GPU>
-__device__ __noinline__ void gemv_phase(WarpStream<GPU>* ws_io, int op, const GemvPhase* pp, int layer, unsigned epoch,
+__device__ __noinline__ void gemv_phase(WarpRing<GPU>* ring_io, const OpDesc* op, const GemvPhase* pp, int g, int nw,
                                         int lane) {
-  WarpStream<GPU> ws = *ws_io;
+  WarpRing<GPU> ring = *ring_io;
   const GemvPhase& p = *pp;
-  int wb, we;
-  ws.warp_range(op, wb, we);
+  const int upr = op->upr;
+  const int T = op->n_rb * upr;
+  const int wb = part_start(T, g, nw), we = part_start(T, g + 1, nw);
   if (wb >= we) return;
-  const int upr = ws.ops[op].upr;
-  const int T = ws.ops[op].n_rb * upr;
-  const int g = ws.cta * ws.cta_warps + ws.warp, nw = ws.n_cta * ws.cta_warps;
   const uint16_t* actp = p.act;
   const uint32_t acts = p.act_s;
   const int act_ld = acts ? p.act_s_ld : p.act_ld, M = p.M;
-  const bool skip = p.skip;
   int rb = wb / upr;
   int ku = wb - rb * upr;
   uint4 nxt[NT][2][2];
-  load_act<NT>(nxt, actp, acts, act_ld, M, skip, ku, lane);
+  load_act<NT>(nxt, actp, acts, act_ld, M, ku, lane);
   for (int u = wb; u < we; ++rb) {
     const int seg_begin = u, rb_end = (rb + 1) * upr;
     const int seg_end = we < rb_end ? we : rb_end;
@@ -564,7 +438,7 @@ __device__ __noinline__ void gemv_phase(WarpStream<GPU>* ws_io, int op, const Ge
       for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
         for (int q = 0; q < 4; ++q) tot[rt][nt][q] = 0.f;
-#pragma unroll 2  // alternating activation registers instead of copies (measured ~1 % faster)
+#pragma unroll 2  // alternating activation registers instead of copies
     for (; u < seg_end; ++u) {
       uint4 cur[NT][2][2];
 #pragma unroll
@@ -574,27 +448,16 @@ __device__ __noinline__ void gemv_phase(WarpStream<GPU>* ws_io, int op, const Ge
 #pragma unroll
           for (int h = 0; h < 2; ++h) cur[nt][kc][h] = nxt[nt][kc][h];
       if (++ku == upr) ku = 0;
-      if (u + 1 < we) load_act<NT>(nxt, actp, acts, act_ld, M, skip, ku, lane);
-      const uint8_t* U = ws.acquire();
-      if (!skip && !ws.timed_out) mma_unit<NT, GPU>(U, cur, tot, lane);
-      ws.release(lane);
+      if (u + 1 < we) load_act<NT>(nxt, actp, acts, act_ld, M, ku, lane);
+      const uint8_t* U = ring.acquire();
+      if (!ring.timed_out) mma_unit<NT, GPU>(U, cur, tot, lane);
+      ring.release(lane);
     }
-    if (!skip) {
-      const bool whole = (seg_begin == rb * upr && seg_end == rb_end);
-      piece_end<NT>(pp, layer, tot, rb, whole, seg_end == rb_end, seg_begin == wb ? 0 : 1, g, nw, T, upr, epoch,
-                    lane);
-    }
+    segment_end<NT>(pp, tot, rb, seg_end - seg_begin, upr, lane);
   }
   __syncwarp();
-  if (lane == 0) *ws_io = ws;
+  if (lane == 0) *ring_io = ring;
   __syncwarp();
-  if (!skip) {
-    // merge the split row-blocks whose last unit is this warp's
-    for (int r = wb / upr; r * upr + upr <= we; ++r) {
-      if (r * upr >= wb) continue;  // whole inside the run: already finished
-      merge_rowblock(pp, layer, r, part_of(T, r * upr, nw), g, T, nw, upr, epoch, lane);
-    }
-  }
 }
 
 }  // namespace shard

@@ -260,9 +260,8 @@ struct head_s {
   uint16_t* act = nullptr;      // fp16 [16][Kp], padding columns zero
   float* logits = nullptr;      // fp32 [16][ld]
   int ld = 0;
-  float* partials = nullptr;    // projection pieces
-  unsigned* flags = nullptr;    // projection piece flags
-  unsigned epoch = 1;
+  long long* acc = nullptr;     // projection sums [16][n_rb * 64], fixed point, zero between calls
+  int* cnt = nullptr;           // projection units finished per row-block, zero between calls
   int* status = nullptr;
   Top1Part* parts = nullptr;    // [16][max chunks]
   int* done = nullptr;          // [16] chunk arrivals per row (self-resetting)
@@ -282,8 +281,8 @@ void destroy(head_s* h) {
   cudaFree(h->norm);
   cudaFree(h->act);
   cudaFree(h->logits);
-  cudaFree(h->partials);
-  cudaFree(h->flags);
+  cudaFree(h->acc);
+  cudaFree(h->cnt);
   cudaFree(h->status);
   cudaFree(h->parts);
   cudaFree(h->done);
@@ -304,16 +303,6 @@ int chunk_of(const head_s* h, int M, int* n_chunks) {
   return chunk;
 }
 
-unsigned next_epoch(head_s* h) {
-  if (h->epoch >= 0xFFFFFFF0u) {  // wrap-around: no stale flag may match a reused epoch
-    cudaDeviceSynchronize();
-    cudaMemset(h->flags, 0, sizeof(unsigned) * gemv_flags_count(h->grid[0]));
-    cudaDeviceSynchronize();
-    h->epoch = 1;
-  }
-  return h->epoch++;
-}
-
 // norm -> projection -> top-1 (logits only, when token == nullptr).  No
 // status copy per call: a copy-engine transfer between the calls' kernels
 // measured ~9 us of stream time per call; the top-1 kernel reports a failed
@@ -330,13 +319,12 @@ int run(head_s* h, const uint16_t* hidden, int M, int32_t* token, float* p_max, 
   g.act = h->act;
   g.act_ld = h->op.Kp;
   g.M = M;
-  g.sp = nullptr;
-  g.partials = h->partials;
-  g.flags = h->flags;
-  g.epoch = next_epoch(h);
   g.status = h->status;
   g.ep.kind = EPI_STORE;
   g.ep.dims = h->op.dims;
+  g.ep.acc = h->acc;
+  g.ep.acc_ld = h->op.n_rb * kRowsPerBlock;
+  g.ep.cnt = h->cnt;
   g.ep.y = logits;
   g.ep.y_ld = ld;
   const int nt = M <= 8 ? 1 : 2;
@@ -428,9 +416,11 @@ int head_create(const head_config* cfg, const head_weights_host* w, head_t* out)
          HEAD_CUDA_TRY(cudaMemset(h->act, 0, sizeof(uint16_t) * kMaxTokens * op.Kp));
          h->ld = (c.vocab + 3) / 4 * 4;
          HEAD_CUDA_TRY(cudaMalloc(&h->logits, sizeof(float) * kMaxTokens * h->ld));
-         HEAD_CUDA_TRY(cudaMalloc(&h->partials, sizeof(float) * gemv_partials_floats(h->grid[0])));
-         HEAD_CUDA_TRY(cudaMalloc(&h->flags, sizeof(unsigned) * gemv_flags_count(h->grid[0])));
-         HEAD_CUDA_TRY(cudaMemset(h->flags, 0, sizeof(unsigned) * gemv_flags_count(h->grid[0])));
+         const size_t acc_n = (size_t)kMaxTokens * op.n_rb * kRowsPerBlock;
+         HEAD_CUDA_TRY(cudaMalloc(&h->acc, sizeof(long long) * acc_n));
+         HEAD_CUDA_TRY(cudaMemset(h->acc, 0, sizeof(long long) * acc_n));
+         HEAD_CUDA_TRY(cudaMalloc(&h->cnt, sizeof(int) * op.n_rb));
+         HEAD_CUDA_TRY(cudaMemset(h->cnt, 0, sizeof(int) * op.n_rb));
          HEAD_CUDA_TRY(cudaMalloc(&h->status, sizeof(int)));
          HEAD_CUDA_TRY(cudaMemset(h->status, 0, sizeof(int)));
          h->max_chunks = (c.vocab + kTopChunkMin - 1) / kTopChunkMin + 1;

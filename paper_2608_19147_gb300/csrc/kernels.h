@@ -95,8 +95,19 @@ struct PackedOp {
   OpDims dims{};
 };
 
-// Step parameters, written on the device by the step prologue and read by
-// every later kernel of the step.
+// Fixed-point accumulation.  Split projections add their partial sums with
+// 64-bit integer atomics into accumulators holding round(value * 2^32):
+// integer addition is associative, so a sum does not depend on the order in
+// which contributions arrive -- results are deterministic and a request's
+// rows are independent of what else is in the batch -- and the sum of the
+// fp32 partials is exact (partials above 2^-9 in magnitude convert without
+// rounding; the range is +-2^31).
+constexpr float kFixOne = 4294967296.0f;             // 2^32
+constexpr double kFixInv = 2.3283064365386962890625e-10;  // 2^-32
+
+// Per-step request/token bookkeeping.  The step kernel derives it in every
+// CTA from the step's arguments (the same values everywhere), so no CTA waits
+// for another to publish it.
 struct StepParams {
   int M, B, abort_step, pad0;
   int tok_req[kMaxTokens];
@@ -104,57 +115,98 @@ struct StepParams {
   int tok_pos[kMaxTokens];
   int tok_slot[kMaxTokens];   // physical slot: phys_row * capacity + position in row
   int req_tok0[kMaxRequests + 1];
+  int req_src[kMaxRequests];  // beam_idx[b] (the row whose entries row b continues)
   int req_P[kMaxRequests];    // row length after the gather, before the append
   int req_len[kMaxRequests];  // row length after the append
-  const uint8_t* mask;
-  int mask_stride, pad1;
-  uint16_t* hidden_out;
-  const int* bt;     // current beam table [n_rows][capacity]
 };
 
 enum EpiKind { EPI_STORE = 0, EPI_QKV = 1, EPI_RESID = 2, EPI_SWIGLU = 3 };
 
+// Where a projection's row-block sums go.
+//   EPI_RESID   acc = the residual stream X [16][H] (fixed point): x += W a.
+//   EPI_QKV     acc = q|k|v sums [16][acc_ld] in the op's row order; each
+//               segment then adds its unit count to cnt[kv head of the
+//               row-block] (release), which the attention items wait for.
+//   EPI_SWIGLU  acc = gate|up sums [16][acc_ld]; cnt[row-block] counts the
+//               units added; the contributor that completes a row-block reads
+//               the sums, writes h = fp16(silu(gate) * up) and clears the
+//               sums and the count.
+//   EPI_STORE   as EPI_SWIGLU, but the completing contributor writes the fp32
+//               sums to y[m][natural row].
 struct EpiArgs {
   int kind;
   OpDims dims;
-  float* y;  // EPI_STORE: y[m][natural row], row stride y_ld
+  long long* acc;
+  int acc_ld;
+  int* cnt;
+  float* y;       // EPI_STORE: y[m][natural row], row stride y_ld
   int y_ld;
-  float* q;                   // EPI_QKV: q fp32 [M][Hq*d]
-  uint16_t* kpool;            // EPI_QKV: layer 0's K pool [n_rows][Hkv][cap][d]; layer l at + l * layer_stride
-  uint16_t* vpool;
-  size_t layer_stride;
-  int cap;
-  const float2* rope;         // [max_position][d/2] (cos, sin)
-  float* x;                   // EPI_RESID: residual [M][H]
-  float* ss;                  // EPI_RESID (or nullptr): per row-block sums of squares of x [n_rb][16]
-  int out_layer;              // EPI_RESID: in this layer also write fp16(x) to sp->hidden_out (-1: never)
-  uint16_t* h;                // EPI_SWIGLU: fp16 [M][h_ld]
+  uint16_t* h;    // EPI_SWIGLU: fp16 [M][h_ld]
   int h_ld;
 };
 
 struct GemvArgs {
   const uint8_t* units;
   int n_rb, upr;
-  const uint16_t* act;  // fp16 activations [M][act_ld]
+  const uint16_t* act;  // fp16 activations [M][act_ld] (act_ld a multiple of 128, zero padded)
   int act_ld;
-  int M;                // tokens when sp == nullptr
-  const StepParams* sp; // step parameters (nullptr on the standalone path)
-  float* partials;      // [grid warps][2][piece] fp32 scratch, gemv_partials_floats(grid)
-  unsigned* flags;      // [grid warps][2] piece flags (gemv_flags_count(grid)), zero-initialised
-  unsigned epoch;       // nonzero, different from every earlier launch on these flags
+  int M;
   int* status;
-  EpiArgs ep;
+  EpiArgs ep;           // EPI_STORE: acc [16][n_rb * 64] and cnt [n_rb] zero on entry (left zero)
 };
 
-// Launch geometry of the GEMV for a given token bucket (nt = 1: M <= 8,
-// nt = 2: M <= 16).
+// Launch geometry of the standalone projection for a given token bucket
+// (nt = 1: M <= 8, nt = 2: M <= 16).
 int gemv_grid(int nt, int num_sms);
-size_t gemv_partials_floats(int grid);
-size_t gemv_flags_count(int grid);
 cudaError_t launch_gemv(const GemvArgs& a, int nt, int group, int grid, cudaStream_t s, bool pdl);
 // One-time per-device kernel attribute setup (dynamic shared memory limits).
 cudaError_t gemv_setup();
 int gemv_warps_per_cta();
+
+// Many-token projection on the tensor cores (gemm_tc.cu): y[n][natural
+// row] = sum_k W[r][k] act[n][k] for n < S.
+struct GemmArgs {
+  const uint8_t* units;
+  int n_rb, upr;
+  const uint16_t* act;  // fp16 [S][act_ld], act_ld a multiple of 128, zero padded past K
+  int act_ld, S;
+  float* y;             // fp32 [S][y_ld]
+  int y_ld;
+  OpDims dims;
+  int* status;
+};
+cudaError_t gemm_tc_setup();
+int gemm_tc_tile(int S);
+cudaError_t launch_gemm_tc(const GemmArgs& a, int group, cudaStream_t s);
+
+// Prefill (prefill.cu): per-token kernels around the tensor-core projections.
+struct PrefillLayerArgs {
+  const float* y;        // q|k|v projection outputs [S][y_ld], natural rows
+  int y_ld, S, Hq, Hkv, d;
+  const int* pos;        // [S] RoPE positions
+  int max_position;
+  const float2* rope;    // [max_position][d/2]
+  float* q;              // [S][Hq*d] rotated queries
+  uint16_t* kpool;       // this layer's K pool [n_rows][Hkv][cap][d]
+  uint16_t* vpool;
+  int row, cap, slot0;   // the row and the position in it of the first new entry
+  const int* bt_row;     // the row's beam table
+  const uint8_t* mask;   // the row's attention mask
+  int P;                 // entries before the first token of this chunk
+  uint16_t* attn;        // [S][attn_ld] fp16 attention output
+  int attn_ld;
+};
+cudaError_t launch_prefill_check(const int* token_ids, int vocab, const int* pos, int max_position, const uint8_t* mask,
+                                 int P, int S, int* status, cudaStream_t s);
+cudaError_t launch_prefill_embed(const uint16_t* hidden_in, const int* token_ids, const uint16_t* embedding, int H,
+                                 int S, int vocab, float* x, cudaStream_t s);
+cudaError_t launch_prefill_norm(const float* x, int H, const uint16_t* w, float eps, uint16_t* act, int act_ld, int S,
+                                cudaStream_t s);
+cudaError_t launch_prefill_rope_append(const PrefillLayerArgs& a, cudaStream_t s);
+cudaError_t launch_prefill_attention(const PrefillLayerArgs& a, cudaStream_t s);
+cudaError_t launch_prefill_swiglu(const float* y, int y_ld, int S, int F, uint16_t* h, int h_ld, cudaStream_t s);
+cudaError_t launch_prefill_residual(float* x, const float* y, int y_ld, int S, int H, uint16_t* out, cudaStream_t s);
+cudaError_t launch_set_int(int* p, int v, cudaStream_t s);
 
 struct PrologueArgs {
   int B, M;
@@ -166,16 +218,14 @@ struct PrologueArgs {
   const int* position_ids;
   const uint8_t* mask;
   int mask_stride;
+  int packed;            // the mask has one row per token (one request): shard_step_packed
   uint16_t* hidden_out;
   const int* bt_src;
   int* bt_dst;
-  int* lens;             // [n_rows] row lengths (updated)
+  int* lens;             // [n_rows] row lengths (updated at the end of the step)
   int cap, max_position, vocab, H;
   const uint16_t* embedding;
-  float* x;              // residual [M][H]
-  float* ss;             // per 64-row block sums of squares of x [n_rb_H][16]
   int* status;
-  StepParams* sp;
 };
 
 // A projection's unit stream as the device code walks it.
@@ -192,28 +242,31 @@ struct StepKernelArgs {
   float eps;
   const uint16_t* norms;     // [L][2][H]
   const float2* rope;        // [max_position][d/2]
-  float* x;                  // residual [16][H]
-  float* ss;                 // per 64-row block sums of squares of x [n_rb_H][16]
-  uint16_t* act_h;           // [16][Kp_H]
+  long long* X;              // residual [16][H], fixed point
+  long long* acc_qkv;        // [16][qkv rows], zero between steps
+  long long* acc_gu;         // [16][gate|up rows], zero between steps
+  int* cnt_kv;               // [Hkv] q|k|v units finished per kv head, zero between steps
+  int* cnt_gu;               // [gate|up row-blocks], zero between steps
+  uint16_t* act_h;           // [16][Kp_H] (normalised rows, when they do not fit in shared memory)
   uint16_t* act_attn;        // [16][Kp_dq]
   uint16_t* act_f;           // [16][Kp_F]
-  float* q;                  // [16][Hq*d]
-  float* partials;           // projection pieces, gemv_partials_floats(grid)
-  unsigned* flags;           // projection piece flags, gemv_flags_count(grid), zero-initialised
-  unsigned epoch_base;       // projection op of this launch publishes epoch_base + op (unique per launch)
   uint16_t* kpool;           // [L][n_rows][Hkv][cap][d]
   uint16_t* vpool;
   size_t layer_stride;
   int cap, n_chunks;         // items per row at kAttnChunkMin entries (the partials layout)
+  const uint8_t* mask;
+  int mask_stride;
+  int packed;                // mask row per token (one request), no implicit causal bound
   float* attn_part;          // [B][Hkv][n_chunks][16*G][d+4]
   int* attn_cnt;             // [16][Hkv] finished chunks per (request, kv head); zero, self-resetting
-  unsigned* rb_done;         // [max row-blocks] epoch of each q|k|v row-block's finish
   int* status;
   unsigned long long* barrier;         // grid-barrier counter (monotonic)
   unsigned long long barrier_base;     // its value when this launch starts
   unsigned long long* phase_clock;     // [step_barriers(L) + 1] globaltimer at each barrier
   int* status_out;           // host-mapped mirror: the last CTA to finish copies a nonzero status there
   int* exit_count;           // CTAs finished in this launch (zero between launches; the last resets it)
+  int debug_skip_arrival;    // test knob: >= 0 makes CTA 1 skip that grid barrier's arrival
+  unsigned wait_limit;       // polls before a cross-CTA wait gives up
 };
 // One-time attribute setup of the step kernel variants for a group size and
 // head dim; number of grid barriers per step; launch (cooperative, one CTA

@@ -7,8 +7,8 @@
 // running while another thread holds the allocator, or a latency-critical
 // loop where an allocation's implicit device synchronisation is not
 // allowed.  Such a caller still owns its inputs and outputs; only the
-// kernel's scratch (the partial sums of split row-blocks, the flags that
-// publish them and a zero-padded copy of the activations) moves into the
+// kernel's scratch (the fixed-point row sums of split row-blocks, their
+// arrival counts and a zero-padded copy of the activations) moves into the
 // static array below, which every GPU that loads the library holds until
 // exit.
 #include <algorithm>
@@ -21,18 +21,14 @@
 namespace shard {
 namespace {
 
-// 4 MiB: at a fixed offset the piece flags of up to kMaxGrid CTAs and a
-// status word, then the partial sums of as many CTAs as fit next to the
-// padded activations (16 rows of up to 28672 inputs: 896 KiB).  The flags
-// only ever hold epochs, which are unique per device, so they need no
-// clearing between calls.
+// 4 MiB: the arrival counts of the op's row-blocks, then the row sums
+// (16 rows of up to 57344 int64 fit for M <= 8), then the padded
+// activations.  Every part is cleared by the call before its kernel runs.
 constexpr size_t kNoAllocScratchBytes = 4u << 20;
-constexpr int kMaxGrid = 256;
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 
 constexpr int kMaxDevices = 64;
 void* g_scratch_addr[kMaxDevices] = {};  // per-device address of g_noalloc_scratch
-unsigned g_epoch[kMaxDevices] = {};      // per-device last epoch used
 
 }  // namespace
 
@@ -41,6 +37,7 @@ unsigned g_epoch[kMaxDevices] = {};      // per-device last epoch used
 struct NoAllocView {
   const PackedOp* op;
   int group, grid_nt1, grid_nt2, device, rows;
+  int* status;  // the shard's device status word (shard_sync_status reports it)
 };
 int shard_noalloc_view(shard_t sh, int layer, int op, NoAllocView* v);
 int shard_noalloc_fail(int code, const char* msg);
@@ -51,6 +48,7 @@ using namespace shard;
 
 namespace {
 thread_local char g_msg[256];
+size_t align256(size_t v) { return (v + 255) / 256 * 256; }
 }
 
 extern "C" {
@@ -67,23 +65,15 @@ int shard_gemv_noalloc(shard_t sh, int layer, int op, const uint16_t* x, int M, 
   }
   const PackedOp& p = *v.op;
   const int nt = M <= 8 ? 1 : 2;
-  // Scratch layout: [flags + status word | partials | activations],
-  // 256-byte aligned parts.  The grid shrinks until its partials fit.
-  const size_t flag_bytes = ((gemv_flags_count(kMaxGrid) + 1) * sizeof(unsigned) + 255) / 256 * 256;
+  // Scratch layout: [counts | sums | activations], 256-byte aligned parts.
+  const size_t cnt_bytes = align256(sizeof(int) * (size_t)p.n_rb);
+  const size_t acc_ld = (size_t)p.n_rb * kRowsPerBlock;
+  const size_t acc_bytes = align256(sizeof(long long) * acc_ld * M);
   const size_t act_bytes = (size_t)M * p.Kp * sizeof(uint16_t);
-  const size_t per_cta = gemv_partials_floats(1) * sizeof(float);
-  long long fit = 0;
-  if (flag_bytes + act_bytes < kNoAllocScratchBytes)
-    fit = (long long)((kNoAllocScratchBytes - flag_bytes - act_bytes) / per_cta);
-  const int grid = static_cast<int>(std::min<long long>(
-      std::min<long long>(std::min<long long>(nt == 1 ? v.grid_nt1 : v.grid_nt2, kMaxGrid), fit),
-      (long long)p.n_rb * p.upr));
-  const size_t part_bytes = (gemv_partials_floats(grid > 0 ? grid : 0) * sizeof(float) + 255) / 256 * 256;
-  if (grid < 1 || flag_bytes + part_bytes + act_bytes > kNoAllocScratchBytes) {
+  if (cnt_bytes + acc_bytes + act_bytes > kNoAllocScratchBytes) {
     snprintf(g_msg, sizeof(g_msg),
-             "shard_gemv_noalloc: needs %zu bytes of scratch for M=%d and K=%d plus %zu per CTA; "
-             "the fixed array has %zu",
-             flag_bytes + act_bytes, M, p.K, per_cta, kNoAllocScratchBytes);
+             "shard_gemv_noalloc: needs %zu bytes of scratch for M=%d, %d rows and K=%d; the fixed array has %zu",
+             cnt_bytes + acc_bytes + act_bytes, M, v.rows, p.K, kNoAllocScratchBytes);
     return shard_noalloc_fail(SHARD_ECAPACITY, g_msg);
   }
   if (y_ld < v.rows) {
@@ -107,20 +97,14 @@ int shard_gemv_noalloc(shard_t sh, int layer, int op, const uint16_t* x, int M, 
     g_scratch_addr[v.device] = ptr;
   }
   unsigned char* base = static_cast<unsigned char*>(g_scratch_addr[v.device]);
-  unsigned* flags = reinterpret_cast<unsigned*>(base);
-  int* status = reinterpret_cast<int*>(flags + gemv_flags_count(kMaxGrid));
-  float* partials = reinterpret_cast<float*>(base + flag_bytes);
-  uint16_t* act = reinterpret_cast<uint16_t*>(base + flag_bytes + part_bytes);
+  int* cnt = reinterpret_cast<int*>(base);
+  long long* acc = reinterpret_cast<long long*>(base + cnt_bytes);
+  uint16_t* act = reinterpret_cast<uint16_t*>(base + cnt_bytes + acc_bytes);
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
-  // The array keeps the previous call's contents: zero the status word and
-  // the activation padding; partial sums are written before being read.
-  if (g_epoch[v.device] == 0xFFFFFFFFu) {  // wrap-around: clear the flags first
-    e = cudaMemsetAsync(flags, 0, flag_bytes, s);
-    g_epoch[v.device] = 0;
-  }
-  const unsigned epoch = ++g_epoch[v.device];
-  if (e == cudaSuccess) e = cudaMemsetAsync(status, 0, sizeof(int), s);
-  if (e == cudaSuccess) e = cudaMemsetAsync(act, 0, act_bytes, s);
+  // The array keeps the previous call's contents: clear the counts, the sums
+  // and the activation padding (a completed call leaves counts and sums zero,
+  // one that gave up may not).
+  e = cudaMemsetAsync(base, 0, cnt_bytes + acc_bytes + act_bytes, s);
   if (e == cudaSuccess)
     e = cudaMemcpy2DAsync(act, sizeof(uint16_t) * p.Kp, x, sizeof(uint16_t) * p.K, sizeof(uint16_t) * p.K, M,
                           cudaMemcpyDeviceToDevice, s);
@@ -135,15 +119,15 @@ int shard_gemv_noalloc(shard_t sh, int layer, int op, const uint16_t* x, int M, 
   g.act = act;
   g.act_ld = p.Kp;
   g.M = M;
-  g.sp = nullptr;
-  g.partials = partials;
-  g.flags = flags;
-  g.epoch = epoch;
-  g.status = status;
+  g.status = v.status;
   g.ep.kind = EPI_STORE;
   g.ep.dims = p.dims;
+  g.ep.acc = acc;
+  g.ep.acc_ld = static_cast<int>(acc_ld);
+  g.ep.cnt = cnt;
   g.ep.y = y;
   g.ep.y_ld = y_ld;
+  const int grid = std::min<long long>(nt == 1 ? v.grid_nt1 : v.grid_nt2, (long long)p.n_rb * p.upr);
   e = launch_gemv(g, nt, v.group, grid, s, false);
   if (e != cudaSuccess) {
     snprintf(g_msg, sizeof(g_msg), "shard_gemv_noalloc: launch failed: %s", cudaGetErrorString(e));

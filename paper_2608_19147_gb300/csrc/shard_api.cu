@@ -76,24 +76,35 @@ struct shard_s {
   uint16_t* norms = nullptr;       // [L][2][H]
   uint16_t* embedding = nullptr;   // [V][H]
   float2* rope = nullptr;          // [max_position][d/2]
-  // per-step work buffers (one set per shard)
-  float* x = nullptr;              // [16][H]
-  float* ss = nullptr;             // [n_rb_H][16] per 64-row block sums of squares of x
+  // per-step work buffers (one set per shard); sums and counts are zero
+  // between launches (each launch leaves them so)
+  long long* X = nullptr;          // residual [16][H], fixed point
+  long long* acc_qkv = nullptr;    // [16][qkv rows]
+  long long* acc_gu = nullptr;     // [16][gate|up rows]
+  long long* acc_store = nullptr;  // [16][max_rb * 64] (the standalone projection)
+  int* cnt_kv = nullptr;           // [Hkv]
+  int* cnt_gu = nullptr;           // [gate|up row-blocks]
+  int* cnt_store = nullptr;        // [max_rb]
   int* attn_cnt = nullptr;         // [16][Hkv] attention chunks finished per (request, kv head)
-  unsigned* rb_done = nullptr;     // [max_rb] epoch of each q|k|v row-block's last finish
   uint16_t* act_h = nullptr;       // [16][Kp_H]
   uint16_t* act_attn = nullptr;    // [16][Kp_dq]
   uint16_t* act_f = nullptr;       // [16][Kp_F]
-  float* q = nullptr;              // [16][dq]
-  float* partials = nullptr;
-  unsigned* flags = nullptr;        // projection piece flags
-  unsigned epoch = 1;               // next epoch for the flags
   int max_rb = 0;
+  size_t acc_qkv_n = 0, acc_gu_n = 0, acc_store_n = 0;
+  int n_rb_gu = 0;
+  // prefill work buffers, allocated at the first shard_prefill (chunks of kPrefillChunk tokens)
+  float* pf_x = nullptr;           // [C][H] residual
+  uint16_t* pf_act = nullptr;      // [C][Kp_H] normalised rows (padding zero)
+  uint16_t* pf_attn = nullptr;     // [C][Kp_dq] attention output (padding zero)
+  uint16_t* pf_h = nullptr;        // [C][Kp_F] SwiGLU output (padding zero)
+  float* pf_y = nullptr;           // [C][max projection rows] projection outputs
+  float* pf_q = nullptr;           // [C][dq] rotated queries
+  int debug_skip_arrival = -1;     // test knob (shard_debug_set_wait)
+  unsigned wait_limit = 1u << 22;  // polls before a cross-CTA wait gives up
   int* status = nullptr;           // device status word
   int* status_host = nullptr;      // host-mapped mirror the step kernel writes a nonzero status to
   int* status_host_dev = nullptr;  // its device address
   int* exit_count = nullptr;       // step kernel: CTAs finished (zero between launches)
-  StepParams* sp = nullptr;
   int grid[3] = {0, 0, 0};         // standalone GEMV grid per token bucket
   OpDesc* ops_dev = nullptr;       // [4L] op descriptors for the step kernel
   unsigned long long* barrier = nullptr;  // grid-barrier counter
@@ -185,18 +196,21 @@ int op_K(int kind, const shard_s& s) {
 
 int nt_for(int M) { return M <= 8 ? 1 : 2; }
 
-// Reserves n consecutive flag epochs (never 0).  On wrap-around (after 2^32
-// epochs) the flags are cleared first, so no stale flag can match.
-unsigned next_epochs(shard_s* sh, unsigned n) {
-  if (sh->epoch > 0xFFFFFFFFu - n) {
-    cudaDeviceSynchronize();
-    cudaMemset(sh->flags, 0, sizeof(unsigned) * gemv_flags_count(std::max(std::max(sh->grid[1], sh->grid[2]), sh->num_sms)));
-    cudaMemset(sh->rb_done, 0, sizeof(unsigned) * sh->max_rb);
-    cudaDeviceSynchronize();
-    sh->epoch = 1;
-  }
-  const unsigned e = sh->epoch;
-  sh->epoch += n;
+// After a wait that gave up, the launch's sums, counts and grid-barrier
+// count are left in an unknown state: put every work buffer back to zero.
+cudaError_t reset_work_buffers(shard_s* sh) {
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e == cudaSuccess) e = cudaMemset(sh->acc_qkv, 0, sizeof(long long) * sh->acc_qkv_n);
+  if (e == cudaSuccess) e = cudaMemset(sh->acc_gu, 0, sizeof(long long) * sh->acc_gu_n);
+  if (e == cudaSuccess) e = cudaMemset(sh->acc_store, 0, sizeof(long long) * sh->acc_store_n);
+  if (e == cudaSuccess) e = cudaMemset(sh->cnt_kv, 0, sizeof(int) * sh->Hkv);
+  if (e == cudaSuccess) e = cudaMemset(sh->cnt_gu, 0, sizeof(int) * sh->n_rb_gu);
+  if (e == cudaSuccess) e = cudaMemset(sh->cnt_store, 0, sizeof(int) * sh->max_rb);
+  if (e == cudaSuccess) e = cudaMemset(sh->attn_cnt, 0, sizeof(int) * kMaxRequests * sh->Hkv);
+  if (e == cudaSuccess) e = cudaMemset(sh->exit_count, 0, sizeof(int));
+  if (e == cudaSuccess) e = cudaMemset(sh->barrier, 0, sizeof(unsigned long long));
+  if (e == cudaSuccess) e = cudaDeviceSynchronize();
+  sh->barrier_base = 0;
   return e;
 }
 
@@ -205,6 +219,7 @@ int check_pending_status(shard_s* sh) {
   if (bits) {
     *reinterpret_cast<volatile int*>(sh->status_host) = 0;
     for (auto* st : sh->states) st->poisoned = true;
+    if (bits & ST_WAIT_TIMEOUT) reset_work_buffers(sh);
     return fail(SHARD_EINVAL, "an earlier step was rejected on the device: %s", status_message(bits).c_str());
   }
   return SHARD_OK;
@@ -239,6 +254,7 @@ int shard_create(const shard_config* cfg, const shard_weights_host* w, shard_t* 
   CUDA_TRY(cudaDeviceGetAttribute(&sh->num_sms, cudaDevAttrMultiProcessorCount, sh->device));
   if (c.head_dim != 64 && c.head_dim != 128) return fail(SHARD_EUNSUPPORTED, "head_dim must be 64 or 128");
   CUDA_TRY(gemv_setup());
+  CUDA_TRY(gemm_tc_setup());
   CUDA_TRY(step_setup(c.group, c.head_dim));
   sh->cfg = c;
   sh->H = c.hidden;
@@ -370,29 +386,25 @@ int shard_create(const shard_config* cfg, const shard_weights_host* w, shard_t* 
   }
 
   // Work buffers.
-  CUDA_TRY(cudaMalloc(&sh->x, sizeof(float) * kMaxTokens * sh->H));
-  CUDA_TRY(cudaMalloc(&sh->ss, sizeof(float) * kMaxTokens * ((sh->H + kRowsPerBlock - 1) / kRowsPerBlock)));
+  CUDA_TRY(cudaMalloc(&sh->X, sizeof(long long) * kMaxTokens * sh->H));
+  sh->acc_qkv_n = (size_t)kMaxTokens * (sh->dq + 2 * sh->dkv);
+  sh->n_rb_gu = sh->ops[OP_GU].n_rb;
+  sh->acc_gu_n = (size_t)kMaxTokens * sh->n_rb_gu * kRowsPerBlock;
+  sh->acc_store_n = (size_t)kMaxTokens * sh->max_rb * kRowsPerBlock;
+  CUDA_TRY(cudaMalloc(&sh->acc_qkv, sizeof(long long) * sh->acc_qkv_n));
+  CUDA_TRY(cudaMalloc(&sh->acc_gu, sizeof(long long) * sh->acc_gu_n));
+  CUDA_TRY(cudaMalloc(&sh->acc_store, sizeof(long long) * sh->acc_store_n));
+  CUDA_TRY(cudaMalloc(&sh->cnt_kv, sizeof(int) * sh->Hkv));
+  CUDA_TRY(cudaMalloc(&sh->cnt_gu, sizeof(int) * sh->n_rb_gu));
+  CUDA_TRY(cudaMalloc(&sh->cnt_store, sizeof(int) * sh->max_rb));
   CUDA_TRY(cudaMalloc(&sh->attn_cnt, sizeof(int) * kMaxRequests * sh->Hkv));
-  CUDA_TRY(cudaMemset(sh->attn_cnt, 0, sizeof(int) * kMaxRequests * sh->Hkv));
-  CUDA_TRY(cudaMalloc(&sh->rb_done, sizeof(unsigned) * sh->max_rb));
-  CUDA_TRY(cudaMemset(sh->rb_done, 0, sizeof(unsigned) * sh->max_rb));
   CUDA_TRY(cudaMalloc(&sh->act_h, sizeof(uint16_t) * kMaxTokens * sh->Kp_H));
   CUDA_TRY(cudaMalloc(&sh->act_attn, sizeof(uint16_t) * kMaxTokens * sh->Kp_dq));
   CUDA_TRY(cudaMalloc(&sh->act_f, sizeof(uint16_t) * kMaxTokens * sh->Kp_F));
   CUDA_TRY(cudaMemset(sh->act_h, 0, sizeof(uint16_t) * kMaxTokens * sh->Kp_H));
   CUDA_TRY(cudaMemset(sh->act_attn, 0, sizeof(uint16_t) * kMaxTokens * sh->Kp_dq));
   CUDA_TRY(cudaMemset(sh->act_f, 0, sizeof(uint16_t) * kMaxTokens * sh->Kp_F));
-  CUDA_TRY(cudaMalloc(&sh->q, sizeof(float) * kMaxTokens * sh->dq));
   for (int nt = 1; nt <= 2; ++nt) sh->grid[nt] = gemv_grid(nt, sh->num_sms);
-  {
-    const size_t n = gemv_partials_floats(std::max(std::max(sh->grid[1], sh->grid[2]), sh->num_sms));
-    CUDA_TRY(cudaMalloc(&sh->partials, sizeof(float) * n));
-  }
-  {
-    const size_t nf = gemv_flags_count(std::max(std::max(sh->grid[1], sh->grid[2]), sh->num_sms));
-    CUDA_TRY(cudaMalloc(&sh->flags, sizeof(unsigned) * nf));
-    CUDA_TRY(cudaMemset(sh->flags, 0, sizeof(unsigned) * nf));
-  }
   CUDA_TRY(cudaMalloc(&sh->status, sizeof(int)));
   CUDA_TRY(cudaMemset(sh->status, 0, sizeof(int)));
   CUDA_TRY(cudaHostAlloc(&sh->status_host, sizeof(int), cudaHostAllocMapped));
@@ -400,8 +412,6 @@ int shard_create(const shard_config* cfg, const shard_weights_host* w, shard_t* 
   CUDA_TRY(cudaHostGetDevicePointer(reinterpret_cast<void**>(&sh->status_host_dev), sh->status_host, 0));
   CUDA_TRY(cudaMalloc(&sh->exit_count, sizeof(int)));
   CUDA_TRY(cudaMemset(sh->exit_count, 0, sizeof(int)));
-  CUDA_TRY(cudaMalloc(&sh->sp, sizeof(StepParams)));
-  CUDA_TRY(cudaMemset(sh->sp, 0, sizeof(StepParams)));
   {
     std::vector<OpDesc> od(sh->ops.size());
     for (size_t i = 0; i < od.size(); ++i) od[i] = OpDesc{sh->ops[i].units, sh->ops[i].n_rb, sh->ops[i].upr};
@@ -410,10 +420,9 @@ int shard_create(const shard_config* cfg, const shard_weights_host* w, shard_t* 
   }
   sh->n_barriers = step_barriers(sh->L);
   CUDA_TRY(cudaMalloc(&sh->barrier, sizeof(unsigned long long)));
-  CUDA_TRY(cudaMemset(sh->barrier, 0, sizeof(unsigned long long)));
   CUDA_TRY(cudaMalloc(&sh->phase_clock, sizeof(unsigned long long) * (sh->n_barriers + 1)));
   CUDA_TRY(cudaMemset(sh->phase_clock, 0, sizeof(unsigned long long) * (sh->n_barriers + 1)));
-  CUDA_TRY(cudaDeviceSynchronize());
+  CUDA_TRY(reset_work_buffers(sh.get()));
   *out = sh.release();
   return SHARD_OK;
 }
@@ -427,19 +436,25 @@ int shard_destroy(shard_t sh) {
   cudaFree(sh->norms);
   cudaFree(sh->embedding);
   cudaFree(sh->rope);
-  cudaFree(sh->x);
-  cudaFree(sh->ss);
+  cudaFree(sh->pf_x);
+  cudaFree(sh->pf_act);
+  cudaFree(sh->pf_attn);
+  cudaFree(sh->pf_h);
+  cudaFree(sh->pf_y);
+  cudaFree(sh->pf_q);
+  cudaFree(sh->X);
+  cudaFree(sh->acc_qkv);
+  cudaFree(sh->acc_gu);
+  cudaFree(sh->acc_store);
+  cudaFree(sh->cnt_kv);
+  cudaFree(sh->cnt_gu);
+  cudaFree(sh->cnt_store);
   cudaFree(sh->attn_cnt);
-  cudaFree(sh->rb_done);
   cudaFree(sh->act_h);
   cudaFree(sh->act_attn);
   cudaFree(sh->act_f);
-  cudaFree(sh->q);
-  cudaFree(sh->partials);
-  cudaFree(sh->flags);
   cudaFree(sh->status);
   cudaFree(sh->exit_count);
-  cudaFree(sh->sp);
   cudaFree(sh->dstage);
   if (sh->pin) cudaFreeHost(sh->pin);
   if (sh->status_host) cudaFreeHost(sh->status_host);
@@ -665,13 +680,36 @@ int kv_trim(kvstate_t st, int row, const uint8_t* keep, int len) {
   return SHARD_OK;
 }
 
+static int step_impl(shard_t sh, kvstate_t st, const uint16_t* hidden_in, const int32_t* token_ids,
+                     const int32_t* n_new, int B, const int32_t* position_ids, const uint8_t* attention_mask,
+                     int mask_stride, const int32_t* beam_idx, uint16_t* hidden_out, void* cuda_stream, int packed);
+
 int shard_step(shard_t sh, kvstate_t st, const uint16_t* hidden_in, const int32_t* token_ids, const int32_t* n_new,
                int B, const int32_t* position_ids, const uint8_t* attention_mask, int mask_stride,
                const int32_t* beam_idx, uint16_t* hidden_out, void* cuda_stream) {
+  return step_impl(sh, st, hidden_in, token_ids, n_new, B, position_ids, attention_mask, mask_stride, beam_idx,
+                   hidden_out, cuda_stream, 0);
+}
+
+int shard_step_packed(shard_t sh, kvstate_t st, const uint16_t* hidden_in, const int32_t* token_ids, int S,
+                      const int32_t* position_ids, const uint8_t* mask2d, int mask_stride, uint16_t* hidden_out,
+                      void* cuda_stream) {
+  if (!st || st->n_rows != 1) return fail(SHARD_EINVAL, "shard_step_packed: the state must have exactly one row");
+  if (S < 1 || S > SHARD_MAX_TOKENS) return fail(SHARD_EINVAL, "shard_step_packed: S = %d outside [1, %d]", S, SHARD_MAX_TOKENS);
+  const int32_t n_new[1] = {S};
+  return step_impl(sh, st, hidden_in, token_ids, n_new, 1, position_ids, mask2d, mask_stride, nullptr, hidden_out,
+                   cuda_stream, 1);
+}
+
+static int step_impl(shard_t sh, kvstate_t st, const uint16_t* hidden_in, const int32_t* token_ids,
+                     const int32_t* n_new, int B, const int32_t* position_ids, const uint8_t* attention_mask,
+                     int mask_stride, const int32_t* beam_idx, uint16_t* hidden_out, void* cuda_stream, int packed) {
   if (!sh || !st || st->sh != sh) return fail(SHARD_EINVAL, "shard_step: shard/state mismatch");
   if (!n_new || !position_ids || !attention_mask || !hidden_out) return fail(SHARD_EINVAL, "shard_step: null argument");
   if ((hidden_in == nullptr) == (token_ids == nullptr))
     return fail(SHARD_EINVAL, "shard_step: pass exactly one of hidden_in and token_ids");
+  if (reinterpret_cast<uintptr_t>(hidden_in) % 16)
+    return fail(SHARD_EINVAL, "shard_step: hidden_in must be 16-byte aligned");
   if (token_ids && sh->cfg.vocab <= 0) return fail(SHARD_EUNSUPPORTED, "shard_step: this shard has no embedding");
   if (B != st->n_rows) return fail(SHARD_EINVAL, "shard_step: B (%d) must equal the state's n_rows (%d)", B, st->n_rows);
   if (mask_stride < 1) return fail(SHARD_EINVAL, "shard_step: mask_stride must be >= 1");
@@ -711,6 +749,7 @@ int shard_step(shard_t sh, kvstate_t st, const uint16_t* hidden_in, const int32_
   pa.position_ids = position_ids;
   pa.mask = attention_mask;
   pa.mask_stride = mask_stride;
+  pa.packed = packed;
   pa.hidden_out = hidden_out;
   pa.bt_src = st->bt[st->bt_cur];
   pa.bt_dst = st->bt[beam_idx ? st->bt_cur ^ 1 : st->bt_cur];
@@ -720,10 +759,7 @@ int shard_step(shard_t sh, kvstate_t st, const uint16_t* hidden_in, const int32_
   pa.vocab = sh->cfg.vocab;
   pa.H = sh->H;
   pa.embedding = sh->embedding;
-  pa.x = sh->x;
-  pa.ss = sh->ss;
   pa.status = sh->status;
-  pa.sp = sh->sp;
   StepKernelArgs ka{};
   ka.pro = pa;
   ka.ops = sh->ops_dev;
@@ -739,15 +775,17 @@ int shard_step(shard_t sh, kvstate_t st, const uint16_t* hidden_in, const int32_
   ka.eps = static_cast<float>(sh->cfg.rms_eps);
   ka.norms = sh->norms;
   ka.rope = sh->rope;
-  ka.x = sh->x;
-  ka.ss = sh->ss;
+  ka.X = sh->X;
+  ka.acc_qkv = sh->acc_qkv;
+  ka.acc_gu = sh->acc_gu;
+  ka.cnt_kv = sh->cnt_kv;
+  ka.cnt_gu = sh->cnt_gu;
   ka.act_h = sh->act_h;
   ka.act_attn = sh->act_attn;
   ka.act_f = sh->act_f;
-  ka.q = sh->q;
-  ka.partials = sh->partials;
-  ka.flags = sh->flags;
-  ka.epoch_base = next_epochs(sh, 4 * sh->L);
+  ka.mask = attention_mask;
+  ka.mask_stride = mask_stride;
+  ka.packed = packed;
   ka.kpool = st->k;
   ka.vpool = st->v;
   ka.layer_stride = st->layer_stride;
@@ -755,8 +793,9 @@ int shard_step(shard_t sh, kvstate_t st, const uint16_t* hidden_in, const int32_
   ka.n_chunks = st->n_chunks;
   ka.attn_part = st->attn_part;
   ka.attn_cnt = sh->attn_cnt;
-  ka.rb_done = sh->rb_done;
   ka.status = sh->status;
+  ka.debug_skip_arrival = sh->debug_skip_arrival;
+  ka.wait_limit = sh->wait_limit;
   ka.barrier = sh->barrier;
   ka.barrier_base = sh->barrier_base;
   ka.phase_clock = sh->phase_clock;
@@ -776,6 +815,108 @@ int shard_step(shard_t sh, kvstate_t st, const uint16_t* hidden_in, const int32_
   } else {
     for (int b = 0; b < B; ++b) st->len_host[b] += n_new[b];
   }
+  return SHARD_OK;
+}
+
+// Prefill chunk: tokens per pass through the layers (buffers scale with it).
+constexpr int kPrefillChunk = 256;
+
+int shard_prefill(shard_t sh, kvstate_t st, int row, const uint16_t* hidden_in, const int32_t* token_ids, int S,
+                  const int32_t* position_ids, const uint8_t* attention_mask, int mask_len, uint16_t* hidden_out,
+                  void* cuda_stream) {
+  if (!sh || !st || st->sh != sh) return fail(SHARD_EINVAL, "shard_prefill: shard/state mismatch");
+  if (!position_ids || !attention_mask || !hidden_out) return fail(SHARD_EINVAL, "shard_prefill: null argument");
+  if ((hidden_in == nullptr) == (token_ids == nullptr))
+    return fail(SHARD_EINVAL, "shard_prefill: pass exactly one of hidden_in and token_ids");
+  if (token_ids && sh->cfg.vocab <= 0) return fail(SHARD_EUNSUPPORTED, "shard_prefill: this shard has no embedding");
+  if (row < 0 || row >= st->n_rows || S < 1) return fail(SHARD_EINVAL, "shard_prefill: row or S out of range");
+  if (st->poisoned) return fail(SHARD_EINVAL, "shard_prefill: the KV state was left inconsistent; reset it");
+  if (st->shared) return fail(SHARD_EUNSUPPORTED, "shard_prefill: rows share entries after a beam gather; reset first");
+  int rc = check_pending_status(sh);
+  if (rc) return rc;
+  const int P = st->len_host[row];
+  if (st->cursor[row] != P) return fail(SHARD_EINVAL, "shard_prefill: row %d is not contiguous", row);
+  if (P + S > st->cap) return fail(SHARD_ECAPACITY, "shard_prefill: %d + %d entries > capacity %d", P, S, st->cap);
+  if (mask_len < P + S) return fail(SHARD_EINVAL, "shard_prefill: mask_len %d < %d", mask_len, P + S);
+  CUDA_TRY(cudaSetDevice(sh->device));
+  cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+  const int C = kPrefillChunk;
+  const int y_rows = std::max(std::max(sh->dq + 2 * sh->dkv, 2 * sh->F), sh->H);
+  if (!sh->pf_x) {
+    CUDA_TRY(cudaMalloc(&sh->pf_x, sizeof(float) * C * sh->H));
+    CUDA_TRY(cudaMalloc(&sh->pf_act, sizeof(uint16_t) * C * sh->Kp_H));
+    CUDA_TRY(cudaMalloc(&sh->pf_attn, sizeof(uint16_t) * C * sh->Kp_dq));
+    CUDA_TRY(cudaMalloc(&sh->pf_h, sizeof(uint16_t) * C * sh->Kp_F));
+    CUDA_TRY(cudaMalloc(&sh->pf_y, sizeof(float) * C * y_rows));
+    CUDA_TRY(cudaMalloc(&sh->pf_q, sizeof(float) * C * sh->dq));
+    CUDA_TRY(cudaMemset(sh->pf_act, 0, sizeof(uint16_t) * C * sh->Kp_H));
+    CUDA_TRY(cudaMemset(sh->pf_attn, 0, sizeof(uint16_t) * C * sh->Kp_dq));
+    CUDA_TRY(cudaMemset(sh->pf_h, 0, sizeof(uint16_t) * C * sh->Kp_F));
+  }
+  CUDA_TRY(launch_prefill_check(token_ids, sh->cfg.vocab, position_ids, sh->cfg.max_position, attention_mask, P, S,
+                                sh->status, s));
+  const int* bt_row = st->bt[st->bt_cur] + (size_t)row * st->cap;
+  const float eps = static_cast<float>(sh->cfg.rms_eps);
+  for (int t0 = 0; t0 < S; t0 += C) {
+    const int c = std::min(C, S - t0);
+    CUDA_TRY(launch_prefill_embed(hidden_in ? hidden_in + (size_t)t0 * sh->H : nullptr,
+                                  token_ids ? token_ids + t0 : nullptr, sh->embedding, sh->H, c, sh->cfg.vocab,
+                                  sh->pf_x, s));
+    for (int l = 0; l < sh->L; ++l) {
+      const uint16_t* nrm = sh->norms + (size_t)l * 2 * sh->H;
+      auto gemm = [&](int k, const uint16_t* act, int act_ld) -> cudaError_t {
+        const PackedOp& p = sh->ops[(size_t)l * N_OPS + k];
+        GemmArgs g{};
+        g.units = p.units;
+        g.n_rb = p.n_rb;
+        g.upr = p.upr;
+        g.act = act;
+        g.act_ld = act_ld;
+        g.S = c;
+        g.y = sh->pf_y;
+        g.y_ld = k == OP_QKV ? sh->dq + 2 * sh->dkv : k == OP_GU ? 2 * sh->F : sh->H;
+        g.dims = p.dims;
+        g.status = sh->status;
+        return launch_gemm_tc(g, sh->cfg.group, s);
+      };
+      CUDA_TRY(launch_prefill_norm(sh->pf_x, sh->H, nrm, eps, sh->pf_act, sh->Kp_H, c, s));
+      CUDA_TRY(gemm(OP_QKV, sh->pf_act, sh->Kp_H));
+      PrefillLayerArgs pa{};
+      pa.y = sh->pf_y;
+      pa.y_ld = sh->dq + 2 * sh->dkv;
+      pa.S = c;
+      pa.Hq = sh->Hq;
+      pa.Hkv = sh->Hkv;
+      pa.d = sh->d;
+      pa.pos = position_ids + t0;
+      pa.max_position = sh->cfg.max_position;
+      pa.rope = sh->rope;
+      pa.q = sh->pf_q;
+      pa.kpool = st->k + (size_t)l * st->layer_stride;
+      pa.vpool = st->v + (size_t)l * st->layer_stride;
+      pa.row = row;
+      pa.cap = st->cap;
+      pa.slot0 = P + t0;
+      pa.bt_row = bt_row;
+      pa.mask = attention_mask;
+      pa.P = P + t0;
+      pa.attn = sh->pf_attn;
+      pa.attn_ld = sh->Kp_dq;
+      CUDA_TRY(launch_prefill_rope_append(pa, s));
+      CUDA_TRY(launch_prefill_attention(pa, s));
+      CUDA_TRY(gemm(OP_O, sh->pf_attn, sh->Kp_dq));
+      CUDA_TRY(launch_prefill_residual(sh->pf_x, sh->pf_y, sh->H, c, sh->H, nullptr, s));
+      CUDA_TRY(launch_prefill_norm(sh->pf_x, sh->H, nrm + sh->H, eps, sh->pf_act, sh->Kp_H, c, s));
+      CUDA_TRY(gemm(OP_GU, sh->pf_act, sh->Kp_H));
+      CUDA_TRY(launch_prefill_swiglu(sh->pf_y, 2 * sh->F, c, sh->F, sh->pf_h, sh->Kp_F, s));
+      CUDA_TRY(gemm(OP_DOWN, sh->pf_h, sh->Kp_F));
+      CUDA_TRY(launch_prefill_residual(sh->pf_x, sh->pf_y, sh->H, c, sh->H,
+                                       l + 1 == sh->L ? hidden_out + (size_t)t0 * sh->H : nullptr, s));
+    }
+  }
+  CUDA_TRY(launch_set_int(st->lens + row, P + S, s));
+  st->cursor[row] += S;
+  st->len_host[row] += S;
   return SHARD_OK;
 }
 
@@ -847,6 +988,7 @@ int shard_sync_status(shard_t sh, void* cuda_stream) {
   CUDA_TRY(cudaMemcpy(&bits, sh->status, sizeof(int), cudaMemcpyDeviceToHost));
   CUDA_TRY(cudaMemset(sh->status, 0, sizeof(int)));
   *reinterpret_cast<volatile int*>(sh->status_host) = 0;
+  if (bits & ST_WAIT_TIMEOUT) CUDA_TRY(reset_work_buffers(sh));
   if (bits) {
     for (auto* st : sh->states) st->poisoned = true;
     return fail(SHARD_EINVAL, "device guard: %s", status_message(bits).c_str());
@@ -897,17 +1039,49 @@ int shard_debug_gemv(shard_t sh, int layer, int op, const uint16_t* x, int M, fl
   g.act = act;
   g.act_ld = ld;
   g.M = M;
-  g.sp = nullptr;
-  g.partials = sh->partials;
-  g.flags = sh->flags;
-  g.epoch = next_epochs(sh, 1);
   g.status = sh->status;
   g.ep.kind = EPI_STORE;
   g.ep.dims = p.dims;
+  g.ep.acc = sh->acc_store;
+  g.ep.acc_ld = p.n_rb * kRowsPerBlock;
+  g.ep.cnt = sh->cnt_store;
   g.ep.y = y;
   g.ep.y_ld = y_ld;
   const int nt = nt_for(M);
   CUDA_TRY(launch_gemv(g, nt, sh->cfg.group, std::min<long long>(sh->grid[nt], (long long)p.n_rb * p.upr), s, false));
+  return SHARD_OK;
+}
+
+int shard_debug_gemm(shard_t sh, int layer, int op, const uint16_t* x, int x_ld, int S, float* y, int y_ld,
+                     void* cuda_stream) {
+  if (!sh || !x || !y || layer < 0 || layer >= sh->L || op < 0 || op >= N_OPS || S < 1)
+    return fail(SHARD_EINVAL, "shard_debug_gemm: bad argument");
+  const PackedOp& p = sh->ops[(size_t)layer * N_OPS + op];
+  const int nat[N_OPS] = {sh->dq + 2 * sh->dkv, sh->H, 2 * sh->F, sh->H};
+  if (y_ld < nat[op]) return fail(SHARD_EINVAL, "shard_debug_gemm: y_ld %d < rows %d", y_ld, nat[op]);
+  if (x_ld < p.Kp || x_ld % kUnitK || reinterpret_cast<uintptr_t>(x) % 16)
+    return fail(SHARD_EINVAL, "shard_debug_gemm: x_ld %d must be a multiple of 128 and >= %d; x 16-byte aligned", x_ld,
+                p.Kp);
+  CUDA_TRY(cudaSetDevice(sh->device));
+  GemmArgs g{};
+  g.units = p.units;
+  g.n_rb = p.n_rb;
+  g.upr = p.upr;
+  g.act = x;
+  g.act_ld = x_ld;
+  g.S = S;
+  g.y = y;
+  g.y_ld = y_ld;
+  g.dims = p.dims;
+  g.status = sh->status;
+  CUDA_TRY(launch_gemm_tc(g, sh->cfg.group, static_cast<cudaStream_t>(cuda_stream)));
+  return SHARD_OK;
+}
+
+int shard_debug_set_wait(shard_t sh, unsigned limit, int skip_arrival) {
+  if (!sh || limit < 1) return fail(SHARD_EINVAL, "shard_debug_set_wait: bad argument");
+  sh->wait_limit = limit;
+  sh->debug_skip_arrival = skip_arrival;
   return SHARD_OK;
 }
 
@@ -932,6 +1106,7 @@ namespace shard {
 struct NoAllocView {
   const PackedOp* op;
   int group, grid_nt1, grid_nt2, device, rows;
+  int* status;  // the shard's device status word (shard_sync_status reports it)
 };
 
 int shard_noalloc_fail(int code, const char* msg) { return fail(code, "%s", msg); }
@@ -948,6 +1123,7 @@ int shard_noalloc_view(shard_t sh, int layer, int op, NoAllocView* v) {
   v->device = sh->device;
   const int nat[N_OPS] = {sh->dq + 2 * sh->dkv, sh->H, 2 * sh->F, sh->H};
   v->rows = nat[op];
+  v->status = sh->status;
   return SHARD_OK;
 }
 

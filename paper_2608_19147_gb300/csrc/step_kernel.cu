@@ -1,26 +1,26 @@
 // The whole decode step of a shard as one persistent, cooperative kernel.
 //
-// One CTA per SM, kCtaWarps warps.  The step runs as a sequence of phases separated
-// by grid-wide barriers ('|'):
-//   prologue (CTA 0) | for each layer: RMSNorm + q|k|v projection (+RoPE,
-//   K/V append) -> attention (chunk partials and merges) | o projection
-//   (+residual) | RMSNorm + gate|up projection (+SwiGLU) | down projection
-//   (+residual; the last layer writes hidden_out).
-// '->' is dataflow instead of a barrier: each q|k|v row-block's finisher
-// release-stores the launch's epoch of that projection into the row-block's
-// flag, and an attention item waits (acquire loads, bounded) only for the
-// row-blocks of its kv head.  Flags are never cleared: an epoch is unique per
-// launch and op.
-// Each RMSNorm is computed by every CTA at the start of the projection that
-// consumes it, from per-row-block sums of squares left by the residual's
-// producer, so it needs no barrier of its own.
-// Every warp owns a ring of weight slots (gemv_core.cuh) that streams, in
-// order, all the projection units the warp will process during the step.
-// The ring refills as soon as a slot is consumed, independent of the
-// barriers, so while a warp waits at a barrier or works on norms and
-// attention, the next projection's weights are already arriving.
+// One CTA per SM: kCtaWarps consumer warps and one producer warp that streams
+// the weights into the consumers' rings (gemv_core.cuh).  The step runs as a
+// sequence of phases separated by grid-wide barriers ('|'):
+//   prologue (every CTA: its share of the beam-table gather, the new
+//   entries' slots and the residual) ~ for each layer: RMSNorm + q|k|v
+//   projection -> attention (chunk partials and merges, with RoPE and the K/V
+//   append) | o projection (+residual) | RMSNorm + gate|up projection
+//   (+SwiGLU) | down projection (+residual) | ... ; then hidden_out.
+// '~' is a split barrier: CTAs arrive after their prologue share and wait only
+// before the first attention, so the first norm and q|k|v projection overlap
+// the prologue.  '->' is dataflow: q|k|v contributors count finished units
+// per kv head (release) and an attention item waits (acquire, bounded) only
+// for its kv head's count.
 //
-// Barrier waits are bounded: a wait that runs out sets a status bit and
+// The residual stream and the projections' sums are 64-bit fixed point
+// (kernels.h): contributors add with integer atomics and nobody waits for a
+// merge; results do not depend on the order of arrival.
+// Each RMSNorm is computed by every CTA at the start of the projection that
+// consumes it, from the whole residual (the same bits in every CTA).
+//
+// Every cross-CTA wait is bounded: a wait that runs out sets a status bit and
 // proceeds (the step's results are then reported invalid) instead of hanging.
 #include <type_traits>
 
@@ -29,21 +29,29 @@
 namespace shard {
 namespace {
 
-constexpr int kWarps = kCtaWarps;
-constexpr int kThreads = kWarps * 32;
+constexpr int kWarps = kCtaWarps;           // consumer warps
+constexpr int kThreads = kWarps * 32;       // consumer threads
+constexpr int kBlockThreads = kThreads + 32;  // + the producer warp
 constexpr int kChunk = kAttnChunk;  // most cache entries per attention item (four per lane)
 constexpr bool kNormInSmem = true;   // normalised activations in shared memory when they fit
-constexpr bool kNormPrefetch = true; // RMSNorm: first x loads issued with the sums-of-squares loads
+constexpr int kNormCache = 6;        // float4 pieces of the first row a thread keeps between the norm's passes
+// Polls of a busy slot before the producer gives up: a slot may legitimately
+// stay busy while its consumer works through a whole attention phase, so this
+// bound is fixed and far above any step's length.
+constexpr uint32_t kProducerLimit = 1u << 22;
 
 template <int GPU>
 struct StepSmem {
   static constexpr size_t kRing = (size_t)kWarps * kRingSlots * Geom<GPU>::kUnitBytes;
-  static constexpr size_t kBars = (size_t)kWarps * kRingSlots * sizeof(uint64_t);
-  // attention item area (AttnSmem)
+  static constexpr size_t kBars = (size_t)2 * kWarps * kRingSlots * sizeof(uint64_t);
+  // attention item area (AttnSmem), also the normalised rows
   static constexpr size_t kQ = 96 * 1024;
   static constexpr size_t kFixed = kRing + kBars + kQ;  // + the op table (4L entries)
   static size_t total(int n_layers) { return kFixed + (size_t)4 * n_layers * sizeof(OpDesc); }
 };
+
+// Barrier among the consumer warps of a CTA (the producer warp runs on its own).
+__device__ __forceinline__ void cbar() { named_bar_sync(1, kThreads); }
 
 __device__ __forceinline__ unsigned long long ld_acquire_u64(const unsigned long long* p) {
   unsigned long long v;
@@ -51,8 +59,6 @@ __device__ __forceinline__ unsigned long long ld_acquire_u64(const unsigned long
   return v;
 }
 
-// Grid-wide barrier on a monotonically increasing counter.  `target` is this
-// CTA's running count of expected arrivals.
 __device__ __forceinline__ unsigned long long globaltimer() {
   unsigned long long t;
   asm volatile("mov.u64 %0, %globaltimer;" : "=l"(t));
@@ -70,63 +76,90 @@ __device__ __forceinline__ uint32_t pack_h2(float lo, float hi) {
   return (uint32_t)f2h(lo) | ((uint32_t)f2h(hi) << 16);
 }
 
-__device__ __forceinline__ void red_release_add_s32(int* p, int v) {
-  asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
-}
-__device__ __forceinline__ int ld_acquire_s32(const int* p) {
-  int v;
-  asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-  return v;
-}
-
 __device__ __forceinline__ void red_release_add(unsigned long long* p, unsigned long long v) {
   asm volatile("red.release.gpu.global.add.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
 }
 
-__device__ void grid_sync(unsigned long long* ctr, unsigned long long& target, int* status,
-                          unsigned long long* clock, int& nsync) {
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    target += gridDim.x;
-    red_release_add(ctr, 1ULL);
-    // bounded: after ~2^22 polls, or once any CTA has given up, stop waiting
-    uint32_t it = 0;
-    while (ld_acquire_u64(ctr) < target) {
-      if (++it > (1u << 22)) {
-        atomicOr(status, ST_WAIT_TIMEOUT);
-        break;
-      }
-      if ((it & 1023) == 0 && (*reinterpret_cast<volatile int*>(status) & ST_WAIT_TIMEOUT)) break;
-      __nanosleep(64);
+// Grid-wide barrier on a monotonically increasing counter, in two halves so
+// that work may sit between arriving and waiting.  `target` is this CTA's
+// running count of expected arrivals.  Called by the consumer warps; the
+// caller has synchronised them (cbar) before grid_arrive.
+struct GridBarrier {
+  unsigned long long* ctr;
+  unsigned long long target;
+  int* status;
+  unsigned long long* clock;
+  int n_arrive, n_wait;
+  int skip_arrival;  // test knob: CTA 1 leaves out this arrival (-1: none)
+  uint32_t limit;
+
+  __device__ __forceinline__ void arrive() {
+    if (threadIdx.x == 0) {
+      if (!(blockIdx.x == 1 && n_arrive == skip_arrival)) red_release_add(ctr, 1ULL);
     }
-    if (blockIdx.x == 0) clock[nsync] = globaltimer();
+    ++n_arrive;
   }
-  ++nsync;
-  __syncthreads();
+  __device__ __forceinline__ void wait() {
+    if (threadIdx.x == 0) {
+      target += gridDim.x;
+      // bounded: after `limit` polls, or once any CTA has given up, stop waiting
+      uint32_t it = 0;
+      while (ld_acquire_u64(ctr) < target) {
+        if (++it > limit) {
+          atomicOr(status, ST_WAIT_TIMEOUT);
+          break;
+        }
+        if ((it & 1023) == 0 && (*reinterpret_cast<volatile int*>(status) & ST_WAIT_TIMEOUT)) break;
+        __nanosleep(64);
+      }
+      if (blockIdx.x == 0) clock[n_wait + 1] = globaltimer();
+    }
+    ++n_wait;
+    cbar();
+  }
+  __device__ __forceinline__ void sync() {
+    cbar();
+    arrive();
+    wait();
+  }
+};
+
+__device__ __forceinline__ bool wait_count(const int* p, int target, int* status, uint32_t limit) {
+  uint32_t it = 0;
+  while (ld_acquire_s32(p) < target) {
+    if (++it > limit) {
+      atomicOr(status, ST_WAIT_TIMEOUT);
+      return false;
+    }
+    if ((it & 1023) == 0 && (*reinterpret_cast<volatile int*>(status) & ST_WAIT_TIMEOUT)) return false;
+    __nanosleep(64);
+  }
+  return true;
 }
 
 // ---------------------------------------------------------------------------
-// Prologue (CTA 0): the beam_idx gather of the entry tables (Section 4: row b
-// continues row beam_idx[b]'s entries; K/V stay where they are), the new
-// entries' slots, device-side argument checks, and the residual stream.
+// Prologue, part 1 (every CTA, all threads): the step's bookkeeping from its
+// arguments -- Section 4's beam_idx gather (row b continues row beam_idx[b]'s
+// entries; K/V stay where they are), the new entries' slots -- and the
+// device-side argument checks.  Every CTA derives the same values.
 // ---------------------------------------------------------------------------
-__device__ __noinline__ void prologue_cta(const PrologueArgs& a) {
-  __shared__ int s_src[kMaxRequests], s_P[kMaxRequests], s_len[kMaxRequests], s_tok0[kMaxRequests + 1];
-  __shared__ int s_req[kMaxTokens], s_idx[kMaxTokens];
+__device__ __noinline__ void prologue_params(const PrologueArgs& a, StepParams* sp, const uint16_t** rowp) {
   __shared__ int s_err;
-  const int tid = threadIdx.x, nth = blockDim.x;
+  const int tid = threadIdx.x;
   if (tid == 0) {
     // a step rejected earlier freezes the state until the host resets it
     s_err = __ldcg(a.status) != 0 ? ST_STICKY : 0;
     int t = 0;
     for (int b = 0; b < a.B; ++b) {
-      s_tok0[b] = t;
+      sp->req_tok0[b] = t;
       for (int i = 0; i < a.n_new[b]; ++i, ++t) {
-        s_req[t] = b;
-        s_idx[t] = i;
+        sp->tok_req[t] = b;
+        sp->tok_idx[t] = i;
       }
     }
-    s_tok0[a.B] = t;
+    sp->req_tok0[a.B] = t;
+    sp->M = a.M;
+    sp->B = a.B;
   }
   __syncthreads();
   if (tid < a.B) {
@@ -135,153 +168,149 @@ __device__ __noinline__ void prologue_cta(const PrologueArgs& a) {
       atomicOr(&s_err, ST_BEAM_IDX);
       src = tid;
     }
-    s_src[tid] = src;
-    s_P[tid] = __ldcg(a.lens + src);
-  }
-  __syncthreads();
-  if (tid < a.B) {
-    const int L = s_P[tid] + a.n_new[tid];
+    sp->req_src[tid] = src;
+    const int P = __ldcg(a.lens + src);
+    const int L = P + a.n_new[tid];
     if (L > a.cap || a.cursor[tid] + a.n_new[tid] > a.cap) atomicOr(&s_err, ST_CAPACITY);
     if (L > a.mask_stride) atomicOr(&s_err, ST_MASK_STRIDE);
-    s_len[tid] = L;
+    sp->req_P[tid] = P;
+    sp->req_len[tid] = L;
   }
   __syncthreads();
-  for (int m = tid; m < a.M; m += nth) {
-    const int b = s_req[m], j = s_P[b] + s_idx[m];
-    if (j < a.mask_stride && __ldcg(a.mask + (size_t)b * a.mask_stride + j) == 0) atomicOr(&s_err, ST_MASK_NEW);
+  if (tid < a.M) {
+    const int m = tid, b = sp->tok_req[m], i = sp->tok_idx[m], j = sp->req_P[b] + i;
+    // a token must see its own entry (packed: in its own mask row, Section 8.6)
+    const size_t mrow = a.packed ? (size_t)m : (size_t)b;
+    if (j < a.mask_stride && __ldcg(a.mask + mrow * a.mask_stride + j) == 0) atomicOr(&s_err, ST_MASK_NEW);
     const int pos = __ldcg(a.position_ids + m);
     if (pos < 0 || pos >= a.max_position) atomicOr(&s_err, ST_POSITION);
+    sp->tok_pos[m] = pos;
+    sp->tok_slot[m] = b * a.cap + a.cursor[b] + i;
     if (a.token_ids) {
       const int tok = __ldcg(a.token_ids + m);
       if (tok < 0 || tok >= a.vocab) atomicOr(&s_err, ST_TOKEN);
+      rowp[m] = a.embedding + (size_t)(tok < 0 || tok >= a.vocab ? 0 : tok) * a.H;
+    } else {
+      rowp[m] = a.hidden_in + (size_t)m * a.H;
     }
   }
   __syncthreads();
-  if (s_err) {
-    if (tid == 0) {
-      atomicOr(a.status, s_err & ~ST_STICKY);
-      a.sp->abort_step = 1;
-    }
-    return;
-  }
+  if (tid == 0) sp->abort_step = s_err;
+  __syncthreads();
+}
+
+// Prologue, part 2 (consumer threads of every CTA, a share each): the beam
+// table's gather and appends, and the residual stream X = the fp16 inputs in
+// fixed point (exact).
+__device__ __noinline__ void prologue_work(const PrologueArgs& a, const StepParams* sp, const uint16_t* const* rowp,
+                                           long long* X) {
+  const int tid = threadIdx.x;
+  const int gt = blockIdx.x * kThreads + tid, gs = gridDim.x * kThreads;
   if (a.beam_idx) {
     for (int b = 0; b < a.B; ++b) {
-      const int* src = a.bt_src + (size_t)s_src[b] * a.cap;
+      const int* src = a.bt_src + (size_t)sp->req_src[b] * a.cap;
       int* dst = a.bt_dst + (size_t)b * a.cap;
-      for (int j = tid; j < s_P[b]; j += nth) dst[j] = __ldcg(src + j);
+      for (int j = gt; j < sp->req_P[b]; j += gs) dst[j] = __ldcg(src + j);
     }
   }
-  for (int m = tid; m < a.M; m += nth) {
-    const int b = s_req[m], i = s_idx[m];
-    a.bt_dst[(size_t)b * a.cap + s_P[b] + i] = b * a.cap + a.cursor[b] + i;
+  if (blockIdx.x == 0 && tid < a.M) {
+    const int b = sp->tok_req[tid], i = sp->tok_idx[tid];
+    a.bt_dst[(size_t)b * a.cap + sp->req_P[b] + i] = sp->tok_slot[tid];
   }
-  if (tid < a.B) a.lens[tid] = s_len[tid];
-  // residual x: warp per (token, 64-row block), which also leaves the
-  // block's sum of squares for the first RMSNorm
-  {
-    const int n_rb = (a.H + kRowsPerBlock - 1) / kRowsPerBlock;
-    const int lane = tid & 31;
-    for (int it = tid >> 5; it < a.M * n_rb; it += nth >> 5) {
-      const int m = it / n_rb, rb = it % n_rb;
-      const uint16_t* src = a.hidden_in ? a.hidden_in + (size_t)m * a.H
-                                        : a.embedding + (size_t)__ldcg(a.token_ids + m) * a.H;
-      float ss = 0.f;
-#pragma unroll
-      for (int r = 0; r < kRowsPerBlock; r += 32) {
-        const int k = rb * kRowsPerBlock + r + lane;
-        if (k < a.H) {
-          const float v = h2f(a.hidden_in ? __ldcg(src + k) : src[k]);
-          a.x[(size_t)m * a.H + k] = v;
-          ss = fmaf(v, v, ss);
-        }
-      }
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
-      if (lane == 0) a.ss[rb * kMaxTokens + m] = ss;
-    }
-  }
-  if (tid == 0) {
-    StepParams* sp = a.sp;
-    sp->M = a.M;
-    sp->B = a.B;
-    sp->abort_step = 0;
-    for (int m = 0; m < a.M; ++m) {
-      const int b = s_req[m];
-      sp->tok_req[m] = b;
-      sp->tok_idx[m] = s_idx[m];
-      sp->tok_pos[m] = __ldcg(a.position_ids + m);
-      sp->tok_slot[m] = b * a.cap + a.cursor[b] + s_idx[m];
-    }
-    for (int b = 0; b <= a.B; ++b) sp->req_tok0[b] = s_tok0[b];
-    for (int b = 0; b < a.B; ++b) {
-      sp->req_P[b] = s_P[b];
-      sp->req_len[b] = s_len[b];
-    }
-    sp->mask = a.mask;
-    sp->mask_stride = a.mask_stride;
-    sp->hidden_out = a.hidden_out;
-    sp->bt = a.bt_dst;
+  const int H4 = a.H / 4;
+  for (int e = gt; e < a.M * H4; e += gs) {
+    const int m = e / H4, k = 4 * (e % H4);
+    const uint2 v = *reinterpret_cast<const uint2*>(rowp[m] + k);
+    const float2 f01 = h2f2(v.x), f23 = h2f2(v.y);
+    longlong2* dst = reinterpret_cast<longlong2*>(X + (size_t)m * a.H + k);
+    dst[0] = make_longlong2(__float2ll_rn(f01.x * kFixOne), __float2ll_rn(f01.y * kFixOne));
+    dst[1] = make_longlong2(__float2ll_rn(f23.x * kFixOne), __float2ll_rn(f23.y * kFixOne));
   }
 }
 
 // ---------------------------------------------------------------------------
-// RMSNorm, run by every CTA at the start of the projection that consumes it.
-// r[m] = 1 / sqrt(mean(x[m]^2) + eps) from the per-row-block sums of squares
-// that the residual's producer left (added in a fixed order, so every CTA
-// gets the same r); then act = fp16(x * r * w).  Every CTA writes the whole
-// act -- the same bits -- so its own warps can start as soon as it is done.
-// H is a multiple of 4.
+// RMSNorm, run by every CTA at the start of the projection that consumes it:
+// r[m] = 1 / sqrt(mean(x[m]^2) + eps), act = fp16(x * r * w).  x is the
+// residual stream (fixed point) or, before the first layer, the step's fp16
+// input rows (the same values).  Two passes: the sums of squares (added in a
+// fixed order, so every CTA gets the same r), then the scaled rows; the first
+// row's pieces stay in registers between the passes.  H is a multiple of 4.
 // ---------------------------------------------------------------------------
-__device__ __noinline__ void rmsnorm_cta(const float* x, int H, const uint16_t* w, float eps, const float* ss,
-                                         uint16_t* out, int out_ld, int M) {
+template <bool kFromX>
+__device__ __forceinline__ float4 norm_load(const long long* X, const uint16_t* const* rowp, int H, int m, int k) {
+  if (kFromX) {
+    const longlong2* p = reinterpret_cast<const longlong2*>(X + (size_t)m * H + k);
+    const longlong2 a = __ldcg(p), b = __ldcg(p + 1);
+    return make_float4(fixed_to_f32(a.x), fixed_to_f32(a.y), fixed_to_f32(b.x), fixed_to_f32(b.y));
+  } else {
+    const uint2 v = *reinterpret_cast<const uint2*>(rowp[m] + k);
+    const float2 f01 = h2f2(v.x), f23 = h2f2(v.y);
+    return make_float4(f01.x, f01.y, f23.x, f23.y);
+  }
+}
+
+template <bool kFromX>
+__device__ __noinline__ void rmsnorm_cta(const long long* X, const uint16_t* const* rowp, int H, const uint16_t* w,
+                                         float eps, uint16_t* out, int out_ld, int M) {
+  __shared__ float s_part[kWarps][kMaxTokens];
   __shared__ float s_r[kMaxTokens];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int n_rb = (H + kRowsPerBlock - 1) / kRowsPerBlock;
-  constexpr int kBatch = 4;  // float4 pieces per thread in flight
-  const int H4 = H / 4, n4 = M * H4;
-  float4 xv[kBatch];
-  uint2 wv[kBatch];
-  auto load = [&](int i0) {
-#pragma unroll
-    for (int j = 0; j < kBatch; ++j) {
-      const int i = i0 + j * kThreads;
-      if (i < n4) {
-        xv[j] = __ldcg(reinterpret_cast<const float4*>(x) + i);
-        wv[j] = *reinterpret_cast<const uint2*>(w + 4 * (i % H4));
-      }
-    }
-  };
-  auto store = [&](int i0) {
-#pragma unroll
-    for (int j = 0; j < kBatch; ++j) {
-      const int i = i0 + j * kThreads;
-      if (i < n4) {
-        const int m = i / H4, k = 4 * (i % H4);
-        const float r = s_r[m];
-        const float2 w01 = h2f2(wv[j].x), w23 = h2f2(wv[j].y);
-        uint2 o;
-        o.x = pack_h2(xv[j].x * r * w01.x, xv[j].y * r * w01.y);
-        o.y = pack_h2(xv[j].z * r * w23.x, xv[j].w * r * w23.y);
-        *reinterpret_cast<uint2*>(out + (size_t)m * out_ld + k) = o;
-      }
-    }
-  };
-  // the first batch of x and weights is in flight with the sums of squares
-  if (kNormPrefetch) load(tid);
-  for (int m = warp; m < M; m += kWarps) {
+  const int H4 = H / 4;
+  float4 keep[kNormCache];
+  for (int m = 0; m < M; ++m) {
     float t = 0.f;
-    for (int rb = lane; rb < n_rb; rb += 32) t += __ldcg(ss + rb * kMaxTokens + m);
+    if (m == 0) {
+#pragma unroll
+      for (int i = 0; i < kNormCache; ++i) {
+        const int c = tid + i * kThreads;
+        keep[i] = c < H4 ? norm_load<kFromX>(X, rowp, H, 0, 4 * c) : make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+#pragma unroll
+      for (int i = 0; i < kNormCache; ++i)
+        t += keep[i].x * keep[i].x + keep[i].y * keep[i].y + keep[i].z * keep[i].z + keep[i].w * keep[i].w;
+      for (int c = tid + kNormCache * kThreads; c < H4; c += kThreads) {
+        const float4 v = norm_load<kFromX>(X, rowp, H, 0, 4 * c);
+        t += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+      }
+    } else {
+      for (int c = tid; c < H4; c += kThreads) {
+        const float4 v = norm_load<kFromX>(X, rowp, H, m, 4 * c);
+        t += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+      }
+    }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
-    if (lane == 0) s_r[m] = rsqrtf(t / H + eps);
+    if (lane == 0) s_part[warp][m] = t;
   }
-  __syncthreads();
-  if (kNormPrefetch) store(tid);
-  for (int i0 = tid + (kNormPrefetch ? kBatch * kThreads : 0); i0 < n4; i0 += kBatch * kThreads) {
-    load(i0);
-    store(i0);
+  cbar();
+  if (tid < M) {
+    float t = 0.f;
+    for (int w8 = 0; w8 < kWarps; ++w8) t += s_part[w8][tid];
+    s_r[tid] = rsqrtf(t / H + eps);
   }
-  __syncthreads();
+  cbar();
+  for (int m = 0; m < M; ++m) {
+    const float r = s_r[m];
+    auto emit = [&](int c, float4 v) {
+      const uint2 wv = *reinterpret_cast<const uint2*>(w + 4 * c);
+      const float2 w01 = h2f2(wv.x), w23 = h2f2(wv.y);
+      uint2 o;
+      o.x = pack_h2(v.x * r * w01.x, v.y * r * w01.y);
+      o.y = pack_h2(v.z * r * w23.x, v.w * r * w23.y);
+      *reinterpret_cast<uint2*>(out + (size_t)m * out_ld + 4 * c) = o;
+    };
+    if (m == 0) {
+#pragma unroll
+      for (int i = 0; i < kNormCache; ++i) {
+        const int c = tid + i * kThreads;
+        if (c < H4) emit(c, keep[i]);
+      }
+      for (int c = tid + kNormCache * kThreads; c < H4; c += kThreads) emit(c, norm_load<kFromX>(X, rowp, H, 0, 4 * c));
+    } else {
+      for (int c = tid; c < H4; c += kThreads) emit(c, norm_load<kFromX>(X, rowp, H, m, 4 * c));
+    }
+  }
+  cbar();
 }
 
 // ---------------------------------------------------------------------------
@@ -301,17 +330,24 @@ __device__ __noinline__ void rmsnorm_cta(const float* x, int H, const uint16_t* 
 __host__ __device__ constexpr int part_stride(int d) { return d + 4; }
 
 struct AttnView {
-  const float* q;
-  const uint16_t* kpool;  // layer 0; layer l at + l * layer_stride
-  const uint16_t* vpool;
+  const long long* acc;     // q|k|v sums [16][acc_ld] (fixed point), GPU row order
+  int acc_ld;
+  const float2* rope;       // [max_position][d/2]
+  uint16_t* kpool;          // layer 0; layer l at + l * layer_stride
+  uint16_t* vpool;
   size_t layer_stride;
   int cap, Hq, Hkv, d, n_chunks, qmax;
   float* part;
-  int* cnt;  // finished chunks per (request, kv head)
-  const unsigned* rb_done;  // q|k|v row-block flags the items wait for
-  int rb_k0, rb_v0;         // first k and v row-block of the q|k|v projection
-  int cs;    // entries per item this step: 32, 64 or 128 (kChunk)
-  int last_merges;  // at most one item per CTA: the CTA finishing the last chunk merges at once
+  int* cnt;                 // finished chunks per (request, kv head)
+  const int* cnt_kv;        // q|k|v units finished per kv head
+  int kv_units;             // units per kv head when its q|k|v rows are complete
+  const int* bt;            // beam table (entry -> physical slot) of this step
+  const uint8_t* mask;
+  int mask_stride;
+  int packed;               // a mask row per token of request 0 instead of one per request
+  int cs;                   // entries per item this step: 32, 64 or 128 (kChunk)
+  int last_merges;          // at most one item per CTA: the CTA finishing the last chunk merges at once
+  uint32_t limit;
   uint16_t* out;
   int out_ld;
 };
@@ -403,8 +439,36 @@ struct AttnSmem {
   static constexpr size_t kV = (size_t)kChunk * d * 2;
   static constexpr size_t kQ = (size_t)kQg * d * 4;
   static constexpr size_t kP = (size_t)kQg * kChunk * 4;
-  static constexpr size_t kBytes = kK + kV + kQ + kP + 2 * kChunk * sizeof(int);
+  static constexpr size_t kVisT = (size_t)kMaxTokens * kChunk;  // packed mode: [token][entry] mask bytes
+  static constexpr size_t kBytes = kK + kV + kQ + kP + 2 * kChunk * sizeof(int) + kVisT;
 };
+
+// Row of the q|k|v projection holding dimension i (< d/2) of q head h, or of
+// k head h when `first` is the first k row; dimension i + d/2 is 8 rows
+// further (kernels.h: rotary pairs share a 16-row tile).
+__device__ __forceinline__ int rot_row(int first, int h, int i, int d) {
+  return first + 16 * (h * (d >> 4) + (i >> 3)) + (i & 7);
+}
+
+// Queries q0 .. q0 + qn of an item into shared memory: the fixed-point q sums
+// of the query's head and token, rotated by the token's position (RoPE,
+// pairs (i, i + d/2)), fp32.
+template <int DPL>
+__device__ __forceinline__ void attn_load_queries(const AttnView& a, const StepParams* sp, int hk, int tok0, int q0,
+                                                  int qn, float* qsm) {
+  constexpr int d = 32 * DPL, half = d / 2;
+  const int G = a.Hq / a.Hkv;
+  for (int e = threadIdx.x; e < qn * half; e += kThreads) {
+    const int qi = e / half, i = e % half, q = q0 + qi;
+    const int m = tok0 + q / G, h = hk * G + q % G;
+    const long long* row = a.acc + (size_t)m * a.acc_ld;
+    const int R = rot_row(0, h, i, d);
+    const float lo = fixed_to_f32(__ldcg(row + R)), hi = fixed_to_f32(__ldcg(row + R + 8));
+    const float2 cs = a.rope[(size_t)sp->tok_pos[m] * half + i];
+    qsm[qi * d + i] = lo * cs.x - hi * cs.y;
+    qsm[qi * d + half + i] = hi * cs.x + lo * cs.y;
+  }
+}
 
 // Merge of one (request, kv head, query): chunks in order, kMergeBatch at a
 // time with all their loads in flight; lane c of a batch holds chunk c's max
@@ -467,31 +531,35 @@ __device__ __noinline__ void attn_merge_warp(const AttnView* ap, const StepParam
   for (int u = 0; u < DPL; ++u) out[u] = f2h(num[u] / den);
 }
 
-// One item, processed by the whole CTA:
+// One item, processed by the CTA's consumer warps:
 //   1. the chunk's slots (beam table) and mask bits;
-//   2. its K and V rows -- those of earlier steps before waiting for this
-//      step's q|k|v row-blocks, the appended ones after -- and the first query
-//      group into shared memory, every load of a thread in flight at once;
-//   3. scores: warp w takes queries w, w + kWarps, ...; lane = entry; the
+//   2. the K and V rows of earlier steps, in flight while the item waits
+//      (bounded) for its kv head's q|k|v units;
+//   3. the rows this step appends, from the fixed-point k and v sums (k
+//      rotated by its token's position, both rounded to fp16) -- written to
+//      the shared tile and, by the one item whose chunk holds them, to the
+//      KV pool -- and the first query group;
+//   4. scores: warp w takes queries w, w + kWarps, ...; lane = entry; the
 //      softmax pieces (max, sum of exp) per query across the lanes;
-//   4. values: thread = (query, pair of head dims), sum over the entries;
-//   5. a release count of the finished chunk for its (request, kv head); when
+//   5. values: thread = (query, pair of head dims), sum over the entries;
+//   6. a release count of the finished chunk for its (request, kv head); when
 //      every CTA has at most one item, the CTA that counts the last chunk
 //      merges at once.
 template <int DPL>
 __device__ __noinline__ void attn_item_cta(const AttnView* ap, int layer, const StepParams* sp, int b, int hk, int c,
-                                           uint8_t* area, unsigned qkv_epoch, int* status) {
+                                           uint8_t* area, int* status) {
   const AttnView& a = *ap;
-  const uint16_t* kpool = a.kpool + (size_t)layer * a.layer_stride;
-  const uint16_t* vpool = a.vpool + (size_t)layer * a.layer_stride;
+  uint16_t* kpool = a.kpool + (size_t)layer * a.layer_stride;
+  uint16_t* vpool = a.vpool + (size_t)layer * a.layer_stride;
   using S = AttnSmem<DPL>;
-  constexpr int d = S::d, KP = d / 8;  // 16-byte pieces per row
+  constexpr int d = S::d, KP = d / 8, half = d / 2;  // 16-byte pieces per row
   uint16_t* Ks = reinterpret_cast<uint16_t*>(area);
   uint16_t* Vs = reinterpret_cast<uint16_t*>(area + S::kK);
   float* qsm = reinterpret_cast<float*>(area + S::kK + S::kV);
   float* ps = reinterpret_cast<float*>(area + S::kK + S::kV + S::kQ);
   int* slot_s = reinterpret_cast<int*>(area + S::kK + S::kV + S::kQ + S::kP);
   int* vis_s = slot_s + kChunk;
+  uint8_t* vis_t = reinterpret_cast<uint8_t*>(vis_s + kChunk);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int L = sp->req_len[b], P = sp->req_P[b];
   const int tok0 = sp->req_tok0[b], nb = sp->req_tok0[b + 1] - tok0;
@@ -499,95 +567,93 @@ __device__ __noinline__ void attn_item_cta(const AttnView* ap, int layer, const 
   const int j0 = c * a.cs, nj = min(a.cs, L - j0);
   const float scale = rsqrtf(static_cast<float>(d));
   float* part = a.part + ((((size_t)b * a.Hkv + hk) * a.n_chunks + c) * a.qmax) * part_stride(d);
-  // query qi of the item is head hk * G + qi % G of token tok0 + qi / G
-  auto q_src = [&](int qi) { return a.q + (size_t)(tok0 + qi / G) * a.Hq * d + (hk * G + qi % G) * d; };
 
-  // 1. the chunk's slots and mask bits (independent of this step's projections)
+  // 1. the chunk's slots and mask bits (independent of this step's projections);
+  //    packed mode (Section 8.6): one mask row per token, each query reads its
+  //    token's row and no implicit causal bound applies
   if (tid < kChunk) {
     int slot = 0, vis = 0;
     if (tid < nj) {
-      slot = __ldcg(sp->bt + (size_t)b * a.cap + j0 + tid);
-      vis = __ldcg(sp->mask + (size_t)b * sp->mask_stride + j0 + tid) != 0;
+      slot = __ldcg(a.bt + (size_t)b * a.cap + j0 + tid);
+      vis = a.packed ? 1 : __ldcg(a.mask + (size_t)b * a.mask_stride + j0 + tid) != 0;
     }
     slot_s[tid] = slot;
     vis_s[tid] = vis;
   }
-  __syncthreads();
+  if (a.packed)
+    for (int e = tid; e < nb * nj; e += kThreads)
+      vis_t[(e / nj) * kChunk + e % nj] = __ldcg(a.mask + (size_t)(tok0 + e / nj) * a.mask_stride + j0 + e % nj) != 0;
+  cbar();
   {
     constexpr int kRowPieces = kChunk * KP;
     constexpr int kPer = (2 * kRowPieces + kThreads - 1) / kThreads;
-    constexpr int kQPieces = S::kQg * d / 4;
-    constexpr int kQPer = (kQPieces + kThreads - 1) / kThreads;
-    const int qn0 = min(S::kQg, Q);
     uint4 v[kPer];
-    float4 qv[kQPer];
-    auto load_row_piece = [&](int pi, int r) {
+    auto row_of = [&](int r) {
       const int sl = slot_s[r];
-      const size_t row = (((size_t)(sl / a.cap) * a.Hkv + hk) * a.cap + sl % a.cap) * d;
-      return __ldcg(reinterpret_cast<const uint4*>((pi >= kRowPieces ? vpool : kpool) + row) + pi % KP);
+      return (((size_t)(sl / a.cap) * a.Hkv + hk) * a.cap + sl % a.cap) * d;
     };
     // 2. K/V rows of entries from earlier steps: in flight during the wait
 #pragma unroll
     for (int i = 0; i < kPer; ++i) {
       const int pi = tid + i * kThreads, r = (pi % kRowPieces) / KP;
       v[i] = make_uint4(0, 0, 0, 0);
-      if (pi < 2 * kRowPieces && r < nj && j0 + r < P) v[i] = load_row_piece(pi, r);
+      if (pi < 2 * kRowPieces && r < nj && j0 + r < P)
+        v[i] = __ldcg(reinterpret_cast<const uint4*>((pi >= kRowPieces ? vpool : kpool) + row_of(r)) + pi % KP);
     }
-    // 3. wait (bounded) for this kv head's q|k|v row-blocks: its G q heads,
-    //    its k and its v
-    {
-      const int per_head = d / kRowsPerBlock > 0 ? d / kRowsPerBlock : 1;
-      const int nq = G * d / kRowsPerBlock, n = nq + 2 * per_head;
-      if (tid < n) {
-        const int r = tid < nq ? hk * G * d / kRowsPerBlock + tid
-                               : (tid < nq + per_head ? a.rb_k0 + hk * per_head + (tid - nq)
-                                                      : a.rb_v0 + hk * per_head + (tid - nq - per_head));
-        uint32_t it = 0;
-        while (ld_acquire_u32(a.rb_done + r) != qkv_epoch) {
-          if (++it > (1u << 22)) {
-            atomicOr(status, ST_WAIT_TIMEOUT);
-            break;
-          }
-          __nanosleep(64);
-        }
-      }
-      __syncthreads();
-    }
-    // 4. the rows this step appended, and the queries
+    if (tid == 0) wait_count(a.cnt_kv + hk, a.kv_units, status, a.limit);
+    cbar();
 #pragma unroll
     for (int i = 0; i < kPer; ++i) {
       const int pi = tid + i * kThreads, r = (pi % kRowPieces) / KP;
-      if (pi < 2 * kRowPieces && r < nj && j0 + r >= P) v[i] = load_row_piece(pi, r);
-    }
-#pragma unroll
-    for (int i = 0; i < kQPer; ++i) {
-      const int pi = tid + i * kThreads, qi = pi / (d / 4);
-      qv[i] = (pi < kQPieces && qi < qn0) ? __ldcg(reinterpret_cast<const float4*>(q_src(qi)) + pi % (d / 4))
-                                          : make_float4(0.f, 0.f, 0.f, 0.f);
-    }
-#pragma unroll
-    for (int i = 0; i < kPer; ++i) {
-      const int pi = tid + i * kThreads, r = (pi % kRowPieces) / KP;
-      if (pi < 2 * kRowPieces) {
+      if (pi < 2 * kRowPieces && r < nj && j0 + r < P) {
         uint4* dst = pi >= kRowPieces ? reinterpret_cast<uint4*>(Vs + r * d) : reinterpret_cast<uint4*>(Ks + r * S::kKld);
         dst[pi % KP] = v[i];
       }
     }
-#pragma unroll
-    for (int i = 0; i < kQPer; ++i) {
-      const int pi = tid + i * kThreads;
-      if (pi < kQPieces) reinterpret_cast<float4*>(qsm)[pi] = qv[i];
+  }
+  // 3. the entries this step appends (they lie in the request's last chunks)
+  {
+    const int r0 = max(P - j0, 0), nnew = nj - r0;
+    if (nnew > 0) {
+      const int k_first = a.Hq * d, v_first = (a.Hq + a.Hkv) * d;
+      for (int e = tid; e < nnew * half; e += kThreads) {
+        const int r = r0 + e / half, i = e % half;
+        const int m = tok0 + (j0 + r - P);
+        const long long* row = a.acc + (size_t)m * a.acc_ld;
+        const int R = rot_row(k_first, hk, i, d);
+        const float lo = fixed_to_f32(__ldcg(row + R)), hi = fixed_to_f32(__ldcg(row + R + 8));
+        const float2 cs = a.rope[(size_t)sp->tok_pos[m] * half + i];
+        const uint16_t klo = f2h(lo * cs.x - hi * cs.y), khi = f2h(hi * cs.x + lo * cs.y);
+        Ks[r * S::kKld + i] = klo;
+        Ks[r * S::kKld + half + i] = khi;
+        const int sl = sp->tok_slot[m];
+        uint16_t* kp = kpool + (((size_t)(sl / a.cap) * a.Hkv + hk) * a.cap + sl % a.cap) * d;
+        kp[i] = klo;
+        kp[half + i] = khi;
+      }
+      for (int e = tid; e < nnew * d; e += kThreads) {
+        const int r = r0 + e / d, i = e % d;
+        const int m = tok0 + (j0 + r - P);
+        const uint16_t vv = f2h(fixed_to_f32(__ldcg(a.acc + (size_t)m * a.acc_ld + v_first + hk * d + i)));
+        Vs[r * d + i] = vv;
+        const int sl = sp->tok_slot[m];
+        vpool[(((size_t)(sl / a.cap) * a.Hkv + hk) * a.cap + sl % a.cap) * d + i] = vv;
+      }
+    }
+    // rows past the chunk's end take part with weight zero: keep them finite
+    for (int e = tid; e < (kChunk - nj) * KP; e += kThreads) {
+      const int r = nj + e / KP;
+      if (r < a.cs) {
+        reinterpret_cast<uint4*>(Ks + r * S::kKld)[e % KP] = make_uint4(0, 0, 0, 0);
+        reinterpret_cast<uint4*>(Vs + r * d)[e % KP] = make_uint4(0, 0, 0, 0);
+      }
     }
   }
   for (int q0 = 0; q0 < Q; q0 += S::kQg) {
     const int qn = min(S::kQg, Q - q0);
-    if (q0 > 0) {
-      __syncthreads();
-      for (int pi = tid; pi < qn * (d / 4); pi += kThreads)
-        reinterpret_cast<float4*>(qsm)[pi] =
-            __ldcg(reinterpret_cast<const float4*>(q_src(q0 + pi / (d / 4))) + pi % (d / 4));
-    }
-    __syncthreads();
+    if (q0 > 0) cbar();
+    attn_load_queries<DPL>(a, sp, hk, tok0, q0, qn, qsm);
+    cbar();
     for (int qi = warp; qi < qn; qi += kWarps) {
       const float* qq = qsm + qi * d;
       // lane scores entries lane, lane + 32, ... (cs / 32 of them)
@@ -608,7 +674,7 @@ __device__ __noinline__ void attn_item_cta(const AttnView* ap, int layer, const 
 #pragma unroll
       for (int k = 0; k < kChunk / 32; ++k) {
         const int e = lane + 32 * k;
-        vis[k] = e < nj && vis_s[e] && j0 + e <= lim;
+        vis[k] = e < nj && vis_s[e] && (a.packed ? vis_t[(q / G) * kChunk + e] != 0 : j0 + e <= lim);
         sc[k] = vis[k] ? sc[k] * scale : -INFINITY;
         mx = fmaxf(mx, sc[k]);
       }
@@ -628,7 +694,7 @@ __device__ __noinline__ void attn_item_cta(const AttnView* ap, int layer, const 
         part[(size_t)q * part_stride(d) + 1] = l;
       }
     }
-    __syncthreads();
+    cbar();
     for (int w = tid; w < qn * (d / 2); w += kThreads) {
       const int qi = w / (d / 2), dp = w % (d / 2);
       const float* pq = ps + qi * kChunk;
@@ -645,17 +711,17 @@ __device__ __noinline__ void attn_item_cta(const AttnView* ap, int layer, const 
   }
   // the item's partials are written (and the area is free for the next item);
   // the release orders them before the count the merging CTA acquires
-  __syncthreads();
+  cbar();
   if (!a.last_merges) {
     if (tid == 0) red_release_add_s32(&a.cnt[b * a.Hkv + hk], 1);
     return;
   }
   __shared__ int s_last;
   if (tid == 0) s_last = atom_add_acq_rel(&a.cnt[b * a.Hkv + hk], 1) == n_chunks_of(L, a.cs) - 1;
-  __syncthreads();
+  cbar();
   if (s_last) {
     for (int qi = warp; qi < Q; qi += kWarps) attn_merge_warp<DPL>(ap, sp, b, hk, qi, lane);
-    __syncthreads();
+    cbar();
     if (tid == 0) a.cnt[b * a.Hkv + hk] = 0;
   }
 }
@@ -669,54 +735,68 @@ __device__ __noinline__ void attn_merge_cta(const AttnView* ap, const StepParams
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int L = sp->req_len[b], nb = sp->req_tok0[b + 1] - sp->req_tok0[b];
   const int Q = nb * (a.Hq / a.Hkv);
-  if (tid == 0) {
-    uint32_t it = 0;
-    while (ld_acquire_s32(&a.cnt[b * a.Hkv + hk]) < n_chunks_of(L, a.cs)) {
-      if (++it > (1u << 22)) {
-        atomicOr(status, ST_WAIT_TIMEOUT);
-        break;
-      }
-      __nanosleep(64);
-    }
-  }
-  __syncthreads();
+  if (tid == 0) wait_count(&a.cnt[b * a.Hkv + hk], n_chunks_of(L, a.cs), status, a.limit);
+  cbar();
   for (int qi = warp; qi < Q; qi += kWarps) attn_merge_warp<DPL>(ap, sp, b, hk, qi, lane);
-  __syncthreads();
+  cbar();
   if (tid == 0) a.cnt[b * a.Hkv + hk] = 0;
 }
 
 template <int NT, int GPU, int DPL>
-__global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant__ StepKernelArgs a) {
+__global__ void __launch_bounds__(kBlockThreads, 1) step_kernel(const __grid_constant__ StepKernelArgs a) {
   extern __shared__ __align__(128) uint8_t smem[];
   __shared__ GemvPhase s_gp[4];            // per projection kind: q|k|v, o, gate|up, down
-  __shared__ WarpStream<GPU> s_ws[kWarps];  // each warp's weight stream, between phases
+  __shared__ WarpRing<GPU> s_ring[kWarps];  // each consumer warp's ring, between phases
   __shared__ AttnView s_av;
+  __shared__ StepParams s_sp;
+  __shared__ const uint16_t* s_rowp[kMaxTokens];  // the step's fp16 input rows
   using SS = StepSmem<GPU>;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  uint8_t* ring = smem + (size_t)warp * kRingSlots * Geom<GPU>::kUnitBytes;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + SS::kRing) + warp * kRingSlots;
+  uint8_t* rings = smem;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + SS::kRing);
+  uint64_t* empty = full + kWarps * kRingSlots;
   uint8_t* att_area = smem + SS::kRing + SS::kBars;
   static_assert(AttnSmem<DPL>::kBytes <= SS::kQ, "attention area too small");
   OpDesc* s_ops = reinterpret_cast<OpDesc*>(smem + SS::kFixed);
-  for (int i = threadIdx.x; i < 4 * a.L; i += kThreads) s_ops[i] = a.ops[i];
-  __syncthreads();
-  unsigned long long target = a.barrier_base;
-  int nsync = 1;
-  if (threadIdx.x == 0 && blockIdx.x == 0) a.phase_clock[0] = globaltimer();
-  {
-    WarpStream<GPU> ws;
-    ws.init(s_ops, 4 * a.L, blockIdx.x, gridDim.x, warp, kWarps, ring, bars, kRingSlots == 4 ? 2 : 1, lane);
-    ws.fill(lane);
-    if (lane == 0) s_ws[warp] = ws;
-    __syncwarp();
+  for (int i = threadIdx.x; i < 4 * a.L; i += kBlockThreads) s_ops[i] = a.ops[i];
+  if (threadIdx.x == 0) {
+    ring_init_barriers(full, empty, kWarps * kRingSlots);
+    if (blockIdx.x == 0) a.phase_clock[0] = globaltimer();
   }
-
-  if (blockIdx.x == 0) prologue_cta(a.pro);
-  grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
-
-  const StepParams* sp = a.pro.sp;
-  const bool skip = __ldcg(&sp->abort_step) != 0;
-  const int M = a.pro.M;
+  prologue_params(a.pro, &s_sp, s_rowp);  // ends with a block-wide barrier
+  const int n_barriers = 4 * a.L + 1;
+  if (s_sp.abort_step) {
+    // every CTA sees the same inputs and rejects the step alike: count this
+    // launch's barrier arrivals at once and write nothing
+    if (threadIdx.x == 0) {
+      red_release_add(a.barrier, (unsigned long long)n_barriers);
+      if (blockIdx.x == 0) {
+        atomicOr(a.pro.status, s_sp.abort_step & ~ST_STICKY);
+        *reinterpret_cast<volatile int*>(a.status_out) = ld_acquire_s32(a.pro.status);
+      }
+    }
+    return;
+  }
+  if (warp == kWarps) {  // the producer warp
+    ring_producer<GPU>(s_ops, 4 * a.L, blockIdx.x, gridDim.x, kWarps, rings, full, empty, kRingSlots == 4 ? 2 : 1,
+                       a.status, kProducerLimit, lane);
+    return;
+  }
+  // ---- consumer warps from here on: CTA barriers are cbar() ----
+  const StepParams* sp = &s_sp;
+  const int M = sp->M;
+  GridBarrier gb{a.barrier, a.barrier_base, a.status, a.phase_clock, 0, 0, a.debug_skip_arrival, a.wait_limit};
+  if (lane == 0) {
+    WarpRing<GPU> r;
+    r.ring = rings + (size_t)warp * kRingSlots * Geom<GPU>::kUnitBytes;
+    r.full = full + warp * kRingSlots;
+    r.empty = empty + warp * kRingSlots;
+    r.slot_mask = kRingSlots - 1;
+    r.slot_shift = kRingSlots == 4 ? 2 : 1;
+    r.n_used = 0;
+    r.timed_out = false;
+    s_ring[warp] = r;
+  }
   // Each CTA normalises the whole hidden state for itself; when the M rows
   // fit, it keeps them in the attention area (idle during the q|k|v and
   // gate|up projections) and the projections read them from there.  Rows are
@@ -726,6 +806,7 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
   const bool xn_smem = kNormInSmem && a.Kp_H == a.H && (size_t)M * xn_ld * 2 <= SS::kQ;
   uint16_t* xn = xn_smem ? reinterpret_cast<uint16_t*>(att_area) : a.act_h;
   const int xn_out_ld = xn_smem ? xn_ld : a.Kp_H;
+  const int G = a.Hq / a.Hkv;
   if (threadIdx.x < 4) {
     const int k = threadIdx.x;
     GemvPhase gp{};
@@ -734,30 +815,25 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
     gp.M = M;
     gp.act_s = (k == 0 || k == 2) && xn_smem ? smem_addr(att_area) : 0u;
     gp.act_s_ld = xn_ld;
-    gp.skip = skip;
-    gp.partials = a.partials;
-    gp.flags = a.flags;
     gp.status = a.status;
-    gp.sp = sp;
     gp.ep.kind = k == 0 ? EPI_QKV : k == 2 ? EPI_SWIGLU : EPI_RESID;
     gp.ep.dims = OpDims{k, a.Hq, a.Hkv, a.d, a.F, a.H};
-    gp.ep.q = a.q;
-    gp.ep.kpool = a.kpool;
-    gp.ep.vpool = a.vpool;
-    gp.ep.layer_stride = a.layer_stride;
-    gp.ep.cap = a.cap;
-    gp.ep.rope = a.rope;
-    gp.ep.x = a.x;
-    gp.ep.ss = (k == 1 || k == 3) ? a.ss : nullptr;
-    gp.ep.out_layer = k == 3 ? a.L - 1 : -1;
+    gp.ep.acc = k == 0 ? a.acc_qkv : k == 2 ? a.acc_gu : a.X;
+    gp.ep.acc_ld = k == 0 ? (a.Hq + 2 * a.Hkv) * a.d : k == 2 ? s_ops[2].n_rb * kRowsPerBlock : a.H;
+    gp.ep.cnt = k == 0 ? a.cnt_kv : k == 2 ? a.cnt_gu : nullptr;
     gp.ep.h = a.act_f;
     gp.ep.h_ld = a.Kp_F;
-    gp.done_flags = k == 0 ? a.rb_done : nullptr;
+    gp.kv_rb_q = G * a.d / kRowsPerBlock;
+    gp.kv_rb_per_head = a.d / kRowsPerBlock;
+    gp.kv_rb_k = a.Hq * a.d / kRowsPerBlock;
+    gp.kv_rb_v = (a.Hq + a.Hkv) * a.d / kRowsPerBlock;
     s_gp[k] = gp;
   }
   if (threadIdx.x == 32) {
     AttnView av{};
-    av.q = a.q;
+    av.acc = a.acc_qkv;
+    av.acc_ld = (a.Hq + 2 * a.Hkv) * a.d;
+    av.rope = a.rope;
     av.kpool = a.kpool;
     av.vpool = a.vpool;
     av.layer_stride = a.layer_stride;
@@ -766,12 +842,16 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
     av.Hkv = a.Hkv;
     av.d = a.d;
     av.n_chunks = a.n_chunks;
-    av.qmax = kMaxTokens * (a.Hq / a.Hkv);
+    av.qmax = kMaxTokens * G;
     av.part = a.attn_part;
     av.cnt = a.attn_cnt;
-    av.rb_done = a.rb_done;
-    av.rb_k0 = a.Hq * a.d / kRowsPerBlock;
-    av.rb_v0 = (a.Hq + a.Hkv) * a.d / kRowsPerBlock;
+    av.cnt_kv = a.cnt_kv;
+    av.kv_units = (G + 2) * (a.d / kRowsPerBlock) * s_ops[0].upr;
+    av.bt = a.pro.bt_dst;
+    av.mask = a.mask;
+    av.mask_stride = a.mask_stride;
+    av.packed = a.packed;
+    av.limit = a.wait_limit;
     int items = 0;
     for (int b = 0; b < sp->B; ++b) items += a.Hkv * n_chunks_of(sp->req_len[b], kAttnChunkMin);
     // the smallest item size that needs one round of CTAs, else the largest
@@ -786,21 +866,32 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
     av.out_ld = a.Kp_dq;
     s_av = av;
   }
-  __syncthreads();
-  auto gemv = [&](int op, int l) { gemv_phase<NT, GPU>(&s_ws[warp], op, &s_gp[op & 3], l, a.epoch_base + op, lane); };
+  cbar();
+  prologue_work(a.pro, sp, s_rowp, a.X);
+  cbar();
+  gb.arrive();  // split barrier: waited for before the first attention
+
+  const int g = blockIdx.x * kWarps + warp, nw = gridDim.x * kWarps;
+  const int gt = blockIdx.x * kThreads + threadIdx.x, gs = gridDim.x * kThreads;
+  auto gemv = [&](int op) { gemv_phase<NT, GPU>(&s_ring[warp], &s_ops[op], &s_gp[op & 3], g, nw, lane); };
+  const int qkv_rows = (a.Hq + 2 * a.Hkv) * a.d;
 
   for (int l = 0; l < a.L; ++l) {
     const uint16_t* nrm = a.norms + (size_t)l * 2 * a.H;
     // attention block
-    if (!skip) rmsnorm_cta(a.x, a.H, nrm, a.eps, a.ss, xn, xn_out_ld, M);
-    gemv(4 * l + 0, l);
-    if (!skip) {
-      if (xn_smem) __syncthreads();  // the attention items reuse the normalised rows' space
+    if (l == 0)
+      rmsnorm_cta<false>(a.X, s_rowp, a.H, nrm, a.eps, xn, xn_out_ld, M);
+    else
+      rmsnorm_cta<true>(a.X, s_rowp, a.H, nrm, a.eps, xn, xn_out_ld, M);
+    gemv(4 * l + 0);
+    if (l == 0) gb.wait();            // the prologue's tables and residual are complete
+    else if (xn_smem) cbar();         // the attention items reuse the normalised rows' space
+    {
       int total = 0;
       for (int b = 0; b < sp->B; ++b) total += a.Hkv * n_chunks_of(sp->req_len[b], s_av.cs);
       for (int item = blockIdx.x; item < total; item += gridDim.x) {
         int b, hk, c;
-        if (decode_item(sp, a.Hkv, s_av.cs, item, b, hk, c)) attn_item_cta<DPL>(&s_av, l, sp, b, hk, c, att_area, a.epoch_base + 4 * l, a.status);
+        if (decode_item(sp, a.Hkv, s_av.cs, item, b, hk, c)) attn_item_cta<DPL>(&s_av, l, sp, b, hk, c, att_area, a.status);
       }
       // merges, when CTAs take several items: (b, hk) goes to the CTA that
       // took its last chunk
@@ -811,20 +902,29 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
         base += a.Hkv * nc;
       }
     }
-    grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
-    gemv(4 * l + 1, l);
-    grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
+    gb.sync();
+    // the q|k|v sums and counts are consumed: clear them for the next layer
+    for (int e = gt; e < M * qkv_rows; e += gs) __stcg(a.acc_qkv + e, 0LL);
+    if (blockIdx.x == 0 && threadIdx.x < a.Hkv) __stcg(a.cnt_kv + threadIdx.x, 0);
+    gemv(4 * l + 1);
+    gb.sync();
     // MLP block
-    if (!skip) rmsnorm_cta(a.x, a.H, nrm + a.H, a.eps, a.ss, xn, xn_out_ld, M);
-    gemv(4 * l + 2, l);
-    grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
-    gemv(4 * l + 3, l);
-    if (l + 1 < a.L) grid_sync(a.barrier, target, a.status, a.phase_clock, nsync);
+    rmsnorm_cta<true>(a.X, s_rowp, a.H, nrm + a.H, a.eps, xn, xn_out_ld, M);
+    gemv(4 * l + 2);
+    gb.sync();
+    gemv(4 * l + 3);
+    gb.sync();
   }
-  if (s_ws[warp].timed_out && lane == 0) atomicOr(a.status, ST_WAIT_TIMEOUT);
+  // hidden_out = fp16(x): one rounding from the exact fixed-point value
+  for (int e = gt; e < M * a.H; e += gs) {
+    const double v = static_cast<double>(__ldcg(a.X + e)) * kFixInv;
+    a.pro.hidden_out[e] = __half_as_ushort(__double2half(v));
+  }
+  if (blockIdx.x == 0 && threadIdx.x < sp->B) a.pro.lens[threadIdx.x] = sp->req_len[threadIdx.x];
+  if (s_ring[warp].timed_out && lane == 0) atomicOr(a.status, ST_WAIT_TIMEOUT);
   // The last CTA to finish hands a nonzero status to the host-mapped mirror,
   // so no copy-engine transfer has to follow the step on the stream.
-  __syncthreads();
+  cbar();
   if (threadIdx.x == 0 && atom_add_acq_rel(a.exit_count, 1) == (int)gridDim.x - 1) {
     *a.exit_count = 0;
     const int st = ld_acquire_s32(a.status);
@@ -837,7 +937,7 @@ cudaError_t launch_t(const StepKernelArgs& a, int grid, cudaStream_t s) {
   auto kern = step_kernel<NT, GPU, DPL>;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
-  cfg.blockDim = dim3(kThreads);
+  cfg.blockDim = dim3(kBlockThreads);
   cfg.dynamicSmemBytes = StepSmem<GPU>::total(a.L);
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
@@ -856,7 +956,7 @@ cudaError_t setup_t() {
 
 }  // namespace
 
-int step_barriers(int n_layers) { return 4 * n_layers; }
+int step_barriers(int n_layers) { return 4 * n_layers + 1; }
 
 size_t step_attention_part_floats(int B, int Hkv, int n_chunks, int G, int d) {
   return (size_t)B * Hkv * n_chunks * (kMaxTokens * G) * part_stride(d);

@@ -20,4 +20,7 @@ def _build_host_libs():
     import synth
     synth.build()
     oracle.build()
+    # the oracle parallelises over independent output rows only: results do
+    # not depend on the thread count
+    oracle.set_threads(os.cpu_count() or 1)
     yield

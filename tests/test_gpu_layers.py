@@ -141,7 +141,7 @@ def test_8b_every_layer_fixed_bar_decode_and_16_verify_steps():
 def test_70b_every_layer_fixed_bar_4096_cache():
     shape = synth.LLAMA70B_STAGE
     seed = 20261203
-    plan = verify_plan(seed, 3, 3)
+    plan = verify_plan(seed, 2, 2)
 
     def first(s, n):
         return "hidden_in", synth.hidden_in(shape, seed, 300 + s, n)

@@ -78,7 +78,7 @@ def test_phase_times_cover_the_step(tiny):
     prefill(eng, TINY, SEED, 0, 40)
     eng.step([1], np.array([40], np.int32), np.ones(41, np.uint8), hidden_in=synth.hidden_in(TINY, SEED, 0, 1))
     t = pkg.shard_debug_phase_times(sh.h, TINY.n_layers)
-    assert len(t) == len(pkg.PHASES) * TINY.n_layers and all(x >= 0 for x in t) and sum(t) > 0
+    assert len(t) == len(pkg.PHASES) * TINY.n_layers + 1 and all(x >= 0 for x in t) and sum(t) > 0
     eng.close()
 
 
