@@ -9,6 +9,7 @@ namespace shard {
 namespace {
 
 constexpr int kW = kGemvWarps;  // consumer warps per CTA
+constexpr int kBlock = (kW + (kSelfRefill ? 0 : 1)) * 32;
 constexpr int kCtasPerSm = 1;
 
 template <int GPU>
@@ -22,13 +23,12 @@ static_assert(smem_bytes<1>() <= 225 * 1024 && smem_bytes<2>() <= 225 * 1024 && 
               "standalone projection ring too large");
 
 template <int NT, int GPU>
-__global__ void __launch_bounds__((kW + 1) * 32, 1) gemv_kernel(const __grid_constant__ GemvArgs a) {
+__global__ void __launch_bounds__(kBlock, 1) gemv_kernel(const __grid_constant__ GemvArgs a) {
+  constexpr int kSlots = Geom<GPU>::kGemvSlots;
   extern __shared__ __align__(128) uint8_t smem[];
   __shared__ OpDesc s_op[1];
   __shared__ GemvPhase s_gp;
-  __shared__ WarpRing<GPU> s_ring[kW];
-  constexpr int kSlots = Geom<GPU>::kGemvSlots;
-  constexpr int kShift = kSlots == 4 ? 2 : 1;
+  __shared__ WarpRing<GPU, kSlots> s_ring[kW];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   uint8_t* rings = smem;
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + (size_t)kW * kSlots * Geom<GPU>::kUnitBytes);
@@ -44,26 +44,27 @@ __global__ void __launch_bounds__((kW + 1) * 32, 1) gemv_kernel(const __grid_con
     s_gp = p;
     ring_init_barriers(full, empty, kW * kSlots);
   }
-  if (lane == 0 && warp < kW) {
-    WarpRing<GPU> r;
+  __syncthreads();
+  if (!kSelfRefill && warp == kW) {
+    // the weights do not depend on the preceding kernel: start streaming them
+    ring_producer<GPU, kSlots>(s_op, 1, blockIdx.x, gridDim.x, kW, rings, full, empty, a.status, 1u << 22, lane);
+    return;
+  }
+  const int g = blockIdx.x * kW + warp, nw = gridDim.x * kW;
+  {
+    WarpRing<GPU, kSlots> r;
     r.ring = rings + (size_t)warp * kSlots * Geom<GPU>::kUnitBytes;
     r.full = full + warp * kSlots;
     r.empty = empty + warp * kSlots;
-    r.slot_mask = kSlots - 1;
-    r.slot_shift = kShift;
     r.n_used = 0;
     r.timed_out = false;
-    s_ring[warp] = r;
-  }
-  __syncthreads();
-  if (warp == kW) {
-    // the weights do not depend on the preceding kernel: start streaming them
-    ring_producer<GPU>(s_op, 1, blockIdx.x, gridDim.x, kW, rings, full, empty, kShift, a.status, 1u << 22, lane);
-    return;
+    if (kSelfRefill) r.start(s_op, 1, g, nw, lane);  // the weights do not depend on the preceding kernel
+    if (lane == 0) s_ring[warp] = r;
+    __syncwarp();
   }
   pdl_launch_dependents();
   pdl_wait();
-  gemv_phase<NT, GPU>(&s_ring[warp], &s_op[0], &s_gp, blockIdx.x * kW + warp, gridDim.x * kW, lane);
+  gemv_phase<NT, GPU, kSlots>(&s_ring[warp], &s_op[0], &s_gp, g, nw, lane);
   if (s_ring[warp].timed_out && lane == 0) atomicOr(a.status, ST_WAIT_TIMEOUT);
 }
 
@@ -71,7 +72,7 @@ template <int NT, int GPU>
 cudaError_t launch_t(const GemvArgs& a, int grid, cudaStream_t s, bool pdl) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
-  cfg.blockDim = dim3((kW + 1) * 32);
+  cfg.blockDim = dim3(kBlock);
   cfg.dynamicSmemBytes = smem_bytes<GPU>();
   cfg.stream = s;
   cudaLaunchAttribute attr[1];

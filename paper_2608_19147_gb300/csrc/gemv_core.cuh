@@ -7,16 +7,15 @@
 // number of bytes and keeps its sums in registers for as long as its run
 // stays inside one row-block.
 //
-// Weight streaming.  Every consumer warp owns a ring of shared-memory slots
-// (a power of two).  One producer warp per CTA fills them: its lane w walks
-// consumer warp w's runs of every projection of the launch in order and
-// issues one bulk copy (TMA, non-tensor) per unit into the next free slot,
-// completion signalled on the slot's "full" mbarrier; the consumer releases
-// the slot on its "empty" mbarrier after the unit's fragments are in
-// registers.  Because the weights never depend on earlier work, the rings run
-// ahead across projections: while consumers wait at a barrier or work on
-// norms and attention, their next projection's first units are already
-// arriving, and consumers execute no stream bookkeeping at all.
+// Weight streaming.  Every consumer warp owns a ring of shared-memory slots,
+// filled with one bulk copy (TMA, non-tensor) per unit, completion signalled
+// on the slot's "full" mbarrier.  The warp's stream is its run of every
+// projection of the launch, in order; because the weights never depend on
+// earlier work, the rings run ahead across projections: while consumers wait
+// at a barrier or work on norms and attention, their next projection's first
+// units are already arriving.  The slot a warp has consumed is refilled
+// either by the warp's own lane 0 at once (kSelfRefill) or by a producer warp
+// that watches the slots' "empty" mbarriers.
 //
 // Per unit, a lane turns each 32-bit code word into the four registers of its
 // m16n8k16 A fragment with one AND per register (the codes as fp16
@@ -38,16 +37,24 @@
 
 namespace shard {
 
-constexpr int kRingSlots = 2;  // step kernel: units in flight per consumer warp (measured: a third adds nothing)
-constexpr int kCtaWarps = 11;   // consumer warps per CTA of the step kernel (+ 1 producer: 3 warps per SM sub-partition)
-constexpr int kGemvWarps = 11;  // consumer warps per CTA of the standalone projection kernel (+ 1 producer)
+// Weight streaming: with kSelfRefill, each consumer warp's lane 0 refills the
+// slot the warp has just consumed with its next unit; otherwise a producer
+// warp per CTA fills every consumer's ring.  Consumer warps per CTA: 12
+// (3 per SM sub-partition), or 11 beside the producer (the sub-partition's
+// register file caps 4 warps at 128 registers each).
+constexpr bool kSelfRefill = true;
+constexpr int kRingSlots = 3;  // step kernel: units in flight per consumer warp (group 64 and 128)
+constexpr int kCtaWarps = kSelfRefill ? 12 : 11;   // consumer warps per CTA of the step kernel
+constexpr int kGemvWarps = kSelfRefill ? 12 : 11;  // consumer warps per CTA of the standalone projection kernel
 
 template <int GPU>
 struct Geom {
   static constexpr int kUnitBytes = kCodeBytes + GPU * kMetaBytesPerGroup;
   static constexpr int kBlocksPerGroup = 8 / GPU;
+  // the step kernel's slots (group 32 units are larger: two)
+  static constexpr int kStepSlots = GPU == 4 ? 2 : kRingSlots;
   // the standalone projection (no attention area competes for shared
-  // memory): four slots per warp where 12 warps' rings fit in 216 KB, else two
+  // memory): four slots per warp where the rings fit in 216 KB, else two
   static constexpr int kGemvSlots = kGemvWarps * 4 * kUnitBytes <= 216 * 1024 ? 4 : 2;
 };
 
@@ -91,8 +98,15 @@ __device__ __forceinline__ void red_add_s64(long long* p, long long v) {
   asm volatile("red.relaxed.gpu.global.add.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
 }
 __device__ __forceinline__ long long to_fixed(float v) { return __float2ll_rn(v * kFixOne); }
-// int64 -> fp32 rounds once; the power-of-two scale is exact
-__device__ __forceinline__ float fixed_to_f32(long long v) { return __ll2float_rn(v) * 2.3283064365386963e-10f; }
+// value = v * 2^-32 with v = hi * 2^32 + lo (lo unsigned): hi + lo * 2^-32
+// in fp32 from two 32-bit conversions (int64 conversions are a slow path).
+// hi is exact (|hi| < 2^24); the result is within one fp32 ulp of the exact
+// value and the same in every CTA.
+__device__ __forceinline__ float fixed_to_f32(long long v) {
+  const int hi = static_cast<int>(v >> 32);
+  const unsigned lo = static_cast<unsigned>(v & 0xFFFFFFFFll);
+  return fmaf(__uint2float_rn(lo), 2.3283064365386963e-10f, static_cast<float>(hi));
+}
 
 // ---------------------------------------------------------------------------
 // Weight rings.
@@ -107,28 +121,94 @@ __device__ __forceinline__ bool mbar_test_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
-// Consumer side of one warp's ring.
-template <int GPU>
+// One warp's view of the weight stream: the warp's run of every projection
+// of the launch, in order (ops[0 .. n_ops)).
+struct StreamCursor {
+  const OpDesc* ops;
+  int n_ops, g, nw;
+  int op, u, end;
+  const uint8_t* src;
+
+  __device__ __forceinline__ void open(int o, int UB) {
+    const int T = ops[o].n_rb * ops[o].upr;
+    u = part_start(T, g, nw);
+    end = part_start(T, g + 1, nw);
+    src = ops[o].units + (size_t)u * UB;
+  }
+  __device__ __forceinline__ void init(const OpDesc* ops_, int n_ops_, int g_, int nw_, int UB) {
+    ops = ops_;
+    n_ops = n_ops_;
+    g = g_;
+    nw = nw_;
+    op = 0;
+    u = end = 0;
+    src = nullptr;
+    if (n_ops > 0) open(0, UB);
+  }
+  // The next unit's address, or false at the end of the stream.
+  __device__ __forceinline__ bool next(const uint8_t*& unit, int UB) {
+    while (u >= end) {
+      if (++op >= n_ops) return false;
+      open(op, UB);
+    }
+    unit = src;
+    src += UB;
+    ++u;
+    return true;
+  }
+};
+
+// Consumer side of one warp's ring of S slots.
+template <int GPU, int S>
 struct WarpRing {
   static constexpr int UB = Geom<GPU>::kUnitBytes;
-  uint8_t* ring;       // [slots][UB]
-  uint64_t* full;      // [slots]
-  uint64_t* empty;     // [slots]
-  uint32_t slot_mask;  // slots - 1
-  int slot_shift;      // log2(slots)
+  uint8_t* ring;       // [S][UB]
+  uint64_t* full;      // [S]
+  uint64_t* empty;     // [S] (producer mode)
   uint32_t n_used;
   bool timed_out;
+  StreamCursor cur;    // self-refill mode: lane 0's copy drives the refills
+  uint64_t policy;
 
+  __device__ __forceinline__ void issue(uint32_t slot, const uint8_t* src) {
+    mbar_arrive_expect_tx(&full[slot], UB);
+    // L2 evict-first: each weight byte is read once per launch
+    bulk_g2s_hint(ring + (size_t)slot * UB, src, UB, &full[slot], policy);
+  }
+  // Self-refill mode: lane 0 fills the first S slots.
+  __device__ __forceinline__ void start(const OpDesc* ops, int n_ops, int g, int nw, int lane) {
+    cur.init(ops, n_ops, g, nw, UB);
+    policy = l2_policy_evict_first();
+    if (lane == 0)
+      for (uint32_t s = 0; s < (uint32_t)S; ++s) {
+        const uint8_t* src;
+        if (!cur.next(src, UB)) break;
+        issue(s, src);
+      }
+  }
   // Waits (bounded) for the next unit; returns its slot.
   __device__ __forceinline__ const uint8_t* acquire() {
-    const uint32_t slot = n_used & slot_mask;
-    if (!timed_out && !mbar_wait(&full[slot], (n_used >> slot_shift) & 1)) timed_out = true;
+    const uint32_t slot = n_used % S;
+    if (!timed_out && !mbar_wait(&full[slot], (n_used / S) & 1)) timed_out = true;
     return ring + (size_t)slot * UB;
   }
-  // The unit's fragments are in registers: hand the slot back.
+  // The unit's fragments are in registers: refill the slot with the warp's
+  // next unit (self-refill), or hand it back to the producer.
   __device__ __forceinline__ void release(int lane) {
     __syncwarp();
-    if (lane == 0) mbar_arrive(&empty[n_used & slot_mask]);
+    const uint32_t slot = n_used % S;
+    if (lane == 0) {
+      if (kSelfRefill) {
+        const uint8_t* src;
+        if (cur.next(src, UB)) {
+          // the warp's generic-proxy reads of the slot come before the copy's writes
+          asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+          issue(slot, src);
+        }
+      } else {
+        mbar_arrive(&empty[slot]);
+      }
+    }
     ++n_used;
   }
 };
@@ -142,42 +222,53 @@ __device__ __forceinline__ void ring_init_barriers(uint64_t* full, uint64_t* emp
   mbar_fence_init();
 }
 
-// Producer: lane w < n_warps fills consumer warp w's ring with the warp's
-// runs of ops[0 .. n_ops), in order.  A slot is refilled once its previous
-// unit was released.  Bounded: a slot that stays busy for `limit` polls sets
-// ST_WAIT_TIMEOUT and ends the producer (the consumers' own bounded waits
+// Producer mode: lane w < n_warps fills consumer warp w's ring of S slots
+// with the warp's runs of ops[0 .. n_ops), in order; a slot is refilled once
+// its previous unit was released.  Every lane runs the same loop (ready
+// lanes issue, others wait for the next pass), so no lane's wait holds up
+// another's copy.  Bounded: `limit` passes without any copy set
+// ST_WAIT_TIMEOUT and end the producer (the consumers' own bounded waits
 // then give up too).
-template <int GPU>
+template <int GPU, int S>
 __device__ __noinline__ void ring_producer(const OpDesc* ops, int n_ops, int cta, int n_cta, int n_warps, uint8_t* rings,
-                                           uint64_t* full, uint64_t* empty, int slot_shift, int* status,
-                                           uint32_t limit, int lane) {
+                                           uint64_t* full, uint64_t* empty, int* status, uint32_t limit, int lane) {
   constexpr int UB = Geom<GPU>::kUnitBytes;
-  if (lane >= n_warps) return;
-  const uint32_t S = 1u << slot_shift, mask = S - 1;
-  uint8_t* ring = rings + (size_t)lane * S * UB;
-  uint64_t* f = full + lane * S;
-  uint64_t* e = empty + lane * S;
-  const int g = cta * n_warps + lane, nw = n_cta * n_warps;
-  const uint64_t policy = l2_policy_evict_first();  // each weight byte is read once per launch
-  uint32_t n = 0, spins = 0;
-  for (int op = 0; op < n_ops; ++op) {
-    const int T = ops[op].n_rb * ops[op].upr;
-    const int ub = part_start(T, g, nw), ue = part_start(T, g + 1, nw);
-    const uint8_t* src = ops[op].units + (size_t)ub * UB;
-    for (int u = ub; u < ue; ++u, ++n, src += UB) {
-      const uint32_t slot = n & mask;
-      if (n >= S) {
-        while (!mbar_test_wait(&e[slot], ((n >> slot_shift) - 1) & 1)) {
-          if (++spins > limit) {
-            atomicOr(status, ST_WAIT_TIMEOUT);
-            return;
-          }
-          __nanosleep(32);
-        }
-        spins = 0;
+  const bool mine = lane < n_warps;
+  uint8_t* ring = rings + (size_t)(mine ? lane : 0) * S * UB;
+  uint64_t* f = full + (mine ? lane : 0) * S;
+  uint64_t* e = empty + (mine ? lane : 0) * S;
+  StreamCursor cur;
+  cur.init(ops, mine ? n_ops : 0, cta * n_warps + lane, n_cta * n_warps, UB);
+  const uint64_t policy = l2_policy_evict_first();
+  bool active = mine;
+  const uint8_t* src = nullptr;
+  bool have = false;  // `src` holds the next unit, not yet issued
+  uint32_t n = 0, idle = 0;
+  while (true) {
+    if (active && !have) {
+      have = cur.next(src, UB);
+      active = have;
+    }
+    bool issued = false;
+    if (have) {
+      const uint32_t slot = n % S;
+      if (n < (uint32_t)S || mbar_test_wait(&e[slot], ((n / S) - 1) & 1)) {
+        mbar_arrive_expect_tx(&f[slot], UB);
+        bulk_g2s_hint(ring + (size_t)slot * UB, src, UB, &f[slot], policy);
+        ++n;
+        have = false;
+        issued = true;
       }
-      mbar_arrive_expect_tx(&f[slot], UB);
-      bulk_g2s_hint(ring + (size_t)slot * UB, src, UB, &f[slot], policy);
+    }
+    if (!__any_sync(0xffffffffu, active)) break;
+    if (__any_sync(0xffffffffu, issued)) {
+      idle = 0;
+    } else {
+      if (++idle > limit) {
+        if (lane == 0) atomicOr(status, ST_WAIT_TIMEOUT);
+        break;
+      }
+      __nanosleep(20);
     }
   }
 }
@@ -412,10 +503,10 @@ __device__ __forceinline__ void segment_end(const GemvPhase* pp, const float (&t
 // live in shared memory (ring_io, pp): nothing crosses the call through the
 // stack, whose local memory would miss the small L1 left next to the weight
 // rings.
-template <int NT, int GPU>
-__device__ __noinline__ void gemv_phase(WarpRing<GPU>* ring_io, const OpDesc* op, const GemvPhase* pp, int g, int nw,
+template <int NT, int GPU, int S>
+__device__ __noinline__ void gemv_phase(WarpRing<GPU, S>* ring_io, const OpDesc* op, const GemvPhase* pp, int g, int nw,
                                         int lane) {
-  WarpRing<GPU> ring = *ring_io;
+  WarpRing<GPU, S> ring = *ring_io;
   const GemvPhase& p = *pp;
   const int upr = op->upr;
   const int T = op->n_rb * upr;

@@ -275,7 +275,7 @@ cudaError_t step_setup(int group, int head_dim);
 int step_barriers(int n_layers);
 cudaError_t launch_step(const StepKernelArgs& a, int nt, int group, int grid, cudaStream_t s);
 size_t step_attention_part_floats(int B, int Hkv, int n_chunks, int G, int d);
-constexpr int kAttnChunk = 128;    // most cache entries per attention item
+constexpr int kAttnChunk = 64;     // most cache entries per attention item
 constexpr int kAttnChunkMin = 32;  // fewest (partials are laid out for this many per item)
 
 // Weight repacking (one fused op; all source pointers device).

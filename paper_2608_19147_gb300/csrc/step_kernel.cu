@@ -31,8 +31,8 @@ namespace {
 
 constexpr int kWarps = kCtaWarps;           // consumer warps
 constexpr int kThreads = kWarps * 32;       // consumer threads
-constexpr int kBlockThreads = kThreads + 32;  // + the producer warp
-constexpr int kChunk = kAttnChunk;  // most cache entries per attention item (four per lane)
+constexpr int kBlockThreads = kThreads + (kSelfRefill ? 0 : 32);  // + the producer warp, if any
+constexpr int kChunk = kAttnChunk;  // most cache entries per attention item (kChunk / 32 per lane)
 constexpr bool kNormInSmem = true;   // normalised activations in shared memory when they fit
 constexpr int kNormCache = 6;        // float4 pieces of the first row a thread keeps between the norm's passes
 // Polls of a busy slot before the producer gives up: a slot may legitimately
@@ -40,12 +40,19 @@ constexpr int kNormCache = 6;        // float4 pieces of the first row a thread 
 // bound is fixed and far above any step's length.
 constexpr uint32_t kProducerLimit = 1u << 22;
 
+// The attention area: one item's tiles at kChunk entries and head_dim 128
+// (AttnSmem), rounded up to 1 KB; it also holds the normalised rows when they fit.
+constexpr size_t kAttnArea =
+    ((size_t)kChunk * (128 + 8) * 2 + (size_t)kChunk * 128 * 2 + 16 * 128 * 4 + 16 * kChunk * 4 + 2 * kChunk * 4 +
+     (size_t)kMaxTokens * kChunk + 1023) / 1024 * 1024;
+
 template <int GPU>
 struct StepSmem {
-  static constexpr size_t kRing = (size_t)kWarps * kRingSlots * Geom<GPU>::kUnitBytes;
-  static constexpr size_t kBars = (size_t)2 * kWarps * kRingSlots * sizeof(uint64_t);
+  static constexpr int kSlots = Geom<GPU>::kStepSlots;
+  static constexpr size_t kRing = (size_t)kWarps * kSlots * Geom<GPU>::kUnitBytes;
+  static constexpr size_t kBars = (size_t)2 * kWarps * kSlots * sizeof(uint64_t);
   // attention item area (AttnSmem), also the normalised rows
-  static constexpr size_t kQ = 96 * 1024;
+  static constexpr size_t kQ = kAttnArea;
   static constexpr size_t kFixed = kRing + kBars + kQ;  // + the op table (4L entries)
   static size_t total(int n_layers) { return kFixed + (size_t)4 * n_layers * sizeof(OpDesc); }
 };
@@ -746,7 +753,8 @@ template <int NT, int GPU, int DPL>
 __global__ void __launch_bounds__(kBlockThreads, 1) step_kernel(const __grid_constant__ StepKernelArgs a) {
   extern __shared__ __align__(128) uint8_t smem[];
   __shared__ GemvPhase s_gp[4];            // per projection kind: q|k|v, o, gate|up, down
-  __shared__ WarpRing<GPU> s_ring[kWarps];  // each consumer warp's ring, between phases
+  constexpr int kSlots = Geom<GPU>::kStepSlots;
+  __shared__ WarpRing<GPU, kSlots> s_ring[kWarps];  // each consumer warp's ring, between phases
   __shared__ AttnView s_av;
   __shared__ StepParams s_sp;
   __shared__ const uint16_t* s_rowp[kMaxTokens];  // the step's fp16 input rows
@@ -754,13 +762,13 @@ __global__ void __launch_bounds__(kBlockThreads, 1) step_kernel(const __grid_con
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   uint8_t* rings = smem;
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + SS::kRing);
-  uint64_t* empty = full + kWarps * kRingSlots;
+  uint64_t* empty = full + kWarps * kSlots;
   uint8_t* att_area = smem + SS::kRing + SS::kBars;
   static_assert(AttnSmem<DPL>::kBytes <= SS::kQ, "attention area too small");
   OpDesc* s_ops = reinterpret_cast<OpDesc*>(smem + SS::kFixed);
   for (int i = threadIdx.x; i < 4 * a.L; i += kBlockThreads) s_ops[i] = a.ops[i];
   if (threadIdx.x == 0) {
-    ring_init_barriers(full, empty, kWarps * kRingSlots);
+    ring_init_barriers(full, empty, kWarps * kSlots);
     if (blockIdx.x == 0) a.phase_clock[0] = globaltimer();
   }
   prologue_params(a.pro, &s_sp, s_rowp);  // ends with a block-wide barrier
@@ -777,25 +785,25 @@ __global__ void __launch_bounds__(kBlockThreads, 1) step_kernel(const __grid_con
     }
     return;
   }
-  if (warp == kWarps) {  // the producer warp
-    ring_producer<GPU>(s_ops, 4 * a.L, blockIdx.x, gridDim.x, kWarps, rings, full, empty, kRingSlots == 4 ? 2 : 1,
-                       a.status, kProducerLimit, lane);
+  if (!kSelfRefill && warp == kWarps) {  // the producer warp
+    ring_producer<GPU, kSlots>(s_ops, 4 * a.L, blockIdx.x, gridDim.x, kWarps, rings, full, empty, a.status,
+                               kProducerLimit, lane);
     return;
   }
   // ---- consumer warps from here on: CTA barriers are cbar() ----
   const StepParams* sp = &s_sp;
   const int M = sp->M;
   GridBarrier gb{a.barrier, a.barrier_base, a.status, a.phase_clock, 0, 0, a.debug_skip_arrival, a.wait_limit};
-  if (lane == 0) {
-    WarpRing<GPU> r;
-    r.ring = rings + (size_t)warp * kRingSlots * Geom<GPU>::kUnitBytes;
-    r.full = full + warp * kRingSlots;
-    r.empty = empty + warp * kRingSlots;
-    r.slot_mask = kRingSlots - 1;
-    r.slot_shift = kRingSlots == 4 ? 2 : 1;
+  {
+    WarpRing<GPU, kSlots> r;
+    r.ring = rings + (size_t)warp * kSlots * Geom<GPU>::kUnitBytes;
+    r.full = full + warp * kSlots;
+    r.empty = empty + warp * kSlots;
     r.n_used = 0;
     r.timed_out = false;
-    s_ring[warp] = r;
+    if (kSelfRefill) r.start(s_ops, 4 * a.L, blockIdx.x * kWarps + warp, gridDim.x * kWarps, lane);
+    if (lane == 0) s_ring[warp] = r;
+    __syncwarp();
   }
   // Each CTA normalises the whole hidden state for itself; when the M rows
   // fit, it keeps them in the attention area (idle during the q|k|v and
@@ -873,7 +881,7 @@ __global__ void __launch_bounds__(kBlockThreads, 1) step_kernel(const __grid_con
 
   const int g = blockIdx.x * kWarps + warp, nw = gridDim.x * kWarps;
   const int gt = blockIdx.x * kThreads + threadIdx.x, gs = gridDim.x * kThreads;
-  auto gemv = [&](int op) { gemv_phase<NT, GPU>(&s_ring[warp], &s_ops[op], &s_gp[op & 3], g, nw, lane); };
+  auto gemv = [&](int op) { gemv_phase<NT, GPU, kSlots>(&s_ring[warp], &s_ops[op], &s_gp[op & 3], g, nw, lane); };
   const int qkv_rows = (a.Hq + 2 * a.Hkv) * a.d;
 
   for (int l = 0; l < a.L; ++l) {

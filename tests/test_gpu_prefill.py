@@ -103,7 +103,7 @@ def test_tiny_prefill_with_masked_holes_and_second_row(tiny):
     # the oracle's step for request 1 alone: row 0 takes no new token, so
     # run it on a one-row copy of row 1
     o1 = OracleEngine(shape, w, 1, cap)
-    prefill(o1, shape, SEED + 1, 0, 50)
+    prefill(o1, shape, SEED + 1, 0, 50, src_row=1)
     want = o1.step([S], pos, mask, hidden_in=h)
     assert_fixed_bar(got, want, "tiny prefill row 1 with holes")
     assert g.length(1) == 50 + S and g.length(0) == 30
