@@ -34,7 +34,7 @@ __global__ void __launch_bounds__(kBlock, 1) gemv_kernel(const __grid_constant__
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + (size_t)kW * kSlots * Geom<GPU>::kUnitBytes);
   uint64_t* empty = full + kW * kSlots;
   if (threadIdx.x == 0) {
-    s_op[0] = OpDesc{a.units, a.n_rb, a.upr};
+    s_op[0] = OpDesc{a.units, a.n_rb, a.upr, 0};
     GemvPhase p{};
     p.act = a.act;
     p.act_ld = a.act_ld;

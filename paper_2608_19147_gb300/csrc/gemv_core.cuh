@@ -97,7 +97,21 @@ __device__ __forceinline__ int ld_acquire_s32(const int* p) {
 __device__ __forceinline__ void red_add_s64(long long* p, long long v) {
   asm volatile("red.relaxed.gpu.global.add.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
 }
-__device__ __forceinline__ long long to_fixed(float v) { return __float2ll_rn(v * kFixOne); }
+// round(t) as a 64-bit integer, exact (ties to even) for |t| < 2^52, without
+// the 64-bit conversion instructions (a slow path on this GPU).  Split
+// t = h 2^31 + r with h = rint(t 2^-31), taken from the bits of a float sum
+// with 1.5 2^23 (exact while |t 2^-31| < 2^22); r = t - h 2^31 is exact in
+// fp32: for |t| < 2^30, h = 0 and r = t; otherwise t is a multiple of 2^7
+// and |r| <= 2^30, so r has at most 23 significant bits.  One 32-bit
+// conversion rounds r.
+__device__ __forceinline__ long long f2fix(float t) {
+  constexpr float kMagic = 12582912.0f;  // 1.5 * 2^23
+  const float y = __fadd_rn(t * 4.656612873077393e-10f, kMagic);  // rint(t 2^-31) + 1.5 2^23
+  const int h = __float_as_int(y) - __float_as_int(kMagic);
+  const float r = fmaf(__fsub_rn(y, kMagic), -2147483648.0f, t);
+  return (static_cast<long long>(h) << 31) + static_cast<long long>(__float2int_rn(r));
+}
+__device__ __forceinline__ long long to_fixed(float v) { return f2fix(v * kFixOne); }
 // value = v * 2^-32 with v = hi * 2^32 + lo (lo unsigned): hi + lo * 2^-32
 // in fp32 from two 32-bit conversions (int64 conversions are a slow path).
 // hi is exact (|hi| < 2^24); the result is within one fp32 ulp of the exact
@@ -121,6 +135,27 @@ __device__ __forceinline__ bool mbar_test_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
+// Units [b, e) of warp g's run of op (OpDesc::q).  q > 0: row-block rb
+// belongs to CTA rb / (kCtaWarps / q); its warps (rb % (kCtaWarps / q)) q + i,
+// i < q, take K ranges i of ceil(upr / q) units.
+__device__ __forceinline__ void run_range(const OpDesc& op, int g, int nw, int& b, int& e) {
+  if (op.q == 0) {
+    const int T = op.n_rb * op.upr;
+    b = part_start(T, g, nw);
+    e = part_start(T, g + 1, nw);
+    return;
+  }
+  const int cta = g / kCtaWarps, w = g - cta * kCtaWarps;
+  const int rb = cta * (kCtaWarps / op.q) + w / op.q, i = w % op.q;
+  const int R = (op.upr + op.q - 1) / op.q;
+  const int k0 = min(i * R, op.upr), k1 = min(k0 + R, op.upr);
+  b = e = 0;
+  if (rb < op.n_rb) {
+    b = rb * op.upr + k0;
+    e = rb * op.upr + k1;
+  }
+}
+
 // One warp's view of the weight stream: the warp's run of every projection
 // of the launch, in order (ops[0 .. n_ops)).
 struct StreamCursor {
@@ -130,9 +165,7 @@ struct StreamCursor {
   const uint8_t* src;
 
   __device__ __forceinline__ void open(int o, int UB) {
-    const int T = ops[o].n_rb * ops[o].upr;
-    u = part_start(T, g, nw);
-    end = part_start(T, g + 1, nw);
+    run_range(ops[o], g, nw, u, end);
     src = ops[o].units + (size_t)u * UB;
   }
   __device__ __forceinline__ void init(const OpDesc* ops_, int n_ops_, int g_, int nw_, int UB) {
@@ -380,6 +413,7 @@ struct GemvPhase {
   EpiArgs ep;
   int kv_rb_q, kv_rb_k;  // EPI_QKV: row-blocks per q head group, first k and v row-block (see kv_head_of)
   int kv_rb_v, kv_rb_per_head;
+  float* part;           // OpDesc::q > 0: the CTA's partial sums (shared memory), see swiglu_cta_write
 };
 
 // Loads the B fragments of input unit ku for tokens gid (and gid + 8).
@@ -452,6 +486,71 @@ static __device__ __noinline__ void finish_store(const GemvPhase* pp, int rb, in
   if (lane == 0) __stcg(p.ep.cnt + rb, 0);
 }
 
+// ---------------------------------------------------------------------------
+// Gate|up with OpDesc::q > 0: row-block rb is reduced inside its CTA.  Each
+// of its q warps writes its sums, in natural scale, to its own slot of the
+// CTA's partial area (fp32 [kCtaWarps][kGuCtaTokens][64]); after a named
+// barrier of the q warps (id 2 + group) they add the q slots in a fixed order
+// and write h = silu(gate) * up as fp16.  No global atomics; the result does
+// not depend on arrival order.
+// ---------------------------------------------------------------------------
+constexpr int kGuCtaTokens = 5;  // tokens up to which the whole-step kernel reduces gate|up this way
+
+template <int NT>
+__device__ __forceinline__ void swiglu_cta_write(const GemvPhase& p, const float (&tot)[4][NT][4], int w, int lane) {
+  const int gid = lane >> 2, tig = lane & 3;
+  float* slot = p.part + (size_t)w * kGuCtaTokens * kRowsPerBlock;
+#pragma unroll
+  for (int rt = 0; rt < 4; ++rt)
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+      for (int c = 0; c < 2; ++c) {
+        const int m = nt * 8 + 2 * tig + c;
+        if (m < p.M) {
+          slot[m * kRowsPerBlock + rt * 16 + gid] = tot[rt][nt][c] * 16777216.0f;        // 2^24
+          slot[m * kRowsPerBlock + rt * 16 + gid + 8] = tot[rt][nt][2 + c] * 1048576.0f;  // 2^20
+        }
+      }
+}
+
+// After the group's barrier: gate row 16 t + r and up row 16 t + r + 8 of the
+// row-block give h index 32 rb + 8 t + r (the unit row order of gate|up).
+static __device__ __forceinline__ void swiglu_cta_finish(const GemvPhase* pp, int rb, int q, int w, int lane) {
+  const GemvPhase& p = *pp;
+  const int grp0 = w - w % q;
+  const float* base = p.part + (size_t)grp0 * kGuCtaTokens * kRowsPerBlock;
+  for (int it = (w - grp0) * 32 + lane; it < 32 * p.M; it += q * 32) {
+    const int m = it >> 5, jl = it & 31;
+    const int Rg = 16 * (jl >> 3) + (jl & 7);
+    // each partial in fixed point as the atomic path adds it (exact integer
+    // sums): the same bits for any token count
+    long long gs = 0, us = 0;
+    for (int i = 0; i < q; ++i) {
+      const float* sl = base + (size_t)i * kGuCtaTokens * kRowsPerBlock + m * kRowsPerBlock;
+      gs += f2fix(sl[Rg] * kFixOne);
+      us += f2fix(sl[Rg + 8] * kFixOne);
+    }
+    const float gv = fixed_to_f32(gs), uv = fixed_to_f32(us);
+    const int j = 32 * rb + jl;
+    if (j < p.ep.dims.F) p.ep.h[(size_t)m * p.ep.h_ld + j] = f2h(silu(gv) * uv);
+  }
+}
+
+// Whole end of a q > 0 run (called by every warp whose group owns a row-block,
+// empty K range or not).
+template <int NT>
+__device__ __forceinline__ void swiglu_cta_end(const GemvPhase* pp, const OpDesc* op, const float (&tot)[4][NT][4],
+                                               int g, int lane) {
+  const int q = op->q;
+  const int cta = g / kCtaWarps, w = g - cta * kCtaWarps;
+  const int rb = cta * (kCtaWarps / q) + w / q;
+  if (rb >= op->n_rb) return;  // the whole group has nothing (same test for each of its warps)
+  swiglu_cta_write<NT>(*pp, tot, w, lane);
+  named_bar_sync(2 + w / q, q * 32);
+  swiglu_cta_finish(pp, rb, q, w, lane);
+}
+
 // End of one row-block segment (units of row-block rb) of a warp's run: add
 // the sums to the accumulator, then count the units (see EpiArgs).
 template <int NT>
@@ -470,9 +569,9 @@ __device__ __forceinline__ void segment_end(const GemvPhase* pp, const float (&t
         const int m = nt * 8 + 2 * tig + c;
         if (m < p.M) {
           long long* a = p.ep.acc + (size_t)m * p.ep.acc_ld + rb * kRowsPerBlock + rt * 16 + gid;
-          if (rb * kRowsPerBlock + rt * 16 + gid < rows) red_add_s64(a, __float2ll_rn(tot[rt][nt][c] * kTotScaleLo));
+          if (rb * kRowsPerBlock + rt * 16 + gid < rows) red_add_s64(a, f2fix(tot[rt][nt][c] * kTotScaleLo));
           if (rb * kRowsPerBlock + rt * 16 + gid + 8 < rows)
-            red_add_s64(a + 8, __float2ll_rn(tot[rt][nt][2 + c] * kTotScaleHi));
+            red_add_s64(a + 8, f2fix(tot[rt][nt][2 + c] * kTotScaleHi));
         }
       }
   if (kind == EPI_RESID) return;
@@ -495,23 +594,30 @@ __device__ __forceinline__ void segment_end(const GemvPhase* pp, const float (&t
 }
 
 // One projection for one warp: consume the warp's run of units from its ring
-// (which the producer fills in the same order) and hand on each row-block
-// segment of it.
-//
-// Not inlined: the step's four projections run this one copy of the code, so
-// it stays in the instruction cache.  The ring state and the phase arguments
-// live in shared memory (ring_io, pp): nothing crosses the call through the
-// stack, whose local memory would miss the small L1 left next to the weight
-// rings.
+// (which is filled in the same order) and hand on each row-block segment of
+// it.  Inlined at one call site (the whole-step kernel's layer loop, which
+// keeps the ring in registers), so no call boundary spills the caller's
+// registers.
 template <int NT, int GPU, int S>
-__device__ __noinline__ void gemv_phase(WarpRing<GPU, S>* ring_io, const OpDesc* op, const GemvPhase* pp, int g, int nw,
-                                        int lane) {
-  WarpRing<GPU, S> ring = *ring_io;
+__device__ __forceinline__ void gemv_run(WarpRing<GPU, S>& ring, const OpDesc* op, const GemvPhase* pp, int g, int nw,
+                                         int lane) {
   const GemvPhase& p = *pp;
   const int upr = op->upr;
-  const int T = op->n_rb * upr;
-  const int wb = part_start(T, g, nw), we = part_start(T, g + 1, nw);
-  if (wb >= we) return;
+  int wb, we;
+  run_range(*op, g, nw, wb, we);
+  if (wb >= we) {
+    if (op->q > 0 && p.M <= kGuCtaTokens) {  // a group member without units still adds (zero) sums
+      float zero[4][NT][4];
+#pragma unroll
+      for (int rt = 0; rt < 4; ++rt)
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+          for (int e = 0; e < 4; ++e) zero[rt][nt][e] = 0.f;
+      swiglu_cta_end<NT>(pp, op, zero, g, lane);
+    }
+    return;
+  }
   const uint16_t* actp = p.act;
   const uint32_t acts = p.act_s;
   const int act_ld = acts ? p.act_s_ld : p.act_ld, M = p.M;
@@ -544,8 +650,19 @@ __device__ __noinline__ void gemv_phase(WarpRing<GPU, S>* ring_io, const OpDesc*
       if (!ring.timed_out) mma_unit<NT, GPU>(U, cur, tot, lane);
       ring.release(lane);
     }
-    segment_end<NT>(pp, tot, rb, seg_end - seg_begin, upr, lane);
+    if (op->q > 0 && p.M <= kGuCtaTokens)
+      swiglu_cta_end<NT>(pp, op, tot, g, lane);  // the run is one whole segment
+    else
+      segment_end<NT>(pp, tot, rb, seg_end - seg_begin, upr, lane);
   }
+}
+
+// gemv_run with the ring state in shared memory (the standalone kernel).
+template <int NT, int GPU, int S>
+__device__ __noinline__ void gemv_phase(WarpRing<GPU, S>* ring_io, const OpDesc* op, const GemvPhase* pp, int g, int nw,
+                                        int lane) {
+  WarpRing<GPU, S> ring = *ring_io;
+  gemv_run<NT, GPU, S>(ring, op, pp, g, nw, lane);
   __syncwarp();
   if (lane == 0) *ring_io = ring;
   __syncwarp();

@@ -232,6 +232,12 @@ struct PrologueArgs {
 struct OpDesc {
   const uint8_t* units;
   int n_rb, upr;
+  // Work split.  q = 0: the unit stream is cut into one contiguous run per
+  // warp of the grid.  q > 0 (whole-step kernel, gate|up): row-block rb
+  // belongs to one CTA, whose q warps take its units in q contiguous K
+  // ranges and reduce them in shared memory (set only when every row-block
+  // of the projection finds its CTA in one round).
+  int q;
 };
 
 // Arguments of the whole-step kernel (step_kernel.cu).
@@ -267,11 +273,21 @@ struct StepKernelArgs {
   int* exit_count;           // CTAs finished in this launch (zero between launches; the last resets it)
   int debug_skip_arrival;    // test knob: >= 0 makes CTA 1 skip that grid barrier's arrival
   unsigned wait_limit;       // polls before a cross-CTA wait gives up
+  int gu_part;               // 1: shared memory holds the gate|up partial sums (OpDesc::q may be used)
 };
 // One-time attribute setup of the step kernel variants for a group size and
 // head dim; number of grid barriers per step; launch (cooperative, one CTA
 // per SM).
 cudaError_t step_setup(int group, int head_dim);
+// Warps per row-block for the shared-memory reduction of a gate|up
+// projection of n_rb row-blocks of upr units on `grid` CTAs (0: the
+// grid-wide split), when the kernel's shared memory for L layers leaves room
+// for the partial sums.
+int step_gu_split(int n_rb, int upr, int grid, int group, int L);
+// Token count up to which the whole-step kernel uses that reduction.
+int step_gu_cta_tokens();
+// Whether the kernel's shared memory for L layers has room for the partial sums.
+bool step_gu_part_fits(int group, int L);
 int step_barriers(int n_layers);
 cudaError_t launch_step(const StepKernelArgs& a, int nt, int group, int grid, cudaStream_t s);
 size_t step_attention_part_floats(int B, int Hkv, int n_chunks, int G, int d);

@@ -414,7 +414,12 @@ int shard_create(const shard_config* cfg, const shard_weights_host* w, shard_t* 
   CUDA_TRY(cudaMemset(sh->exit_count, 0, sizeof(int)));
   {
     std::vector<OpDesc> od(sh->ops.size());
-    for (size_t i = 0; i < od.size(); ++i) od[i] = OpDesc{sh->ops[i].units, sh->ops[i].n_rb, sh->ops[i].upr};
+    for (size_t i = 0; i < od.size(); ++i) {
+      const auto& o = sh->ops[i];
+      // gate|up (op 2 of each layer): shared-memory reduction when it fits
+      const int q = i % 4 == 2 ? step_gu_split(o.n_rb, o.upr, sh->num_sms, sh->cfg.group, sh->L) : 0;
+      od[i] = OpDesc{o.units, o.n_rb, o.upr, q};
+    }
     CUDA_TRY(cudaMalloc(&sh->ops_dev, sizeof(OpDesc) * od.size()));
     CUDA_TRY(cudaMemcpy(sh->ops_dev, od.data(), sizeof(OpDesc) * od.size(), cudaMemcpyHostToDevice));
   }
@@ -796,6 +801,7 @@ static int step_impl(shard_t sh, kvstate_t st, const uint16_t* hidden_in, const 
   ka.status = sh->status;
   ka.debug_skip_arrival = sh->debug_skip_arrival;
   ka.wait_limit = sh->wait_limit;
+  ka.gu_part = step_gu_part_fits(sh->cfg.group, sh->L) ? 1 : 0;
   ka.barrier = sh->barrier;
   ka.barrier_base = sh->barrier_base;
   ka.phase_clock = sh->phase_clock;

@@ -24,6 +24,8 @@
 // proceeds (the step's results are then reported invalid) instead of hanging.
 #include <type_traits>
 
+#include <algorithm>
+
 #include "gemv_core.cuh"
 
 namespace shard {
@@ -34,7 +36,6 @@ constexpr int kThreads = kWarps * 32;       // consumer threads
 constexpr int kBlockThreads = kThreads + (kSelfRefill ? 0 : 32);  // + the producer warp, if any
 constexpr int kChunk = kAttnChunk;  // most cache entries per attention item (kChunk / 32 per lane)
 constexpr bool kNormInSmem = true;   // normalised activations in shared memory when they fit
-constexpr int kNormCache = 6;        // float4 pieces of the first row a thread keeps between the norm's passes
 // Polls of a busy slot before the producer gives up: a slot may legitimately
 // stay busy while its consumer works through a whole attention phase, so this
 // bound is fixed and far above any step's length.
@@ -54,7 +55,11 @@ struct StepSmem {
   // attention item area (AttnSmem), also the normalised rows
   static constexpr size_t kQ = kAttnArea;
   static constexpr size_t kFixed = kRing + kBars + kQ;  // + the op table (4L entries)
-  static size_t total(int n_layers) { return kFixed + (size_t)4 * n_layers * sizeof(OpDesc); }
+  // gate|up partial sums of the shared-memory reduction (swiglu_cta_write)
+  static constexpr size_t kPart = (size_t)kWarps * kGuCtaTokens * kRowsPerBlock * sizeof(float);
+  __host__ __device__ static size_t ops_bytes(int n_layers) { return ((size_t)4 * n_layers * sizeof(OpDesc) + 15) / 16 * 16; }
+  static size_t total(int n_layers) { return kFixed + ops_bytes(n_layers); }
+  static size_t total_with_part(int n_layers) { return total(n_layers) + kPart; }
 };
 
 // Barrier among the consumer warps of a CTA (the producer warp runs on its own).
@@ -230,8 +235,8 @@ __device__ __noinline__ void prologue_work(const PrologueArgs& a, const StepPara
     const uint2 v = *reinterpret_cast<const uint2*>(rowp[m] + k);
     const float2 f01 = h2f2(v.x), f23 = h2f2(v.y);
     longlong2* dst = reinterpret_cast<longlong2*>(X + (size_t)m * a.H + k);
-    dst[0] = make_longlong2(__float2ll_rn(f01.x * kFixOne), __float2ll_rn(f01.y * kFixOne));
-    dst[1] = make_longlong2(__float2ll_rn(f23.x * kFixOne), __float2ll_rn(f23.y * kFixOne));
+    dst[0] = make_longlong2(to_fixed(f01.x), to_fixed(f01.y));
+    dst[1] = make_longlong2(to_fixed(f23.x), to_fixed(f23.y));
   }
 }
 
@@ -243,9 +248,9 @@ __device__ __noinline__ void prologue_work(const PrologueArgs& a, const StepPara
 // fixed order, so every CTA gets the same r), then the scaled rows; the first
 // row's pieces stay in registers between the passes.  H is a multiple of 4.
 // ---------------------------------------------------------------------------
-template <bool kFromX>
-__device__ __forceinline__ float4 norm_load(const long long* X, const uint16_t* const* rowp, int H, int m, int k) {
-  if (kFromX) {
+__device__ __forceinline__ float4 norm_load(bool from_x, const long long* X, const uint16_t* const* rowp, int H, int m,
+                                            int k) {
+  if (from_x) {
     const longlong2* p = reinterpret_cast<const longlong2*>(X + (size_t)m * H + k);
     const longlong2 a = __ldcg(p), b = __ldcg(p + 1);
     return make_float4(fixed_to_f32(a.x), fixed_to_f32(a.y), fixed_to_f32(b.x), fixed_to_f32(b.y));
@@ -256,38 +261,55 @@ __device__ __forceinline__ float4 norm_load(const long long* X, const uint16_t* 
   }
 }
 
-template <bool kFromX>
-__device__ __noinline__ void rmsnorm_cta(const long long* X, const uint16_t* const* rowp, int H, const uint16_t* w,
-                                         float eps, uint16_t* out, int out_ld, int M) {
+// kP pieces (float4) per row and thread are held in registers (the rest of a
+// longer row is streamed).  Rows go kR at a time, every piece of the kR rows
+// requested at once (one memory round trip per batch; the norm weights come
+// with the first).  When all M rows fit in one batch they stay in registers
+// for the second pass, so X is read once.
+template <int kP, int kR>
+__device__ __forceinline__ void rmsnorm_rows(bool from_x, const long long* X, const uint16_t* const* rowp, int H,
+                                             const uint16_t* w, float eps, uint16_t* out, int out_ld, int M) {
   __shared__ float s_part[kWarps][kMaxTokens];
   __shared__ float s_r[kMaxTokens];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int H4 = H / 4;
-  float4 keep[kNormCache];
-  for (int m = 0; m < M; ++m) {
-    float t = 0.f;
-    if (m == 0) {
+  uint2 wv[kP];
+  float4 v[kR][kP];
 #pragma unroll
-      for (int i = 0; i < kNormCache; ++i) {
+  for (int i = 0; i < kP; ++i) {
+    const int c = tid + i * kThreads;
+    wv[i] = c < H4 ? *reinterpret_cast<const uint2*>(w + 4 * c) : make_uint2(0, 0);
+  }
+  auto load_batch = [&](int m0) {
+#pragma unroll
+    for (int h = 0; h < kR; ++h)
+#pragma unroll
+      for (int i = 0; i < kP; ++i) {
         const int c = tid + i * kThreads;
-        keep[i] = c < H4 ? norm_load<kFromX>(X, rowp, H, 0, 4 * c) : make_float4(0.f, 0.f, 0.f, 0.f);
+        v[h][i] = c < H4 && m0 + h < M ? norm_load(from_x, X, rowp, H, m0 + h, 4 * c) : make_float4(0.f, 0.f, 0.f, 0.f);
       }
+  };
+  for (int m0 = 0; m0 < M; m0 += kR) {
+    load_batch(m0);
+    float t[kR];
 #pragma unroll
-      for (int i = 0; i < kNormCache; ++i)
-        t += keep[i].x * keep[i].x + keep[i].y * keep[i].y + keep[i].z * keep[i].z + keep[i].w * keep[i].w;
-      for (int c = tid + kNormCache * kThreads; c < H4; c += kThreads) {
-        const float4 v = norm_load<kFromX>(X, rowp, H, 0, 4 * c);
-        t += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
-      }
-    } else {
-      for (int c = tid; c < H4; c += kThreads) {
-        const float4 v = norm_load<kFromX>(X, rowp, H, m, 4 * c);
-        t += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
-      }
+    for (int h = 0; h < kR; ++h) {
+      t[h] = 0.f;
+#pragma unroll
+      for (int i = 0; i < kP; ++i)
+        t[h] += v[h][i].x * v[h][i].x + v[h][i].y * v[h][i].y + v[h][i].z * v[h][i].z + v[h][i].w * v[h][i].w;
+      if (m0 + h < M)
+        for (int c = tid + kP * kThreads; c < H4; c += kThreads) {
+          const float4 u = norm_load(from_x, X, rowp, H, m0 + h, 4 * c);
+          t[h] += u.x * u.x + u.y * u.y + u.z * u.z + u.w * u.w;
+        }
     }
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
-    if (lane == 0) s_part[warp][m] = t;
+    for (int h = 0; h < kR; ++h) {
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) t[h] += __shfl_xor_sync(0xffffffffu, t[h], o);
+      if (lane == 0 && m0 + h < M) s_part[warp][m0 + h] = t[h];
+    }
   }
   cbar();
   if (tid < M) {
@@ -296,28 +318,41 @@ __device__ __noinline__ void rmsnorm_cta(const long long* X, const uint16_t* con
     s_r[tid] = rsqrtf(t / H + eps);
   }
   cbar();
-  for (int m = 0; m < M; ++m) {
-    const float r = s_r[m];
-    auto emit = [&](int c, float4 v) {
-      const uint2 wv = *reinterpret_cast<const uint2*>(w + 4 * c);
-      const float2 w01 = h2f2(wv.x), w23 = h2f2(wv.y);
-      uint2 o;
-      o.x = pack_h2(v.x * r * w01.x, v.y * r * w01.y);
-      o.y = pack_h2(v.z * r * w23.x, v.w * r * w23.y);
-      *reinterpret_cast<uint2*>(out + (size_t)m * out_ld + 4 * c) = o;
-    };
-    if (m == 0) {
+  for (int m0 = 0; m0 < M; m0 += kR) {
+    if (M > kR) load_batch(m0);  // else the one batch is still in registers
 #pragma unroll
-      for (int i = 0; i < kNormCache; ++i) {
+    for (int h = 0; h < kR; ++h) {
+      const int m = m0 + h;
+      if (m >= M) break;
+      const float r = s_r[m];
+      auto emit = [&](int c, float4 x, uint2 wq) {
+        const float2 w01 = h2f2(wq.x), w23 = h2f2(wq.y);
+        uint2 o;
+        o.x = pack_h2(x.x * r * w01.x, x.y * r * w01.y);
+        o.y = pack_h2(x.z * r * w23.x, x.w * r * w23.y);
+        *reinterpret_cast<uint2*>(out + (size_t)m * out_ld + 4 * c) = o;
+      };
+#pragma unroll
+      for (int i = 0; i < kP; ++i) {
         const int c = tid + i * kThreads;
-        if (c < H4) emit(c, keep[i]);
+        if (c < H4) emit(c, v[h][i], wv[i]);
       }
-      for (int c = tid + kNormCache * kThreads; c < H4; c += kThreads) emit(c, norm_load<kFromX>(X, rowp, H, 0, 4 * c));
-    } else {
-      for (int c = tid; c < H4; c += kThreads) emit(c, norm_load<kFromX>(X, rowp, H, m, 4 * c));
+      for (int c = tid + kP * kThreads; c < H4; c += kThreads)
+        emit(c, norm_load(from_x, X, rowp, H, m, 4 * c), *reinterpret_cast<const uint2*>(w + 4 * c));
     }
   }
   cbar();
+}
+
+// Rows of up to 3 pieces per thread (H <= 4608) go three at a time; longer
+// rows two at a time with 6 pieces in registers.  from_x: the residual
+// stream, else the step's fp16 input rows (before the first layer).
+__device__ __forceinline__ void rmsnorm_cta(bool from_x, const long long* X, const uint16_t* const* rowp, int H,
+                                            const uint16_t* w, float eps, uint16_t* out, int out_ld, int M) {
+  if (H / 4 <= 3 * kThreads)
+    rmsnorm_rows<3, 3>(from_x, X, rowp, H, w, eps, out, out_ld, M);
+  else
+    rmsnorm_rows<6, 2>(from_x, X, rowp, H, w, eps, out, out_ld, M);
 }
 
 // ---------------------------------------------------------------------------
@@ -482,7 +517,7 @@ __device__ __forceinline__ void attn_load_queries(const AttnView& a, const StepP
 // and sum, each lane DPL output dims.  The running result is rescaled when a
 // batch raises the maximum (online softmax).
 template <int DPL>
-__device__ __noinline__ void attn_merge_warp(const AttnView* ap, const StepParams* sp, int b, int hk, int qi, int lane) {
+__device__ __forceinline__ void attn_merge_warp(const AttnView* ap, const StepParams* sp, int b, int hk, int qi, int lane) {
   const AttnView& a = *ap;
   constexpr int d = 32 * DPL;
   constexpr int kMergeBatch = 16;
@@ -553,7 +588,7 @@ __device__ __noinline__ void attn_merge_warp(const AttnView* ap, const StepParam
 //      every CTA has at most one item, the CTA that counts the last chunk
 //      merges at once.
 template <int DPL>
-__device__ __noinline__ void attn_item_cta(const AttnView* ap, int layer, const StepParams* sp, int b, int hk, int c,
+__device__ __forceinline__ void attn_item_cta(const AttnView* ap, int layer, const StepParams* sp, int b, int hk, int c,
                                            uint8_t* area, int* status) {
   const AttnView& a = *ap;
   uint16_t* kpool = a.kpool + (size_t)layer * a.layer_stride;
@@ -737,7 +772,7 @@ __device__ __noinline__ void attn_item_cta(const AttnView* ap, int layer, const 
 // own items: wait until every chunk is counted (bounded), merge the queries
 // (one warp each), reset the count.
 template <int DPL>
-__device__ __noinline__ void attn_merge_cta(const AttnView* ap, const StepParams* sp, int b, int hk, int* status) {
+__device__ __forceinline__ void attn_merge_cta(const AttnView* ap, const StepParams* sp, int b, int hk, int* status) {
   const AttnView& a = *ap;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int L = sp->req_len[b], nb = sp->req_tok0[b + 1] - sp->req_tok0[b];
@@ -754,7 +789,6 @@ __global__ void __launch_bounds__(kBlockThreads, 1) step_kernel(const __grid_con
   extern __shared__ __align__(128) uint8_t smem[];
   __shared__ GemvPhase s_gp[4];            // per projection kind: q|k|v, o, gate|up, down
   constexpr int kSlots = Geom<GPU>::kStepSlots;
-  __shared__ WarpRing<GPU, kSlots> s_ring[kWarps];  // each consumer warp's ring, between phases
   __shared__ AttnView s_av;
   __shared__ StepParams s_sp;
   __shared__ const uint16_t* s_rowp[kMaxTokens];  // the step's fp16 input rows
@@ -794,17 +828,14 @@ __global__ void __launch_bounds__(kBlockThreads, 1) step_kernel(const __grid_con
   const StepParams* sp = &s_sp;
   const int M = sp->M;
   GridBarrier gb{a.barrier, a.barrier_base, a.status, a.phase_clock, 0, 0, a.debug_skip_arrival, a.wait_limit};
-  {
-    WarpRing<GPU, kSlots> r;
-    r.ring = rings + (size_t)warp * kSlots * Geom<GPU>::kUnitBytes;
-    r.full = full + warp * kSlots;
-    r.empty = empty + warp * kSlots;
-    r.n_used = 0;
-    r.timed_out = false;
-    if (kSelfRefill) r.start(s_ops, 4 * a.L, blockIdx.x * kWarps + warp, gridDim.x * kWarps, lane);
-    if (lane == 0) s_ring[warp] = r;
-    __syncwarp();
-  }
+  // this warp's ring (its state stays in registers for the whole step)
+  WarpRing<GPU, kSlots> ring;
+  ring.ring = rings + (size_t)warp * kSlots * Geom<GPU>::kUnitBytes;
+  ring.full = full + warp * kSlots;
+  ring.empty = empty + warp * kSlots;
+  ring.n_used = 0;
+  ring.timed_out = false;
+  if (kSelfRefill) ring.start(s_ops, 4 * a.L, blockIdx.x * kWarps + warp, gridDim.x * kWarps, lane);
   // Each CTA normalises the whole hidden state for itself; when the M rows
   // fit, it keeps them in the attention area (idle during the q|k|v and
   // gate|up projections) and the projections read them from there.  Rows are
@@ -835,6 +866,7 @@ __global__ void __launch_bounds__(kBlockThreads, 1) step_kernel(const __grid_con
     gp.kv_rb_per_head = a.d / kRowsPerBlock;
     gp.kv_rb_k = a.Hq * a.d / kRowsPerBlock;
     gp.kv_rb_v = (a.Hq + a.Hkv) * a.d / kRowsPerBlock;
+    gp.part = reinterpret_cast<float*>(smem + SS::kFixed + SS::ops_bytes(a.L));
     s_gp[k] = gp;
   }
   if (threadIdx.x == 32) {
@@ -881,20 +913,26 @@ __global__ void __launch_bounds__(kBlockThreads, 1) step_kernel(const __grid_con
 
   const int g = blockIdx.x * kWarps + warp, nw = gridDim.x * kWarps;
   const int gt = blockIdx.x * kThreads + threadIdx.x, gs = gridDim.x * kThreads;
-  auto gemv = [&](int op) { gemv_phase<NT, GPU, kSlots>(&s_ring[warp], &s_ops[op], &s_gp[op & 3], g, nw, lane); };
   const int qkv_rows = (a.Hq + 2 * a.Hkv) * a.d;
 
-  for (int l = 0; l < a.L; ++l) {
-    const uint16_t* nrm = a.norms + (size_t)l * 2 * a.H;
-    // attention block
-    if (l == 0)
-      rmsnorm_cta<false>(a.X, s_rowp, a.H, nrm, a.eps, xn, xn_out_ld, M);
-    else
-      rmsnorm_cta<true>(a.X, s_rowp, a.H, nrm, a.eps, xn, xn_out_ld, M);
-    gemv(4 * l + 0);
-    if (l == 0) gb.wait();            // the prologue's tables and residual are complete
-    else if (xn_smem) cbar();         // the attention items reuse the normalised rows' space
-    {
+  // Phase k of layer l = ph / 4: q|k|v (k = 0), o, gate|up, down.  Every
+  // phase body has one call site, so all of it is inlined into the kernel.
+  for (int ph = 0; ph < 4 * a.L; ++ph) {
+    const int l = ph >> 2, k = ph & 3;
+    if (k == 0 || k == 2) {
+      // RMSNorm of the attention (k = 0) or MLP block; before the first
+      // layer from the step's input rows
+      rmsnorm_cta(ph != 0, a.X, s_rowp, a.H, a.norms + (size_t)l * 2 * a.H + (k == 2 ? a.H : 0), a.eps, xn,
+                  xn_out_ld, M);
+    } else if (k == 1) {
+      // the q|k|v sums and counts are consumed: clear them for the next layer
+      for (int e = gt; e < M * qkv_rows; e += gs) __stcg(a.acc_qkv + e, 0LL);
+      if (blockIdx.x == 0 && threadIdx.x < a.Hkv) __stcg(a.cnt_kv + threadIdx.x, 0);
+    }
+    gemv_run<NT, GPU, kSlots>(ring, &s_ops[ph], &s_gp[k], g, nw, lane);
+    if (k == 0) {
+      if (l == 0) gb.wait();        // the prologue's tables and residual are complete
+      else if (xn_smem) cbar();     // the attention items reuse the normalised rows' space
       int total = 0;
       for (int b = 0; b < sp->B; ++b) total += a.Hkv * n_chunks_of(sp->req_len[b], s_av.cs);
       for (int item = blockIdx.x; item < total; item += gridDim.x) {
@@ -911,17 +949,6 @@ __global__ void __launch_bounds__(kBlockThreads, 1) step_kernel(const __grid_con
       }
     }
     gb.sync();
-    // the q|k|v sums and counts are consumed: clear them for the next layer
-    for (int e = gt; e < M * qkv_rows; e += gs) __stcg(a.acc_qkv + e, 0LL);
-    if (blockIdx.x == 0 && threadIdx.x < a.Hkv) __stcg(a.cnt_kv + threadIdx.x, 0);
-    gemv(4 * l + 1);
-    gb.sync();
-    // MLP block
-    rmsnorm_cta<true>(a.X, s_rowp, a.H, nrm + a.H, a.eps, xn, xn_out_ld, M);
-    gemv(4 * l + 2);
-    gb.sync();
-    gemv(4 * l + 3);
-    gb.sync();
   }
   // hidden_out = fp16(x): one rounding from the exact fixed-point value
   for (int e = gt; e < M * a.H; e += gs) {
@@ -929,7 +956,7 @@ __global__ void __launch_bounds__(kBlockThreads, 1) step_kernel(const __grid_con
     a.pro.hidden_out[e] = __half_as_ushort(__double2half(v));
   }
   if (blockIdx.x == 0 && threadIdx.x < sp->B) a.pro.lens[threadIdx.x] = sp->req_len[threadIdx.x];
-  if (s_ring[warp].timed_out && lane == 0) atomicOr(a.status, ST_WAIT_TIMEOUT);
+  if (ring.timed_out && lane == 0) atomicOr(a.status, ST_WAIT_TIMEOUT);
   // The last CTA to finish hands a nonzero status to the host-mapped mirror,
   // so no copy-engine transfer has to follow the step on the stream.
   cbar();
@@ -946,7 +973,7 @@ cudaError_t launch_t(const StepKernelArgs& a, int grid, cudaStream_t s) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
   cfg.blockDim = dim3(kBlockThreads);
-  cfg.dynamicSmemBytes = StepSmem<GPU>::total(a.L);
+  cfg.dynamicSmemBytes = a.gu_part ? StepSmem<GPU>::total_with_part(a.L) : StepSmem<GPU>::total(a.L);
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeCooperative;
@@ -957,14 +984,61 @@ cudaError_t launch_t(const StepKernelArgs& a, int grid, cudaStream_t s) {
 }
 
 template <int NT, int GPU, int DPL>
+size_t dyn_limit_t() {
+  int dev = 0, optin = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess) return 0;
+  cudaFuncAttributes fa;
+  if (cudaFuncGetAttributes(&fa, step_kernel<NT, GPU, DPL>) != cudaSuccess) return 0;
+  return (size_t)optin > fa.sharedSizeBytes ? (size_t)optin - fa.sharedSizeBytes : 0;
+}
+
+// The largest dynamic shared memory the kernel may take.
+template <int NT, int GPU, int DPL>
 cudaError_t setup_t() {
   return cudaFuncSetAttribute(step_kernel<NT, GPU, DPL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              (int)StepSmem<GPU>::total(64));
+                              (int)dyn_limit_t<NT, GPU, DPL>());
+}
+
+// Dynamic shared memory every kernel of a group size may take (0: unknown group).
+template <int GPU>
+size_t dyn_limit_group() {
+  size_t m = dyn_limit_t<1, GPU, 4>();
+  m = std::min(m, dyn_limit_t<2, GPU, 4>());
+  m = std::min(m, dyn_limit_t<1, GPU, 2>());
+  return std::min(m, dyn_limit_t<2, GPU, 2>());
+}
+
+template <int GPU>
+bool part_fits(int L) {
+  return StepSmem<GPU>::total_with_part(L) <= dyn_limit_group<GPU>();
 }
 
 }  // namespace
 
 int step_barriers(int n_layers) { return 4 * n_layers + 1; }
+
+int step_gu_cta_tokens() { return kGuCtaTokens; }
+
+bool step_gu_part_fits(int group, int L) {
+  if (group == 128) return part_fits<1>(L);
+  if (group == 64) return part_fits<2>(L);
+  if (group == 32) return part_fits<4>(L);
+  return false;
+}
+
+int step_gu_split(int n_rb, int upr, int grid, int group, int L) {
+  if (n_rb < 1 || upr < 1 || grid < 1 || !step_gu_part_fits(group, L)) return 0;
+  const long long nw = (long long)grid * kWarps;
+  const long long even = ((long long)n_rb * upr + nw - 1) / nw;  // most units per warp, grid-wide split
+  int best = 0;
+  for (int q = 1; q <= kWarps; ++q) {
+    if (kWarps % q != 0 || (long long)n_rb * q > nw) continue;  // one round of CTAs
+    const long long most = (upr + q - 1) / q;
+    if (most <= even + std::max(1LL, even / 16)) best = q;  // about as balanced as the grid-wide split
+  }
+  return best;
+}
 
 size_t step_attention_part_floats(int B, int Hkv, int n_chunks, int G, int d) {
   return (size_t)B * Hkv * n_chunks * (kMaxTokens * G) * part_stride(d);
