@@ -43,7 +43,7 @@ namespace shard {
 // (3 per SM sub-partition), or 11 beside the producer (the sub-partition's
 // register file caps 4 warps at 128 registers each).
 constexpr bool kSelfRefill = true;
-constexpr int kRingSlots = 3;  // step kernel: units in flight per consumer warp (group 64 and 128)
+constexpr int kRingSlots = 2;  // step kernel: units in flight per consumer warp (a deeper ring takes the L1 that the norm and attention loads use)
 constexpr int kCtaWarps = kSelfRefill ? 12 : 11;   // consumer warps per CTA of the step kernel
 constexpr int kGemvWarps = kSelfRefill ? 12 : 11;  // consumer warps per CTA of the standalone projection kernel
 

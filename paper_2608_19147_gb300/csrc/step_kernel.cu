@@ -344,6 +344,76 @@ __device__ __forceinline__ void rmsnorm_rows(bool from_x, const long long* X, co
   cbar();
 }
 
+// One row from the residual stream (M = 1, H <= 24 * kThreads) through
+// shared memory: the row's H fixed-point values arrive with bulk copies
+// (`stage`, 16-byte aligned, H * 8 bytes; completion on `bar`, whose phase
+// the caller tracks), so the read runs at copy-engine bandwidth instead of
+// being bounded by each thread's loads in flight; both passes then read
+// shared memory.  The values and the arithmetic are those of rmsnorm_rows.
+__device__ __forceinline__ void rmsnorm_staged(const long long* X, int H, const uint16_t* w, float eps, uint16_t* out,
+                                               long long* stage, uint64_t* bar, uint32_t& phase, int* status) {
+  constexpr int kP = 6;
+  constexpr uint32_t kPiece = 8192;  // bytes per bulk copy
+  __shared__ float s_part[kWarps];
+  __shared__ float s_r;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int H4 = H / 4;
+  if (tid == 0) {
+    // X was written through the generic proxy (made visible by the grid
+    // barrier); the area was last used by generic accesses of this CTA
+    asm volatile("fence.proxy.async;" ::: "memory");
+    const uint32_t bytes = (uint32_t)H * 8u;
+    mbar_arrive_expect_tx(bar, bytes);
+    for (uint32_t off = 0; off < bytes; off += kPiece)
+      bulk_g2s(reinterpret_cast<uint8_t*>(stage) + off, reinterpret_cast<const uint8_t*>(X) + off,
+               bytes - off < kPiece ? bytes - off : kPiece, bar);
+  }
+  uint2 wv[kP];
+#pragma unroll
+  for (int i = 0; i < kP; ++i) {
+    const int c = tid + i * kThreads;
+    wv[i] = c < H4 ? *reinterpret_cast<const uint2*>(w + 4 * c) : make_uint2(0, 0);
+  }
+  if (!mbar_wait(bar, phase) && tid == 0) atomicOr(status, ST_WAIT_TIMEOUT);
+  phase ^= 1u;
+  float4 v[kP];
+  float t = 0.f;
+#pragma unroll
+  for (int i = 0; i < kP; ++i) {
+    const int c = tid + i * kThreads;
+    v[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (c < H4) {
+      const longlong2 a = reinterpret_cast<const longlong2*>(stage)[2 * c];
+      const longlong2 b = reinterpret_cast<const longlong2*>(stage)[2 * c + 1];
+      v[i] = make_float4(fixed_to_f32(a.x), fixed_to_f32(a.y), fixed_to_f32(b.x), fixed_to_f32(b.y));
+    }
+    t += v[i].x * v[i].x + v[i].y * v[i].y + v[i].z * v[i].z + v[i].w * v[i].w;
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+  if (lane == 0) s_part[warp] = t;
+  cbar();
+  if (tid == 0) {
+    float u = 0.f;
+    for (int w8 = 0; w8 < kWarps; ++w8) u += s_part[w8];
+    s_r = rsqrtf(u / H + eps);
+  }
+  cbar();
+  const float r = s_r;
+#pragma unroll
+  for (int i = 0; i < kP; ++i) {
+    const int c = tid + i * kThreads;
+    if (c < H4) {
+      const float2 w01 = h2f2(wv[i].x), w23 = h2f2(wv[i].y);
+      uint2 o;
+      o.x = pack_h2(v[i].x * r * w01.x, v[i].y * r * w01.y);
+      o.y = pack_h2(v[i].z * r * w23.x, v[i].w * r * w23.y);
+      *reinterpret_cast<uint2*>(out + 4 * c) = o;
+    }
+  }
+  cbar();
+}
+
 // Rows of up to 3 pieces per thread (H <= 4608) go three at a time; longer
 // rows two at a time with 6 pieces in registers.  from_x: the residual
 // stream, else the step's fp16 input rows (before the first layer).
@@ -790,6 +860,7 @@ __global__ void __launch_bounds__(kBlockThreads, 1) step_kernel(const __grid_con
   __shared__ GemvPhase s_gp[4];            // per projection kind: q|k|v, o, gate|up, down
   constexpr int kSlots = Geom<GPU>::kStepSlots;
   __shared__ AttnView s_av;
+  __shared__ uint64_t s_nbar;              // the staged RMSNorm's bulk copies
   __shared__ StepParams s_sp;
   __shared__ const uint16_t* s_rowp[kMaxTokens];  // the step's fp16 input rows
   using SS = StepSmem<GPU>;
@@ -802,7 +873,8 @@ __global__ void __launch_bounds__(kBlockThreads, 1) step_kernel(const __grid_con
   OpDesc* s_ops = reinterpret_cast<OpDesc*>(smem + SS::kFixed);
   for (int i = threadIdx.x; i < 4 * a.L; i += kBlockThreads) s_ops[i] = a.ops[i];
   if (threadIdx.x == 0) {
-    ring_init_barriers(full, empty, kWarps * kSlots);
+    mbar_init(&s_nbar, 1);
+    ring_init_barriers(full, empty, kWarps * kSlots);  // ends with the barrier-init fence
     if (blockIdx.x == 0) a.phase_clock[0] = globaltimer();
   }
   prologue_params(a.pro, &s_sp, s_rowp);  // ends with a block-wide barrier
@@ -845,6 +917,12 @@ __global__ void __launch_bounds__(kBlockThreads, 1) step_kernel(const __grid_con
   const bool xn_smem = kNormInSmem && a.Kp_H == a.H && (size_t)M * xn_ld * 2 <= SS::kQ;
   uint16_t* xn = xn_smem ? reinterpret_cast<uint16_t*>(att_area) : a.act_h;
   const int xn_out_ld = xn_smem ? xn_ld : a.Kp_H;
+  // one row from the residual stream: staged through shared memory behind
+  // the normalised row (rmsnorm_staged)
+  const size_t stage_off = ((size_t)M * xn_ld * 2 + 127) / 128 * 128;
+  const bool norm_staged = M == 1 && xn_smem && a.H <= 24 * kThreads && stage_off + (size_t)a.H * 8 <= SS::kQ;
+  long long* stage = reinterpret_cast<long long*>(att_area + stage_off);
+  uint32_t nphase = 0;
   const int G = a.Hq / a.Hkv;
   if (threadIdx.x < 4) {
     const int k = threadIdx.x;
@@ -922,8 +1000,11 @@ __global__ void __launch_bounds__(kBlockThreads, 1) step_kernel(const __grid_con
     if (k == 0 || k == 2) {
       // RMSNorm of the attention (k = 0) or MLP block; before the first
       // layer from the step's input rows
-      rmsnorm_cta(ph != 0, a.X, s_rowp, a.H, a.norms + (size_t)l * 2 * a.H + (k == 2 ? a.H : 0), a.eps, xn,
-                  xn_out_ld, M);
+      const uint16_t* nw_ = a.norms + (size_t)l * 2 * a.H + (k == 2 ? a.H : 0);
+      if (norm_staged && ph != 0)
+        rmsnorm_staged(a.X, a.H, nw_, a.eps, xn, stage, &s_nbar, nphase, a.status);
+      else
+        rmsnorm_cta(ph != 0, a.X, s_rowp, a.H, nw_, a.eps, xn, xn_out_ld, M);
     } else if (k == 1) {
       // the q|k|v sums and counts are consumed: clear them for the next layer
       for (int e = gt; e < M * qkv_rows; e += gs) __stcg(a.acc_qkv + e, 0LL);
