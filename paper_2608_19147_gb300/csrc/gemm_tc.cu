@@ -5,60 +5,62 @@
 // is filled by running the prompt through the stage) -- where the per-token
 // GEMV of the decode step would stream every weight once per 16 tokens.
 //
-// One CTA (8 warps) computes a tile of 128 weight rows (two 64-row blocks)
-// by N tokens, walking K one 128-input unit at a time, as a two-stage
-// software pipeline (every buffer below exists twice, used by alternate
-// steps):
-//   - thread 0 bulk-copies the tile's two units (codes, scales, zero points)
-//     into shared memory (TMA, non-tensor; mbarrier completion) two steps
-//     ahead;
-//   - the CTA stages the N x 128 token tile into shared memory in the
-//     canonical K-major layout without swizzle (8-row x 16-byte core
-//     matrices: element (row, k) at (row/8)*2048 + (k/8)*128 + (row%8)*16
-//     + (k%8)*2 bytes) and dequantises the weights into the same layout as
-//     exact fp16 (q - z) -- the per-group fp16 scale is applied later in
-//     fp32, so no rounding is added to the W4A16 arithmetic;
-//   - thread 0 issues tcgen05.mma (kind::f16, M = 128, N tokens, K = 16 per
-//     instruction) from the two shared-memory operands into a tensor-memory
-//     accumulator per quantisation group and commits them to an mbarrier;
-//   - while those run, the CTA prepares the next step and reads back the
-//     accumulators of the step before (tcgen05.ld; warp w holds rows
-//     32 (w % 4) .. + 31, half of the token columns), multiplies them by the
-//     row's group scale and adds them into fp32 registers.
-// At the end each thread writes its row's outputs.  Waits are bounded; a wait
-// that runs out sets the status word.  The tensor memory is freed before the
-// CTA exits.
+// One CTA computes a tile of 128 weight rows (two 64-row blocks) by N tokens,
+// walking K one 128-input unit per step, with warp roles joined by mbarriers:
+//   - warp 0 (producer): bulk-copies the step's two units (codes, scales,
+//     zero points) and loads the token tile with 2-D tensor copies, one box of
+//     8 inputs x N tokens per 16-byte K chunk; 3 stages ahead;
+//   - warps 10..13 (dequantise): turn the codes into exact fp16 (q - z) in the
+//     A tile; 2 stages;
+//   - warp 1 (MMA): issues tcgen05.mma (kind::f16, M = 128, N tokens, K = 16
+//     per instruction) into a TMEM accumulator per quantisation group and
+//     commits to the stages' mbarriers; 2 accumulator stages;
+//   - warps 2..9 (epilogue): read the step's accumulators (tcgen05.ld; warp w
+//     owns TMEM lanes 32 (w % 4) .. + 31 = tile rows, half the token columns
+//     each), multiply by the row's fp32 group scale and add into registers;
+//     at the end they write their rows' outputs.
+// Both operands sit in shared memory as [K chunk][row][8 values] (16-byte
+// rows): the canonical K-major layout without swizzle, with the 8-row groups
+// 128 bytes apart and the K chunks rows * 16 bytes apart -- the layout the
+// tensor copy writes for a box of 8 inputs, and one in which the dequantise
+// warps' 16-byte stores of 8 consecutive rows hit distinct banks.  The
+// arithmetic is the decode projection's: exact (q - z), fp32 sums per group,
+// the fp16 scale applied in fp32.  Every wait is bounded; a wait that runs out
+// sets the status word.  The TMEM columns are freed before the CTA exits.
+#include <cuda.h>
+
+#include <mutex>
+
 #include "gemv_core.cuh"
 
 namespace shard {
 namespace {
 
-constexpr int kTcRows = 128;       // weight rows per CTA tile (two row-blocks)
-constexpr int kTcThreads = 256;    // 8 warps: warp w owns rows 32 (w % 4) .. + 31, columns half w / 4
-constexpr uint32_t kCoreK = 128;   // bytes between core matrices adjacent in K
-constexpr uint32_t kCoreMN = 2048; // bytes between 8-row groups (16 core matrices of K)
+constexpr int kTcRows = 128;        // weight rows per CTA tile (two row-blocks)
+constexpr int kTcWarps = 14;        // producer, MMA, 8 epilogue, 4 dequantise
+constexpr int kTcThreads = kTcWarps * 32;
+constexpr int kEpiWarp0 = 2, kDqWarp0 = 10;
+constexpr int kUStages = 3, kBStages = 3, kAStages = 2, kDStages = 2;
 
 template <int N, int GPU>
 struct TcSmem {
   static constexpr size_t kUnit = Geom<GPU>::kUnitBytes;
-  static constexpr size_t kUnits = 2 * kUnit;          // the tile's two units
-  static constexpr size_t kA = (size_t)kTcRows * 256;  // 128 rows x 128 fp16
-  static constexpr size_t kB = (size_t)N * 256;        // N tokens x 128 fp16
-  static constexpr size_t kSc = (size_t)GPU * kTcRows * 4;  // the step's scales, fp32 [group][row]
-  static constexpr size_t kUnitsOff = 0;                            // [2][kUnits]
-  static constexpr size_t kAOff = (2 * kUnits + 1023) / 1024 * 1024;  // [2][kA]
-  static constexpr size_t kBOff = kAOff + 2 * kA;                   // [2][kB]
-  static constexpr size_t kScOff = kBOff + 2 * kB;                  // [2][kSc]
-  static constexpr size_t kTotal = kScOff + 2 * kSc;
+  static constexpr size_t kUnits = 2 * kUnit;                          // the tile's two units
+  static constexpr size_t kA = (size_t)kTcRows * 256;                  // 16 K chunks x 128 rows x 16 B
+  static constexpr size_t kB = (size_t)N * 256;                        // 16 K chunks x N tokens x 16 B
+  static constexpr size_t kAOff = 0;                                   // [kAStages][kA]
+  static constexpr size_t kBOff = kAOff + kAStages * kA;               // [kBStages][kB]
+  static constexpr size_t kUOff = kBOff + kBStages * kB;               // [kUStages][kUnits]
+  static constexpr size_t kTotal = kUOff + kUStages * kUnits + 1024;   // + alignment slack
 };
 
-// Shared-memory matrix descriptor: K-major, no swizzle; LBO = distance of
-// core matrices adjacent in K, SBO = distance of 8-row groups.
-__device__ __forceinline__ uint64_t smem_desc(uint32_t addr) {
+// Shared-memory matrix descriptor, K-major without swizzle: lbo = bytes between
+// core matrices adjacent in K, sbo = bytes between 8-row groups.
+__device__ __forceinline__ uint64_t smem_desc(uint32_t addr, uint32_t lbo, uint32_t sbo) {
   uint64_t d = 0;
   d |= (uint64_t)((addr & 0x3FFFFu) >> 4);
-  d |= (uint64_t)(kCoreK >> 4) << 16;
-  d |= (uint64_t)(kCoreMN >> 4) << 32;
+  d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
+  d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
   d |= 1ull << 46;  // descriptor version for this architecture
   return d;         // base offset 0, layout type 0 (no swizzle)
 }
@@ -81,12 +83,13 @@ __device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t adesc, uint64_t
       : "memory");
 }
 
+// Arrive on `bar` once every tcgen05 operation this thread issued so far is done.
 __device__ __forceinline__ void tc_commit(uint64_t* bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_addr(bar))
                : "memory");
 }
 
-// 32 consecutive fp32 columns of this thread's tensor-memory lane.
+// 32 (or 16) consecutive fp32 columns of this thread's tensor-memory lane.
 __device__ __forceinline__ void tc_ld32(uint32_t taddr, float (&v)[32]) {
   uint32_t r[32];
   asm volatile(
@@ -102,8 +105,6 @@ __device__ __forceinline__ void tc_ld32(uint32_t taddr, float (&v)[32]) {
 #pragma unroll
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
-
-// 16 consecutive fp32 columns of this thread's tensor-memory lane.
 __device__ __forceinline__ void tc_ld16(uint32_t taddr, float (&v)[32]) {
   uint32_t r[16];
   asm volatile(
@@ -118,37 +119,73 @@ __device__ __forceinline__ void tc_ld16(uint32_t taddr, float (&v)[32]) {
   for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
 
-__device__ __forceinline__ uint32_t a_off(int row, int k) {
-  return (uint32_t)(row >> 3) * kCoreMN + (uint32_t)(k >> 3) * kCoreK + (uint32_t)(row & 7) * 16u + (uint32_t)(k & 7) * 2u;
+// 2-D tensor copy of one box into shared memory, completion on `bar`.
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, int x, int y, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+          smem_addr(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_addr(bar))
+      : "memory");
 }
 
+// Offset of element (row, k) of a [K chunk][rows][8] operand tile.
+__device__ __forceinline__ uint32_t op_off(int rows, int row, int k) {
+  return (uint32_t)(k >> 3) * (uint32_t)(rows * 16) + (uint32_t)row * 16u + (uint32_t)(k & 7) * 2u;
+}
+
+// Kernel arguments: the projection and the tensor map of its activations
+// (fp16 [S][act_ld], box 8 inputs x N tokens).
+struct TcParams {
+  GemmArgs a;
+  CUtensorMap act_map;
+};
+
 template <int N, int GPU>
-__global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_constant__ GemmArgs a) {
+__global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_constant__ TcParams P) {
+  const GemmArgs& a = P.a;
   using L = TcSmem<N, GPU>;
   constexpr int UB = Geom<GPU>::kUnitBytes;
-  constexpr int G = GPU;                       // quantisation groups per unit
-  constexpr int kMmaPerGroup = 8 / GPU;        // K = 16 per instruction
-  constexpr int kHalf = N / 2;                 // token columns per thread
-  constexpr int kBPer = (N * 16 + kTcThreads - 1) / kTcThreads;  // 16-byte token pieces per thread
-  constexpr uint32_t kColsNeed = 2u * G * N;   // two steps' accumulators
+  constexpr int G = GPU;                        // quantisation groups per unit
+  constexpr int kMmaPerGroup = 8 / GPU;         // K = 16 per instruction
+  constexpr int kHalf = N / 2;                  // token columns per epilogue thread
+  constexpr uint32_t kLboA = kTcRows * 16, kLboB = N * 16, kSbo = 128;
+  constexpr uint32_t kColsNeed = (uint32_t)kDStages * G * N;
   constexpr uint32_t kCols = kColsNeed <= 32 ? 32u : kColsNeed <= 64 ? 64u : kColsNeed <= 128 ? 128u
                              : kColsNeed <= 256 ? 256u : 512u;
   static_assert(kColsNeed <= 512, "accumulators exceed tensor memory");
-  static_assert(kHalf % 32 == 0 || kHalf == 16, "columns per thread");
-  extern __shared__ __align__(1024) uint8_t smem[];
-  __shared__ uint64_t s_ubar[2], s_mbar[2];
+  static_assert(kHalf == 16 || kHalf % 32 == 0, "columns per epilogue thread");
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  __shared__ uint64_t u_full[kUStages], u_empty[kUStages], b_full[kBStages], b_empty[kBStages];
+  __shared__ uint64_t a_full[kAStages], a_empty[kAStages], d_full[kDStages], d_empty[kDStages];
   __shared__ uint32_t s_tmem;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int rb0 = 2 * blockIdx.x;              // the tile's first row-block
-  const int n0 = blockIdx.y * N;               // the tile's first token
+  const int rb0 = 2 * blockIdx.x;   // the tile's first row-block
+  const int n0 = blockIdx.y * N;    // the tile's first token
+  const int steps = a.upr;
+  auto A_of = [&](int s) { return smem + L::kAOff + (size_t)s * L::kA; };
+  auto B_of = [&](int s) { return smem + L::kBOff + (size_t)s * L::kB; };
+  auto U_of = [&](int s) { return smem + L::kUOff + (size_t)s * L::kUnits; };
   if (tid == 0) {
-    for (int i = 0; i < 2; ++i) {
-      mbar_init(&s_ubar[i], 1);
-      mbar_init(&s_mbar[i], 1);
+    for (int i = 0; i < kUStages; ++i) {
+      mbar_init(&u_full[i], 1);
+      mbar_init(&u_empty[i], 4 + 8);  // the dequantise and the epilogue warps (scales)
+    }
+    for (int i = 0; i < kBStages; ++i) {
+      mbar_init(&b_full[i], 1);
+      mbar_init(&b_empty[i], 1);
+    }
+    for (int i = 0; i < kAStages; ++i) {
+      mbar_init(&a_full[i], 4);
+      mbar_init(&a_empty[i], 1);
+    }
+    for (int i = 0; i < kDStages; ++i) {
+      mbar_init(&d_full[i], 1);
+      mbar_init(&d_empty[i], 8);
     }
     mbar_fence_init();
   }
-  if (warp == 0) {
+  if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_addr(&s_tmem)),
                  "r"(kCols)
                  : "memory");
@@ -158,146 +195,200 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = s_tmem;
-  const int row = 32 * (warp & 3) + lane;      // this thread's row of the tile (its tensor-memory lane)
-  const int c0 = kHalf * (warp >> 2);          // its first token column
-  auto units_of = [&](int s) { return smem + L::kUnitsOff + (size_t)s * L::kUnits; };
-  auto A_of = [&](int s) { return smem + L::kAOff + (size_t)s * L::kA; };
-  auto B_of = [&](int s) { return smem + L::kBOff + (size_t)s * L::kB; };
-  auto sc_of = [&](int s) { return reinterpret_cast<float*>(smem + L::kScOff + (size_t)s * L::kSc); };
-  auto issue_units = [&](int ku, int s) {
-    mbar_arrive_expect_tx(&s_ubar[s], 2 * UB);
-    for (int u = 0; u < 2; ++u) {
-      const int rb = rb0 + u < a.n_rb ? rb0 + u : rb0;  // a missing second block repeats the first (unused)
-      bulk_g2s(units_of(s) + (size_t)u * UB, a.units + ((size_t)rb * a.upr + ku) * UB, UB, &s_ubar[s]);
-    }
+  bool ok = true;  // false once a wait gave up: the role skips the rest of its waits
+  auto wait = [&](uint64_t* bar, uint32_t parity) {
+    if (ok && !mbar_wait(bar, parity)) ok = false;
   };
-  float tot[kHalf];
-#pragma unroll
-  for (int c = 0; c < kHalf; ++c) tot[c] = 0.f;
-  bool ok = true;
-  // scale and add the accumulators of step j (slot j & 1)
-  auto epilogue = [&](int j) {
-    const int s = j & 1;
-    if (ok && !mbar_wait(&s_mbar[s], (j >> 1) & 1)) ok = false;
-    tc_fence_after();
-    const float* sc = sc_of(s);
-#pragma unroll
-    for (int gq = 0; gq < G; ++gq) {
-      const float sv = sc[gq * kTcRows + row];
-#pragma unroll
-      for (int cc = 0; cc < kHalf; cc += 32) {
-        float v[32];
-        const uint32_t ta = tmem + ((uint32_t)(32 * (warp & 3)) << 16) + (uint32_t)((s * G + gq) * N + c0 + cc);
-        if (kHalf >= 32)
-          tc_ld32(ta, v);
-        else
-          tc_ld16(ta, v);  // 16 columns: only those of this thread's half
-#pragma unroll
-        for (int c = 0; c < 32; ++c)
-          if (cc + c < kHalf) tot[cc + c] = fmaf(sv, v[c], tot[cc + c]);
+
+  if (warp == 0) {
+    // ---- producer: units and token tiles, kUStages / kBStages steps ahead ----
+    if (lane == 0) {
+      for (int k = 0; k < steps; ++k) {
+        const int su = k % kUStages, sb = k % kBStages;
+        wait(&u_empty[su], ((k / kUStages) & 1) ^ 1);
+        mbar_arrive_expect_tx(&u_full[su], 2 * UB);
+        for (int u = 0; u < 2; ++u) {
+          const int rb = rb0 + u < a.n_rb ? rb0 + u : rb0;  // a missing second block repeats the first (unused)
+          bulk_g2s(U_of(su) + (size_t)u * UB, a.units + ((size_t)rb * a.upr + k) * UB, UB, &u_full[su]);
+        }
+        wait(&b_empty[sb], ((k / kBStages) & 1) ^ 1);
+        mbar_arrive_expect_tx(&b_full[sb], N * 256);
+        for (int kc = 0; kc < 16; ++kc)  // tokens past S read as zero
+          tma_load_2d(B_of(sb) + (size_t)kc * N * 16, &P.act_map, k * kUnitK + kc * 8, n0, &b_full[sb]);
       }
     }
-  };
-  if (tid == 0) {
-    issue_units(0, 0);
-    if (a.upr > 1) issue_units(1, 1);
-  }
-  for (int k = 0; k < a.upr; ++k) {
-    const int s = k & 1;
-    // the step's token tile, into registers (its latency overlaps the epilogue)
-    uint4 bv[kBPer];
+  } else if (warp == 1) {
+    // ---- MMA issue: one thread ----
+    if (lane == 0) {
+      for (int k = 0; k < steps; ++k) {
+        const int sa = k % kAStages, sb = k % kBStages, sd = k % kDStages;
+        wait(&a_full[sa], (k / kAStages) & 1);
+        wait(&b_full[sb], (k / kBStages) & 1);
+        wait(&d_empty[sd], ((k / kDStages) & 1) ^ 1);
+        tc_fence_after();
+        if (ok) {
+          const uint32_t aBase = smem_addr(A_of(sa)), bBase = smem_addr(B_of(sb));
 #pragma unroll
-    for (int i = 0; i < kBPer; ++i) {
-      const int e = tid + i * kTcThreads, n = e >> 4, kc = e & 15;
-      bv[i] = make_uint4(0, 0, 0, 0);
-      if (e < N * 16 && n0 + n < a.S)
-        bv[i] = __ldcg(reinterpret_cast<const uint4*>(a.act + (size_t)(n0 + n) * a.act_ld + k * kUnitK + 8 * kc));
-    }
-    // step k - 2 used this slot: its MMAs are done once its accumulators are read
-    if (k >= 2) epilogue(k - 2);
-    tc_fence_before();
-    __syncthreads();  // slot s (tiles, scales, accumulators) is free
-    if (ok && !mbar_wait(&s_ubar[s], (k >> 1) & 1)) ok = false;
-    uint8_t* Bs = B_of(s);
+          for (int gq = 0; gq < G; ++gq)
 #pragma unroll
-    for (int i = 0; i < kBPer; ++i) {
-      const int e = tid + i * kTcThreads;
-      if (e < N * 16) *reinterpret_cast<uint4*>(Bs + a_off(e >> 4, 8 * (e & 15))) = bv[i];
-    }
-    // dequantise: word (ft, l, j) of unit u holds rows 16 rt + gid (+8) at
-    // inputs k0 .. k0 + 3 (kernels.h); q - z exactly, as fp16
-    const uint8_t* Us = units_of(s);
-    uint8_t* As = A_of(s);
-    for (int e = tid; e < 2 * (kCodeBytes / 4); e += kTcThreads) {
-      const int u = e / (kCodeBytes / 4), wi = e % (kCodeBytes / 4);
-      const int ft = wi >> 7, l = (wi >> 2) & 31, j = wi & 3;
-      const int kc = ft >> 2, rt = ft & 3, gid = l >> 2, tig = l & 3;
-      const int k0 = 64 * kc + 32 * (j >> 1) + 8 * tig + 4 * (j & 1);
-      const uint8_t* U = Us + (size_t)u * UB;
-      const uint32_t w = reinterpret_cast<const uint32_t*>(U)[wi];
-      const uint8_t* meta = U + kCodeBytes + (k0 / (kUnitK / G)) * kMetaBytesPerGroup;
-      const int idx = gid * 8 + rt * 2;
-      const uint32_t zlo = meta[128 + idx], z16hi = meta[128 + idx + 1];
-      const uint32_t zsub = (0x6400u | zlo) * 0x00010001u;         // fp16x2 (1024 + z)
-      const uint32_t zfma = (0xD400u | z16hi) * 0x00010001u;       // fp16x2 -(64 + z)
-      const uint32_t w2 = w >> 8;
-      const uint32_t q01 = hsub2_u32(lop3_and_or(w, 0x000F000Fu, 0x64006400u), zsub);
-      const uint32_t q23 = hsub2_u32(lop3_and_or(w2, 0x000F000Fu, 0x64006400u), zsub);
-      const uint32_t h01 = hfma2_u32(lop3_and_or(w, 0x00F000F0u, 0x64006400u), 0x2C002C00u, zfma);
-      const uint32_t h23 = hfma2_u32(lop3_and_or(w2, 0x00F000F0u, 0x64006400u), 0x2C002C00u, zfma);
-      const int r = 64 * u + 16 * rt + gid;
-      *reinterpret_cast<uint2*>(As + a_off(r, k0)) = make_uint2(q01, q23);
-      *reinterpret_cast<uint2*>(As + a_off(r + 8, k0)) = make_uint2(h01, h23);
-    }
-    // the step's scales, fp32 [group][row]
-    float* sc = sc_of(s);
-    for (int e = tid; e < G * kTcRows; e += kTcThreads) {
-      const int gq = e / kTcRows, r = e % kTcRows, R = r & 63;
-      const int sidx = (R & 7) * 8 + ((R >> 4) & 3) * 2 + ((R >> 3) & 1);
-      sc[e] = h2f(reinterpret_cast<const uint16_t*>(Us + (size_t)(r >> 6) * UB + kCodeBytes +
-                                                    gq * kMetaBytesPerGroup)[sidx]);
-    }
-    // generic-proxy writes of A and B become visible to the tensor cores
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    if (tid == 0) {
-      if (k + 2 < a.upr) issue_units(k + 2, s);  // the slot's units were read above
-      const uint32_t aBase = smem_addr(As), bBase = smem_addr(Bs);
-#pragma unroll
-      for (int gq = 0; gq < G; ++gq)
-#pragma unroll
-        for (int i = 0; i < kMmaPerGroup; ++i) {
-          const int kk = gq * kMmaPerGroup + i;  // K = 16 per instruction: two core matrices
-          tc_mma(tmem + (uint32_t)((s * G + gq) * N), smem_desc(aBase + kk * 2 * kCoreK),
-                 smem_desc(bBase + kk * 2 * kCoreK), instr_desc<N>(), i > 0);
+            for (int i = 0; i < kMmaPerGroup; ++i) {
+              const int kk = gq * kMmaPerGroup + i;  // K = 16: K chunks 2 kk, 2 kk + 1
+              tc_mma(tmem + (uint32_t)((sd * G + gq) * N), smem_desc(aBase + kk * 2 * kLboA, kLboA, kSbo),
+                     smem_desc(bBase + kk * 2 * kLboB, kLboB, kSbo), instr_desc<N>(), i > 0);
+            }
         }
-      tc_commit(&s_mbar[s]);
+        tc_commit(&a_empty[sa]);
+        tc_commit(&b_empty[sb]);
+        tc_commit(&d_full[sd]);
+      }
+    }
+  } else if (warp >= kDqWarp0) {
+    // ---- dequantise: exact fp16 (q - z) into the A tile ----
+    const int dt = (warp - kDqWarp0) * 32 + lane;
+    const int gid = dt & 7, tig = (dt >> 3) & 3;  // 8 consecutive threads: rows gid 0..7 of one K chunk
+    const int l = gid * 4 + tig;                  // the fragment lane whose words this thread takes
+    for (int k = 0; k < steps; ++k) {
+      const int su = k % kUStages, sa = k % kAStages;
+      wait(&u_full[su], (k / kUStages) & 1);
+      wait(&a_empty[sa], ((k / kAStages) & 1) ^ 1);
+      const uint8_t* Us = U_of(su);
+      uint8_t* As = A_of(sa);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int uf = (warp - kDqWarp0) + 4 * i;  // (unit, code tile) 0..15
+        const int u = uf >> 3, ft = uf & 7, rt = ft & 3, kh = ft >> 2;
+        const uint8_t* U = Us + (size_t)u * UB;
+        const uint4 w4 = *reinterpret_cast<const uint4*>(U + ft * 512 + l * 16);
+        const uint32_t wv[4] = {w4.x, w4.y, w4.z, w4.w};
+        const int row = 64 * u + 16 * rt + gid;
+        uint32_t lo[2][4], hi[2][4];  // [K chunk: j / 2][4 fp16 pairs]
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          // word j: rows gid and gid + 8 at inputs k0 .. k0 + 3
+          const int k0 = 64 * kh + 32 * (j >> 1) + 8 * tig + 4 * (j & 1);
+          const uint8_t* meta = U + kCodeBytes + (k0 / (kUnitK / G)) * kMetaBytesPerGroup;
+          const int zi = gid * 8 + rt * 2;
+          const uint32_t zsub = (0x6400u | meta[128 + zi]) * 0x00010001u;      // fp16x2 (1024 + z)
+          const uint32_t zfma = (0xD400u | meta[128 + zi + 1]) * 0x00010001u;  // fp16x2 -(64 + z)
+          const uint32_t w = wv[j], w2 = w >> 8;
+          lo[j >> 1][2 * (j & 1)] = hsub2_u32(lop3_and_or(w, 0x000F000Fu, 0x64006400u), zsub);
+          lo[j >> 1][2 * (j & 1) + 1] = hsub2_u32(lop3_and_or(w2, 0x000F000Fu, 0x64006400u), zsub);
+          hi[j >> 1][2 * (j & 1)] = hfma2_u32(lop3_and_or(w, 0x00F000F0u, 0x64006400u), 0x2C002C00u, zfma);
+          hi[j >> 1][2 * (j & 1) + 1] = hfma2_u32(lop3_and_or(w2, 0x00F000F0u, 0x64006400u), 0x2C002C00u, zfma);
+        }
+#pragma unroll
+        for (int c = 0; c < 2; ++c) {
+          const int kb = 64 * kh + 32 * c + 8 * tig;  // the 8-input chunk's first input
+          *reinterpret_cast<uint4*>(As + op_off(kTcRows, row, kb)) = make_uint4(lo[c][0], lo[c][1], lo[c][2], lo[c][3]);
+          *reinterpret_cast<uint4*>(As + op_off(kTcRows, row + 8, kb)) =
+              make_uint4(hi[c][0], hi[c][1], hi[c][2], hi[c][3]);
+        }
+      }
+      // the generic-proxy stores become visible to the tensor cores
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(&a_full[sa]);
+        mbar_arrive(&u_empty[su]);
+      }
+    }
+  } else {
+    // ---- epilogue: scale and add each step's group sums ----
+    const int quad = warp & 3, half = (warp - kEpiWarp0) >> 2;
+    const int row = 32 * quad + lane;  // tile row = TMEM lane
+    const int c0 = half * kHalf;
+    const int R = row & 63;
+    const int sidx = (R & 7) * 8 + ((R >> 4) & 3) * 2 + ((R >> 3) & 1);  // the row's scale in a group's meta
+    float tot[kHalf];
+#pragma unroll
+    for (int c = 0; c < kHalf; ++c) tot[c] = 0.f;
+    for (int k = 0; k < steps; ++k) {
+      const int su = k % kUStages, sd = k % kDStages;
+      wait(&d_full[sd], (k / kDStages) & 1);
+      wait(&u_full[su], (k / kUStages) & 1);  // the unit (its scales) stays until this warp arrives
+      tc_fence_after();
+      const uint8_t* U = U_of(su) + (size_t)(row >> 6) * UB;
+#pragma unroll
+      for (int gq = 0; gq < G; ++gq) {
+        const float sv = h2f(reinterpret_cast<const uint16_t*>(U + kCodeBytes + gq * kMetaBytesPerGroup)[sidx]);
+#pragma unroll
+        for (int cc = 0; cc < kHalf; cc += 32) {
+          float v[32];
+          const uint32_t ta = tmem + ((uint32_t)(32 * quad) << 16) + (uint32_t)((sd * G + gq) * N + c0 + cc);
+          if (kHalf >= 32)
+            tc_ld32(ta, v);
+          else
+            tc_ld16(ta, v);
+#pragma unroll
+          for (int c = 0; c < 32; ++c)
+            if (cc + c < kHalf) tot[cc + c] = fmaf(sv, v[c], tot[cc + c]);
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(&d_empty[sd]);
+        mbar_arrive(&u_empty[su]);
+      }
+    }
+    // outputs: natural row order, [token][row]
+    const int rbr = rb0 + (row >> 6);
+    if (rbr < a.n_rb) {
+      const int nat = natural_row(a.dims, rbr * kRowsPerBlock + R);
+      if (nat >= 0)
+#pragma unroll
+        for (int c = 0; c < kHalf; ++c)
+          if (n0 + c0 + c < a.S) a.y[(size_t)(n0 + c0 + c) * a.y_ld + nat] = tot[c];
     }
   }
-  for (int j = a.upr >= 2 ? a.upr - 2 : 0; j < a.upr; ++j) epilogue(j);
-  if (!ok && lane == 0) atomicOr(a.status, ST_WAIT_TIMEOUT);
-  // outputs: natural row order, [token][row]
-  const int rbr = rb0 + (row >> 6);
-  if (rbr < a.n_rb) {
-    const int nat = natural_row(a.dims, rbr * kRowsPerBlock + (row & 63));
-    if (nat >= 0)
-#pragma unroll
-      for (int c = 0; c < kHalf; ++c)
-        if (n0 + c0 + c < a.S) a.y[(size_t)(n0 + c0 + c) * a.y_ld + nat] = tot[c];
-  }
+  if (!ok) atomicOr(a.status, ST_WAIT_TIMEOUT);
   tc_fence_before();
   __syncthreads();
-  if (warp == 0)
+  tc_fence_after();
+  if (warp == 1)
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kCols) : "memory");
+}
+
+// cuTensorMapEncodeTiled, from the driver through the runtime (no link
+// against the driver library).
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_tiled() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q{};
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  return fn;
 }
 
 template <int N, int GPU>
 cudaError_t launch_tc(const GemmArgs& a, cudaStream_t s) {
   using L = TcSmem<N, GPU>;
+  EncodeTiledFn enc = encode_tiled();
+  if (!enc) return cudaErrorNotSupported;
+  // the activations: fp16 [S][act_ld] (16-byte aligned rows); box = 8
+  // inputs (16 bytes) x N tokens; tokens past S read as zero
+  if ((reinterpret_cast<uintptr_t>(a.act) & 15) || a.act_ld % 8 || a.upr * kUnitK > a.act_ld || a.S < 1)
+    return cudaErrorInvalidValue;
+  TcParams p;
+  p.a = a;
+  const cuuint64_t dims[2] = {(cuuint64_t)a.upr * kUnitK, (cuuint64_t)a.S};
+  const cuuint64_t strides[1] = {(cuuint64_t)a.act_ld * 2};
+  const cuuint32_t box[2] = {8, (cuuint32_t)N};
+  const cuuint32_t estr[2] = {1, 1};
+  if (enc(&p.act_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<uint16_t*>(a.act), dims, strides, box, estr,
+          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+    return cudaErrorInvalidValue;
   const dim3 grid((a.n_rb + 1) / 2, (a.S + N - 1) / N);
-  gemm_tc_kernel<N, GPU><<<grid, kTcThreads, L::kTotal, s>>>(a);
+  gemm_tc_kernel<N, GPU><<<grid, kTcThreads, L::kTotal, s>>>(p);
   return cudaGetLastError();
 }
 
@@ -322,7 +413,8 @@ cudaError_t gemm_tc_setup() {
   return cudaSuccess;
 }
 
-// Token tile: 128 for long prompts, smaller for short ones.
+// Token tile: 128 for long prompts, smaller for short ones; at group 32 (four
+// accumulators per step) at most 64.
 int gemm_tc_tile(int S) { return S > 64 ? 128 : S > 32 ? 64 : 32; }
 int gemm_tc_tile(int S, int group) { return group == 32 ? (S > 32 ? 64 : 32) : gemm_tc_tile(S); }
 
