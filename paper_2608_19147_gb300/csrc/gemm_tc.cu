@@ -8,9 +8,9 @@
 // One CTA computes a tile of 128 weight rows (two 64-row blocks) by N tokens,
 // walking K one 128-input unit per step, with warp roles joined by mbarriers:
 //   - warp 0 (producer): bulk-copies the step's two units (codes, scales,
-//     zero points) and loads the token tile with 2-D tensor copies, one box of
-//     8 inputs x N tokens per 16-byte K chunk; 3 stages ahead;
-//   - warps 10..13 (dequantise): turn the codes into exact fp16 (q - z) in the
+//     zero points) and loads the token tile with two 2-D tensor copies (64
+//     inputs x N tokens each, 128-byte swizzle); 3 stages ahead;
+//   - warps 10..17 (dequantise): turn the codes into exact fp16 (q - z) in the
 //     A tile; 2 stages;
 //   - warp 1 (MMA): issues tcgen05.mma (kind::f16, M = 128, N tokens, K = 16
 //     per instruction) into a TMEM accumulator per quantisation group and
@@ -19,11 +19,12 @@
 //     owns TMEM lanes 32 (w % 4) .. + 31 = tile rows, half the token columns
 //     each), multiply by the row's fp32 group scale and add into registers;
 //     at the end they write their rows' outputs.
-// Both operands sit in shared memory as [K chunk][row][8 values] (16-byte
-// rows): the canonical K-major layout without swizzle, with the 8-row groups
-// 128 bytes apart and the K chunks rows * 16 bytes apart -- the layout the
-// tensor copy writes for a box of 8 inputs, and one in which the dequantise
-// warps' 16-byte stores of 8 consecutive rows hit distinct banks.  The
+// Both operands sit in shared memory in the canonical K-major layout with the
+// 128-byte swizzle: per 64-input half of the step, row r's 128 bytes at r *
+// 128, its 16-byte chunk c at chunk c ^ (r % 8) -- what the tensor copy writes
+// with that swizzle, whole 32-byte sectors from L2, and a layout in which the
+// dequantise warps' 16-byte stores of 8 consecutive rows hit distinct banks.
+// The
 // arithmetic is the decode projection's: exact (q - z), fp32 sums per group,
 // the fp16 scale applied in fp32.  Every wait is bounded; a wait that runs out
 // sets the status word.  The TMEM columns are freed before the CTA exits.
@@ -37,7 +38,8 @@ namespace shard {
 namespace {
 
 constexpr int kTcRows = 128;        // weight rows per CTA tile (two row-blocks)
-constexpr int kTcWarps = 14;        // producer, MMA, 8 epilogue, 4 dequantise
+constexpr int kTcWarps = 18;        // producer, MMA, 8 epilogue, 8 dequantise
+constexpr int kDqWarps = 8;
 constexpr int kTcThreads = kTcWarps * 32;
 constexpr int kEpiWarp0 = 2, kDqWarp0 = 10;
 constexpr int kUStages = 3, kBStages = 3, kAStages = 2, kDStages = 2;
@@ -54,15 +56,18 @@ struct TcSmem {
   static constexpr size_t kTotal = kUOff + kUStages * kUnits + 1024;   // + alignment slack
 };
 
-// Shared-memory matrix descriptor, K-major without swizzle: lbo = bytes between
-// core matrices adjacent in K, sbo = bytes between 8-row groups.
-__device__ __forceinline__ uint64_t smem_desc(uint32_t addr, uint32_t lbo, uint32_t sbo) {
+// Shared-memory matrix descriptor, K-major with the 128-byte swizzle: 8-row
+// groups 1024 bytes apart (the byte offset between K-adjacent core matrices is
+// implied by the swizzle); the start address may move by 32 bytes per K = 16
+// inside a 64-input half.
+__device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t addr) {
   uint64_t d = 0;
   d |= (uint64_t)((addr & 0x3FFFFu) >> 4);
-  d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
-  d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
-  d |= 1ull << 46;  // descriptor version for this architecture
-  return d;         // base offset 0, layout type 0 (no swizzle)
+  d |= (uint64_t)1 << 16;            // leading byte offset: unused with this swizzle
+  d |= (uint64_t)(1024 >> 4) << 32;  // stride byte offset
+  d |= 1ull << 46;                   // descriptor version for this architecture
+  d |= 2ull << 61;                   // layout: 128-byte swizzle
+  return d;
 }
 
 // Instruction descriptor, kind::f16: fp32 accumulator, fp16 A and B, both
@@ -128,16 +133,18 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, i
       : "memory");
 }
 
-// Offset of element (row, k) of a [K chunk][rows][8] operand tile.
+// Offset of element (row, k) of an operand tile of `rows` rows x 128 inputs,
+// 128-byte swizzled K-major: [64-input half][row][128 B], chunk c at c ^ (row % 8).
 __device__ __forceinline__ uint32_t op_off(int rows, int row, int k) {
-  return (uint32_t)(k >> 3) * (uint32_t)(rows * 16) + (uint32_t)row * 16u + (uint32_t)(k & 7) * 2u;
+  return (uint32_t)(k >> 6) * (uint32_t)(rows * 128) + (uint32_t)row * 128u +
+         (uint32_t)((((k >> 3) & 7) ^ (row & 7)) << 4) + (uint32_t)(k & 7) * 2u;
 }
 
 // Kernel arguments: the projection and the tensor map of its activations
 // (fp16 [S][act_ld], box 8 inputs x N tokens).
 struct TcParams {
   GemmArgs a;
-  CUtensorMap act_map;
+  CUtensorMap act_map;  // {K inputs, S tokens}, box 64 x N, 128-byte swizzle
 };
 
 template <int N, int GPU>
@@ -148,12 +155,12 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
   constexpr int G = GPU;                        // quantisation groups per unit
   constexpr int kMmaPerGroup = 8 / GPU;         // K = 16 per instruction
   constexpr int kHalf = N / 2;                  // token columns per epilogue thread
-  constexpr uint32_t kLboA = kTcRows * 16, kLboB = N * 16, kSbo = 128;
+  constexpr uint32_t kHalfA = kTcRows * 128, kHalfB = N * 128;  // bytes per 64-input half
   constexpr uint32_t kColsNeed = (uint32_t)kDStages * G * N;
   constexpr uint32_t kCols = kColsNeed <= 32 ? 32u : kColsNeed <= 64 ? 64u : kColsNeed <= 128 ? 128u
                              : kColsNeed <= 256 ? 256u : 512u;
   static_assert(kColsNeed <= 512, "accumulators exceed tensor memory");
-  static_assert(kHalf == 16 || kHalf % 32 == 0, "columns per epilogue thread");
+  static_assert(kHalf % 16 == 0, "columns per epilogue thread");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   __shared__ uint64_t u_full[kUStages], u_empty[kUStages], b_full[kBStages], b_empty[kBStages];
@@ -169,14 +176,14 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
   if (tid == 0) {
     for (int i = 0; i < kUStages; ++i) {
       mbar_init(&u_full[i], 1);
-      mbar_init(&u_empty[i], 4 + 8);  // the dequantise and the epilogue warps (scales)
+      mbar_init(&u_empty[i], kDqWarps + 8);  // the dequantise and the epilogue warps (scales)
     }
     for (int i = 0; i < kBStages; ++i) {
       mbar_init(&b_full[i], 1);
       mbar_init(&b_empty[i], 1);
     }
     for (int i = 0; i < kAStages; ++i) {
-      mbar_init(&a_full[i], 4);
+      mbar_init(&a_full[i], kDqWarps);
       mbar_init(&a_empty[i], 1);
     }
     for (int i = 0; i < kDStages; ++i) {
@@ -213,8 +220,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
         }
         wait(&b_empty[sb], ((k / kBStages) & 1) ^ 1);
         mbar_arrive_expect_tx(&b_full[sb], N * 256);
-        for (int kc = 0; kc < 16; ++kc)  // tokens past S read as zero
-          tma_load_2d(B_of(sb) + (size_t)kc * N * 16, &P.act_map, k * kUnitK + kc * 8, n0, &b_full[sb]);
+        for (int h = 0; h < 2; ++h)  // tokens past S read as zero
+          tma_load_2d(B_of(sb) + (size_t)h * kHalfB, &P.act_map, k * kUnitK + h * 64, n0, &b_full[sb]);
       }
     }
   } else if (warp == 1) {
@@ -232,9 +239,10 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
           for (int gq = 0; gq < G; ++gq)
 #pragma unroll
             for (int i = 0; i < kMmaPerGroup; ++i) {
-              const int kk = gq * kMmaPerGroup + i;  // K = 16: K chunks 2 kk, 2 kk + 1
-              tc_mma(tmem + (uint32_t)((sd * G + gq) * N), smem_desc(aBase + kk * 2 * kLboA, kLboA, kSbo),
-                     smem_desc(bBase + kk * 2 * kLboB, kLboB, kSbo), instr_desc<N>(), i > 0);
+              const int kk = gq * kMmaPerGroup + i;  // K = 16: inputs 16 kk .. + 15
+              const uint32_t ko = (uint32_t)(kk & 3) * 32u;  // inside the 64-input half
+              tc_mma(tmem + (uint32_t)((sd * G + gq) * N), smem_desc_sw128(aBase + (kk >> 2) * kHalfA + ko),
+                     smem_desc_sw128(bBase + (kk >> 2) * kHalfB + ko), instr_desc<N>(), i > 0);
             }
         }
         tc_commit(&a_empty[sa]);
@@ -254,27 +262,31 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
       const uint8_t* Us = U_of(su);
       uint8_t* As = A_of(sa);
 #pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const int uf = (warp - kDqWarp0) + 4 * i;  // (unit, code tile) 0..15
+      for (int i = 0; i < 16 / kDqWarps; ++i) {
+        const int uf = (warp - kDqWarp0) + kDqWarps * i;  // (unit, code tile) 0..15
         const int u = uf >> 3, ft = uf & 7, rt = ft & 3, kh = ft >> 2;
         const uint8_t* U = Us + (size_t)u * UB;
         const uint4 w4 = *reinterpret_cast<const uint4*>(U + ft * 512 + l * 16);
         const uint32_t wv[4] = {w4.x, w4.y, w4.z, w4.w};
         const int row = 64 * u + 16 * rt + gid;
         uint32_t lo[2][4], hi[2][4];  // [K chunk: j / 2][4 fp16 pairs]
+        uint32_t zsub[2], zfma[2];     // per K chunk (its 8 inputs lie in one group)
+#pragma unroll
+        for (int c = 0; c < 2; ++c) {
+          const uint8_t* meta = U + kCodeBytes + ((64 * kh + 32 * c + 8 * tig) / (kUnitK / G)) * kMetaBytesPerGroup;
+          const uint16_t zz = *reinterpret_cast<const uint16_t*>(meta + 128 + gid * 8 + rt * 2);
+          zsub[c] = (0x6400u | (zz & 0xFFu)) * 0x00010001u;  // fp16x2 (1024 + z)
+          zfma[c] = (0xD400u | (zz >> 8)) * 0x00010001u;     // fp16x2 -(64 + z)
+        }
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
-          // word j: rows gid and gid + 8 at inputs k0 .. k0 + 3
-          const int k0 = 64 * kh + 32 * (j >> 1) + 8 * tig + 4 * (j & 1);
-          const uint8_t* meta = U + kCodeBytes + (k0 / (kUnitK / G)) * kMetaBytesPerGroup;
-          const int zi = gid * 8 + rt * 2;
-          const uint32_t zsub = (0x6400u | meta[128 + zi]) * 0x00010001u;      // fp16x2 (1024 + z)
-          const uint32_t zfma = (0xD400u | meta[128 + zi + 1]) * 0x00010001u;  // fp16x2 -(64 + z)
+          // word j: rows gid and gid + 8 at inputs 64 kh + 32 (j / 2) + 8 tig + 4 (j % 2) .. + 3
           const uint32_t w = wv[j], w2 = w >> 8;
-          lo[j >> 1][2 * (j & 1)] = hsub2_u32(lop3_and_or(w, 0x000F000Fu, 0x64006400u), zsub);
-          lo[j >> 1][2 * (j & 1) + 1] = hsub2_u32(lop3_and_or(w2, 0x000F000Fu, 0x64006400u), zsub);
-          hi[j >> 1][2 * (j & 1)] = hfma2_u32(lop3_and_or(w, 0x00F000F0u, 0x64006400u), 0x2C002C00u, zfma);
-          hi[j >> 1][2 * (j & 1) + 1] = hfma2_u32(lop3_and_or(w2, 0x00F000F0u, 0x64006400u), 0x2C002C00u, zfma);
+          const uint32_t zs = zsub[j >> 1], zf = zfma[j >> 1];
+          lo[j >> 1][2 * (j & 1)] = hsub2_u32(lop3_and_or(w, 0x000F000Fu, 0x64006400u), zs);
+          lo[j >> 1][2 * (j & 1) + 1] = hsub2_u32(lop3_and_or(w2, 0x000F000Fu, 0x64006400u), zs);
+          hi[j >> 1][2 * (j & 1)] = hfma2_u32(lop3_and_or(w, 0x00F000F0u, 0x64006400u), 0x2C002C00u, zf);
+          hi[j >> 1][2 * (j & 1) + 1] = hfma2_u32(lop3_and_or(w2, 0x00F000F0u, 0x64006400u), 0x2C002C00u, zf);
         }
 #pragma unroll
         for (int c = 0; c < 2; ++c) {
@@ -312,16 +324,11 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
       for (int gq = 0; gq < G; ++gq) {
         const float sv = h2f(reinterpret_cast<const uint16_t*>(U + kCodeBytes + gq * kMetaBytesPerGroup)[sidx]);
 #pragma unroll
-        for (int cc = 0; cc < kHalf; cc += 32) {
+        for (int cc = 0; cc < kHalf; cc += 16) {
           float v[32];
-          const uint32_t ta = tmem + ((uint32_t)(32 * quad) << 16) + (uint32_t)((sd * G + gq) * N + c0 + cc);
-          if (kHalf >= 32)
-            tc_ld32(ta, v);
-          else
-            tc_ld16(ta, v);
+          tc_ld16(tmem + ((uint32_t)(32 * quad) << 16) + (uint32_t)((sd * G + gq) * N + c0 + cc), v);
 #pragma unroll
-          for (int c = 0; c < 32; ++c)
-            if (cc + c < kHalf) tot[cc + c] = fmaf(sv, v[c], tot[cc + c]);
+          for (int c = 0; c < 16; ++c) tot[cc + c] = fmaf(sv, v[c], tot[cc + c]);
         }
       }
       tc_fence_before();
@@ -381,10 +388,10 @@ cudaError_t launch_tc(const GemmArgs& a, cudaStream_t s) {
   p.a = a;
   const cuuint64_t dims[2] = {(cuuint64_t)a.upr * kUnitK, (cuuint64_t)a.S};
   const cuuint64_t strides[1] = {(cuuint64_t)a.act_ld * 2};
-  const cuuint32_t box[2] = {8, (cuuint32_t)N};
+  const cuuint32_t box[2] = {64, (cuuint32_t)N};
   const cuuint32_t estr[2] = {1, 1};
   if (enc(&p.act_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<uint16_t*>(a.act), dims, strides, box, estr,
-          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
     return cudaErrorInvalidValue;
   const dim3 grid((a.n_rb + 1) / 2, (a.S + N - 1) / N);
