@@ -42,7 +42,7 @@ constexpr int kTcWarps = 18;        // producer, MMA, 8 epilogue, 8 dequantise
 constexpr int kDqWarps = 8;
 constexpr int kTcThreads = kTcWarps * 32;
 constexpr int kEpiWarp0 = 2, kDqWarp0 = 10;
-constexpr int kUStages = 3, kBStages = 3, kAStages = 2, kDStages = 2;
+constexpr int kUStages = 4, kBStages = 3, kAStages = 2, kDStages = 2;
 
 template <int N, int GPU>
 struct TcSmem {
@@ -53,7 +53,9 @@ struct TcSmem {
   static constexpr size_t kAOff = 0;                                   // [kAStages][kA]
   static constexpr size_t kBOff = kAOff + kAStages * kA;               // [kBStages][kB]
   static constexpr size_t kUOff = kBOff + kBStages * kB;               // [kUStages][kUnits]
-  static constexpr size_t kTotal = kUOff + kUStages * kUnits + 1024;   // + alignment slack
+  static constexpr size_t kSc = (size_t)GPU * kTcRows * sizeof(float);  // a step's scales [group][row]
+  static constexpr size_t kScOff = kUOff + kUStages * kUnits;          // [kAStages][kSc]
+  static constexpr size_t kTotal = kScOff + kAStages * kSc + 1024;     // + alignment slack
 };
 
 // Shared-memory matrix descriptor, K-major with the 128-byte swizzle: 8-row
@@ -94,22 +96,7 @@ __device__ __forceinline__ void tc_commit(uint64_t* bar) {
                : "memory");
 }
 
-// 32 (or 16) consecutive fp32 columns of this thread's tensor-memory lane.
-__device__ __forceinline__ void tc_ld32(uint32_t taddr, float (&v)[32]) {
-  uint32_t r[32];
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
-      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
-        "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]),
-        "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
-        "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-      : "r"(taddr)
-      : "memory");
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-#pragma unroll
-  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
-}
+// 16 consecutive fp32 columns of this thread's tensor-memory lane (into v[0..15]).
 __device__ __forceinline__ void tc_ld16(uint32_t taddr, float (&v)[32]) {
   uint32_t r[16];
   asm volatile(
@@ -161,6 +148,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
                              : kColsNeed <= 256 ? 256u : 512u;
   static_assert(kColsNeed <= 512, "accumulators exceed tensor memory");
   static_assert(kHalf % 16 == 0, "columns per epilogue thread");
+  static_assert(kAStages == kDStages, "the epilogue reads the scales of its accumulator stage");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   __shared__ uint64_t u_full[kUStages], u_empty[kUStages], b_full[kBStages], b_empty[kBStages];
@@ -173,10 +161,11 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
   auto A_of = [&](int s) { return smem + L::kAOff + (size_t)s * L::kA; };
   auto B_of = [&](int s) { return smem + L::kBOff + (size_t)s * L::kB; };
   auto U_of = [&](int s) { return smem + L::kUOff + (size_t)s * L::kUnits; };
+  auto Sc_of = [&](int s) { return reinterpret_cast<float*>(smem + L::kScOff + (size_t)s * L::kSc); };
   if (tid == 0) {
     for (int i = 0; i < kUStages; ++i) {
       mbar_init(&u_full[i], 1);
-      mbar_init(&u_empty[i], kDqWarps + 8);  // the dequantise and the epilogue warps (scales)
+      mbar_init(&u_empty[i], kDqWarps);
     }
     for (int i = 0; i < kBStages; ++i) {
       mbar_init(&b_full[i], 1);
@@ -259,8 +248,16 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
       const int su = k % kUStages, sa = k % kAStages;
       wait(&u_full[su], (k / kUStages) & 1);
       wait(&a_empty[sa], ((k / kAStages) & 1) ^ 1);
+      wait(&d_empty[sa], ((k / kAStages) & 1) ^ 1);  // the epilogue is done with this stage's scales
       const uint8_t* Us = U_of(su);
       uint8_t* As = A_of(sa);
+      // the step's fp32 scales [group][tile row], for the epilogue
+      for (int e = dt; e < G * kTcRows; e += kDqWarps * 32) {
+        const int gq = e / kTcRows, r = e % kTcRows, R = r & 63;
+        const int sidx = (R & 7) * 8 + ((R >> 4) & 3) * 2 + ((R >> 3) & 1);
+        Sc_of(sa)[e] = h2f(reinterpret_cast<const uint16_t*>(Us + (size_t)(r >> 6) * UB + kCodeBytes +
+                                                            gq * kMetaBytesPerGroup)[sidx]);
+      }
 #pragma unroll
       for (int i = 0; i < 16 / kDqWarps; ++i) {
         const int uf = (warp - kDqWarp0) + kDqWarps * i;  // (unit, code tile) 0..15
@@ -310,19 +307,18 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
     const int row = 32 * quad + lane;  // tile row = TMEM lane
     const int c0 = half * kHalf;
     const int R = row & 63;
-    const int sidx = (R & 7) * 8 + ((R >> 4) & 3) * 2 + ((R >> 3) & 1);  // the row's scale in a group's meta
     float tot[kHalf];
 #pragma unroll
     for (int c = 0; c < kHalf; ++c) tot[c] = 0.f;
     for (int k = 0; k < steps; ++k) {
-      const int su = k % kUStages, sd = k % kDStages;
+      const int sd = k % kDStages;  // = the A stage: kAStages == kDStages
       wait(&d_full[sd], (k / kDStages) & 1);
-      wait(&u_full[su], (k / kUStages) & 1);  // the unit (its scales) stays until this warp arrives
+      wait(&a_full[sd], (k / kAStages) & 1);  // the stage's scales (written before its A tile was released)
       tc_fence_after();
-      const uint8_t* U = U_of(su) + (size_t)(row >> 6) * UB;
+      const float* sc = Sc_of(sd);
 #pragma unroll
       for (int gq = 0; gq < G; ++gq) {
-        const float sv = h2f(reinterpret_cast<const uint16_t*>(U + kCodeBytes + gq * kMetaBytesPerGroup)[sidx]);
+        const float sv = sc[gq * kTcRows + row];
 #pragma unroll
         for (int cc = 0; cc < kHalf; cc += 16) {
           float v[32];
@@ -333,10 +329,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) {
-        mbar_arrive(&d_empty[sd]);
-        mbar_arrive(&u_empty[su]);
-      }
+      if (lane == 0) mbar_arrive(&d_empty[sd]);
     }
     // outputs: natural row order, [token][row]
     const int rbr = rb0 + (row >> 6);
