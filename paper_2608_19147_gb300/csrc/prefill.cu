@@ -218,10 +218,193 @@ __global__ void prefill_residual_kernel(float* x, const float* y, int y_ld, int 
   }
 }
 
+// Causal attention of the new tokens on the tensor cores (mma.sync m16n8k16),
+// one CTA per (block of 64 / G tokens, kv head hk), 4 warps: query row r of
+// the 64 is token t0 + r / G, query head hk G + r % G, and warp w owns rows
+// 16 w .. + 15, so every K/V tile is read once for all the block's queries.
+// Entry tiles of 64 come through the beam table into shared memory.  Scores
+// S = Q K^T with Q split into fp16 hi + lo parts (together ~22 bits of q, so
+// the scores match an fp32 q); online softmax per row in fp32; O += P V with
+// P split the same way; fp32 accumulators.  Entry j is visible to token t iff
+// j <= P + t and mask[j] != 0.
+__device__ __forceinline__ void mma16816(float (&c)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ void ldsm_x4_trans(const void* p, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(smem_addr(p)));
+}
+// fp16x2 of (lo, hi) and the fp16x2 of what each rounding left out
+__device__ __forceinline__ void split_h2(float lo, float hi, uint32_t& h, uint32_t& l) {
+  const uint16_t a = f2h(lo), b = f2h(hi);
+  h = (uint32_t)a | ((uint32_t)b << 16);
+  l = (uint32_t)f2h(lo - h2f(a)) | ((uint32_t)f2h(hi - h2f(b)) << 16);
+}
+
+template <int D, int G>
+__global__ void __launch_bounds__(128) prefill_flash_kernel(const float* q, int Hq, int Hkv, const uint16_t* kpool,
+                                                           const uint16_t* vpool, const int* bt_row, int cap,
+                                                           const uint8_t* mask, int P, int S, uint16_t* out,
+                                                           int out_ld) {
+  constexpr int TB = 64 / G;  // tokens per CTA
+  constexpr int KS = D / 16;  // k16 steps over the head dimension
+  constexpr int ND = D / 8;   // n8 tiles over the head dimension
+  constexpr int LD = D + 8;   // shared row stride (halves): 16-byte rows, conflict-free fragment reads
+  __shared__ __align__(16) uint16_t Ks[64][LD];
+  __shared__ __align__(16) uint16_t Vs[64][LD];
+  __shared__ uint8_t vis[64];
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, gid = lane >> 2, tig = lane & 3;
+  const int t0 = blockIdx.x * TB, hk = blockIdx.y;
+  const float scale = rsqrtf((float)D);
+  // Q rows as fp16 hi (in Ks) and lo (in Vs), then this warp's fragments
+  for (int e = tid; e < 64 * D; e += 128) {
+    const int r = e / D, c = e % D, t = t0 + r / G;
+    const float v = t < S ? q[(size_t)t * Hq * D + (hk * G + r % G) * D + c] : 0.f;
+    const uint16_t hi = f2h(v);
+    Ks[r][c] = hi;
+    Vs[r][c] = f2h(v - h2f(hi));
+  }
+  __syncthreads();
+  const int ra = 16 * warp + gid, rb = ra + 8;  // this thread's two query rows
+  uint32_t qh[KS][4], ql[KS][4];
+#pragma unroll
+  for (int ks = 0; ks < KS; ++ks) {
+    const int c = 16 * ks + 2 * tig;
+    qh[ks][0] = *reinterpret_cast<const uint32_t*>(&Ks[ra][c]);
+    qh[ks][1] = *reinterpret_cast<const uint32_t*>(&Ks[rb][c]);
+    qh[ks][2] = *reinterpret_cast<const uint32_t*>(&Ks[ra][c + 8]);
+    qh[ks][3] = *reinterpret_cast<const uint32_t*>(&Ks[rb][c + 8]);
+    ql[ks][0] = *reinterpret_cast<const uint32_t*>(&Vs[ra][c]);
+    ql[ks][1] = *reinterpret_cast<const uint32_t*>(&Vs[rb][c]);
+    ql[ks][2] = *reinterpret_cast<const uint32_t*>(&Vs[ra][c + 8]);
+    ql[ks][3] = *reinterpret_cast<const uint32_t*>(&Vs[rb][c + 8]);
+  }
+  const int tok_a = t0 + ra / G, tok_b = t0 + rb / G;
+  const int lim_a = P + tok_a, lim_b = P + tok_b;  // causal limits
+  float o[ND][4];
+#pragma unroll
+  for (int nd = 0; nd < ND; ++nd) o[nd][0] = o[nd][1] = o[nd][2] = o[nd][3] = 0.f;
+  float m_a = -INFINITY, m_b = -INFINITY, l_a = 0.f, l_b = 0.f;
+  const int last = P + min(t0 + TB, S) - 1;  // the block's last token's limit
+  for (int j0 = 0; j0 <= last; j0 += 64) {
+    const int nj = min(64, last + 1 - j0);
+    __syncthreads();  // the previous tile (or the Q staging) is read
+    for (int e = tid; e < 64 * (D / 8); e += 128) {
+      const int r = e / (D / 8), c = e % (D / 8);
+      uint4 kv4 = make_uint4(0, 0, 0, 0), vv4 = kv4;
+      if (r < nj) {
+        const int sl = __ldg(bt_row + j0 + r);
+        const size_t off = (((size_t)(sl / cap) * Hkv + hk) * cap + sl % cap) * D;
+        kv4 = *reinterpret_cast<const uint4*>(kpool + off + 8 * c);
+        vv4 = *reinterpret_cast<const uint4*>(vpool + off + 8 * c);
+      }
+      *reinterpret_cast<uint4*>(&Ks[r][8 * c]) = kv4;
+      *reinterpret_cast<uint4*>(&Vs[r][8 * c]) = vv4;
+    }
+    if (tid < 64) vis[tid] = tid < nj && mask[j0 + tid] ? 1 : 0;
+    __syncthreads();
+    float sc[8][4];
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt) sc[nt][0] = sc[nt][1] = sc[nt][2] = sc[nt][3] = 0.f;
+#pragma unroll
+    for (int ks = 0; ks < KS; ++ks)
+#pragma unroll
+      for (int nt = 0; nt < 8; ++nt) {
+        const uint32_t b0 = *reinterpret_cast<const uint32_t*>(&Ks[8 * nt + gid][16 * ks + 2 * tig]);
+        const uint32_t b1 = *reinterpret_cast<const uint32_t*>(&Ks[8 * nt + gid][16 * ks + 8 + 2 * tig]);
+        mma16816(sc[nt], qh[ks], b0, b1);
+        mma16816(sc[nt], ql[ks], b0, b1);
+      }
+    // mask and scale; row maxima over the quad that shares a row
+    float mx_a = -INFINITY, mx_b = -INFINITY;
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt)
+#pragma unroll
+      for (int c = 0; c < 2; ++c) {
+        const int col = 8 * nt + 2 * tig + c, j = j0 + col;
+        sc[nt][c] = vis[col] && j <= lim_a ? sc[nt][c] * scale : -INFINITY;
+        sc[nt][2 + c] = vis[col] && j <= lim_b ? sc[nt][2 + c] * scale : -INFINITY;
+        mx_a = fmaxf(mx_a, sc[nt][c]);
+        mx_b = fmaxf(mx_b, sc[nt][2 + c]);
+      }
+#pragma unroll
+    for (int o_ = 1; o_ <= 2; o_ <<= 1) {
+      mx_a = fmaxf(mx_a, __shfl_xor_sync(0xffffffffu, mx_a, o_));
+      mx_b = fmaxf(mx_b, __shfl_xor_sync(0xffffffffu, mx_b, o_));
+    }
+    const float mn_a = fmaxf(m_a, mx_a), mn_b = fmaxf(m_b, mx_b);
+    const float al_a = m_a == -INFINITY ? 0.f : expf(m_a - mn_a), al_b = m_b == -INFINITY ? 0.f : expf(m_b - mn_b);
+    float su_a = 0.f, su_b = 0.f;
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt)
+#pragma unroll
+      for (int c = 0; c < 2; ++c) {
+        sc[nt][c] = sc[nt][c] == -INFINITY ? 0.f : expf(sc[nt][c] - mn_a);
+        sc[nt][2 + c] = sc[nt][2 + c] == -INFINITY ? 0.f : expf(sc[nt][2 + c] - mn_b);
+        su_a += sc[nt][c];
+        su_b += sc[nt][2 + c];
+      }
+#pragma unroll
+    for (int o_ = 1; o_ <= 2; o_ <<= 1) {
+      su_a += __shfl_xor_sync(0xffffffffu, su_a, o_);
+      su_b += __shfl_xor_sync(0xffffffffu, su_b, o_);
+    }
+    l_a = l_a * al_a + su_a;
+    l_b = l_b * al_b + su_b;
+    m_a = mn_a;
+    m_b = mn_b;
+#pragma unroll
+    for (int nd = 0; nd < ND; ++nd) {
+      o[nd][0] *= al_a;
+      o[nd][1] *= al_a;
+      o[nd][2] *= al_b;
+      o[nd][3] *= al_b;
+    }
+    // O += P V: the score accumulators of n-tiles 2 kk, 2 kk + 1 are the A
+    // fragment of entries 16 kk .. + 15
+#pragma unroll
+    for (int kk = 0; kk < 4; ++kk) {
+      uint32_t ph[4], pl[4];
+      split_h2(sc[2 * kk][0], sc[2 * kk][1], ph[0], pl[0]);
+      split_h2(sc[2 * kk][2], sc[2 * kk][3], ph[1], pl[1]);
+      split_h2(sc[2 * kk + 1][0], sc[2 * kk + 1][1], ph[2], pl[2]);
+      split_h2(sc[2 * kk + 1][2], sc[2 * kk + 1][3], ph[3], pl[3]);
+      const int mtx = lane >> 3, er = 16 * kk + 8 * (mtx & 1) + (lane & 7);
+#pragma unroll
+      for (int nd = 0; nd < ND; nd += 2) {
+        uint32_t v0, v1, v2, v3;
+        ldsm_x4_trans(&Vs[er][8 * (nd + (mtx >> 1))], v0, v1, v2, v3);
+        mma16816(o[nd], ph, v0, v1);
+        mma16816(o[nd], pl, v0, v1);
+        mma16816(o[nd + 1], ph, v2, v3);
+        mma16816(o[nd + 1], pl, v2, v3);
+      }
+    }
+  }
+  const float ia = l_a > 0.f ? 1.f / l_a : 0.f, ib = l_b > 0.f ? 1.f / l_b : 0.f;
+#pragma unroll
+  for (int nd = 0; nd < ND; ++nd)
+#pragma unroll
+    for (int c = 0; c < 2; ++c) {
+      const int dcol = 8 * nd + 2 * tig + c;
+      if (tok_a < S) out[(size_t)tok_a * out_ld + (hk * G + ra % G) * D + dcol] = f2h(o[nd][c] * ia);
+      if (tok_b < S) out[(size_t)tok_b * out_ld + (hk * G + rb % G) * D + dcol] = f2h(o[nd][2 + c] * ib);
+    }
+}
+
 template <int D, int G>
 cudaError_t launch_attn_t(const PrefillLayerArgs& a, cudaStream_t s) {
-  prefill_attention_kernel<D, G><<<dim3(a.S, a.Hkv), D, 0, s>>>(a.q, a.Hq, a.Hkv, a.kpool, a.vpool, a.bt_row, a.cap,
-                                                                 a.mask, a.P, a.attn, a.attn_ld);
+  if (64 % G == 0) {
+    prefill_flash_kernel<D, G><<<dim3((a.S + 64 / G - 1) / (64 / G), a.Hkv), 128, 0, s>>>(
+        a.q, a.Hq, a.Hkv, a.kpool, a.vpool, a.bt_row, a.cap, a.mask, a.P, a.S, a.attn, a.attn_ld);
+  } else {
+    prefill_attention_kernel<D, G><<<dim3(a.S, a.Hkv), D, 0, s>>>(a.q, a.Hq, a.Hkv, a.kpool, a.vpool, a.bt_row,
+                                                                   a.cap, a.mask, a.P, a.attn, a.attn_ld);
+  }
   return cudaGetLastError();
 }
 

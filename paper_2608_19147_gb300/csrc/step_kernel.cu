@@ -122,7 +122,7 @@ struct GridBarrier {
           break;
         }
         if ((it & 1023) == 0 && (*reinterpret_cast<volatile int*>(status) & ST_WAIT_TIMEOUT)) break;
-        __nanosleep(64);
+        __nanosleep(16);
       }
       if (blockIdx.x == 0) clock[n_wait + 1] = globaltimer();
     }
