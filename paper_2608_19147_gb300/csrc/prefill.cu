@@ -11,11 +11,6 @@
 namespace shard {
 namespace {
 
-__device__ __forceinline__ float2 h2f2p(uint32_t u) {
-  __half2 h;
-  memcpy(&h, &u, sizeof(h));
-  return __half22float2(h);
-}
 
 // Device-side argument checks (values that live on the device): token ids in
 // [0, vocab), positions in [0, max_position), the mask open at every new
@@ -108,94 +103,6 @@ __global__ void prefill_rope_append_kernel(const float* y, int y_ld, int S, int 
   }
 }
 
-// Causal attention of the new tokens: CTA (token t, kv head hk), d threads
-// (thread = head dimension).  Entries j <= P + t of the row with mask[j] != 0,
-// read through the beam table; key tiles of 64 with an online softmax per
-// query head.
-constexpr int kPfTile = 64;
-template <int D, int G>
-__global__ void __launch_bounds__(D) prefill_attention_kernel(const float* q, int Hq, int Hkv, const uint16_t* kpool,
-                                                              const uint16_t* vpool, const int* bt_row, int cap,
-                                                              const uint8_t* mask, int P, uint16_t* out, int out_ld) {
-  __shared__ float qs[G][D];
-  __shared__ uint16_t Ks[kPfTile][D + 8];
-  __shared__ uint16_t Vs[kPfTile][D];
-  __shared__ float sc[G][kPfTile];
-  __shared__ float s_m[G], s_l[G], s_alpha[G];
-  const int t = blockIdx.x, hk = blockIdx.y, tid = threadIdx.x, warp = tid / 32, lane = tid % 32;
-  const int n_warps = D / 32;
-  for (int g = 0; g < G; ++g) qs[g][tid] = q[(size_t)t * Hq * D + (hk * G + g) * D + tid];
-  if (tid < G) {
-    s_m[tid] = -INFINITY;
-    s_l[tid] = 0.f;
-  }
-  float acc[G];
-#pragma unroll
-  for (int g = 0; g < G; ++g) acc[g] = 0.f;
-  const int last = P + t;  // causal limit
-  const float scale = rsqrtf((float)D);
-  for (int j0 = 0; j0 <= last; j0 += kPfTile) {
-    const int nj = min(kPfTile, last + 1 - j0);
-    __syncthreads();
-    for (int e = tid; e < kPfTile * (D / 8); e += D) {
-      const int r = e / (D / 8), c = e % (D / 8);
-      uint4 kv4 = make_uint4(0, 0, 0, 0), vv4 = kv4;
-      if (r < nj) {
-        const int sl = __ldg(bt_row + j0 + r);
-        const size_t off = (((size_t)(sl / cap) * Hkv + hk) * cap + sl % cap) * D;
-        kv4 = *reinterpret_cast<const uint4*>(kpool + off + 8 * c);
-        vv4 = *reinterpret_cast<const uint4*>(vpool + off + 8 * c);
-      }
-      *reinterpret_cast<uint4*>(&Ks[r][8 * c]) = kv4;
-      *reinterpret_cast<uint4*>(&Vs[r][8 * c]) = vv4;
-    }
-    __syncthreads();
-    for (int e = tid; e < G * kPfTile; e += D) {
-      const int g = e / kPfTile, r = e % kPfTile;
-      float s = -INFINITY;
-      if (r < nj && mask[j0 + r]) {
-        float dot = 0.f;
-        for (int c = 0; c < D; c += 2) {
-          const float2 kf = h2f2p(*reinterpret_cast<const uint32_t*>(&Ks[r][c]));
-          dot = fmaf(qs[g][c], kf.x, dot);
-          dot = fmaf(qs[g][c + 1], kf.y, dot);
-        }
-        s = dot * scale;
-      }
-      sc[g][r] = s;
-    }
-    __syncthreads();
-    for (int g = warp; g < G; g += n_warps) {
-      float mx = fmaxf(sc[g][lane], sc[g][lane + 32]);
-      for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-      const float m_new = fmaxf(s_m[g], mx);
-      float p0 = 0.f, p1 = 0.f;
-      if (m_new != -INFINITY) {
-        p0 = sc[g][lane] == -INFINITY ? 0.f : expf(sc[g][lane] - m_new);
-        p1 = sc[g][lane + 32] == -INFINITY ? 0.f : expf(sc[g][lane + 32] - m_new);
-      }
-      sc[g][lane] = p0;
-      sc[g][lane + 32] = p1;
-      float ps = p0 + p1;
-      for (int o = 16; o > 0; o >>= 1) ps += __shfl_xor_sync(0xffffffffu, ps, o);
-      if (lane == 0) {
-        const float alpha = s_m[g] == -INFINITY ? 0.f : expf(s_m[g] - m_new);
-        s_alpha[g] = alpha;
-        s_l[g] = s_l[g] * alpha + ps;
-        s_m[g] = m_new;
-      }
-    }
-    __syncthreads();
-#pragma unroll
-    for (int g = 0; g < G; ++g) {
-      float a = acc[g] * s_alpha[g];
-      for (int r = 0; r < nj; ++r) a = fmaf(sc[g][r], h2f(Vs[r][tid]), a);
-      acc[g] = a;
-    }
-  }
-#pragma unroll
-  for (int g = 0; g < G; ++g) out[(size_t)t * out_ld + (hk * G + g) * D + tid] = f2h(acc[g] / s_l[g]);
-}
 
 // h[t][j] = fp16(silu(gate) * up); y holds gate (0..F) then up (F..2F).
 __global__ void prefill_swiglu_kernel(const float* y, int y_ld, int S, int F, uint16_t* h, int h_ld) {
@@ -398,13 +305,9 @@ __global__ void __launch_bounds__(128) prefill_flash_kernel(const float* q, int 
 
 template <int D, int G>
 cudaError_t launch_attn_t(const PrefillLayerArgs& a, cudaStream_t s) {
-  if (64 % G == 0) {
-    prefill_flash_kernel<D, G><<<dim3((a.S + 64 / G - 1) / (64 / G), a.Hkv), 128, 0, s>>>(
-        a.q, a.Hq, a.Hkv, a.kpool, a.vpool, a.bt_row, a.cap, a.mask, a.P, a.S, a.attn, a.attn_ld);
-  } else {
-    prefill_attention_kernel<D, G><<<dim3(a.S, a.Hkv), D, 0, s>>>(a.q, a.Hq, a.Hkv, a.kpool, a.vpool, a.bt_row,
-                                                                   a.cap, a.mask, a.P, a.attn, a.attn_ld);
-  }
+  static_assert(64 % G == 0, "64 query rows per CTA");
+  prefill_flash_kernel<D, G><<<dim3((a.S + 64 / G - 1) / (64 / G), a.Hkv), 128, 0, s>>>(
+      a.q, a.Hq, a.Hkv, a.kpool, a.vpool, a.bt_row, a.cap, a.mask, a.P, a.S, a.attn, a.attn_ld);
   return cudaGetLastError();
 }
 
