@@ -4,8 +4,9 @@
 // same rounding points (fp16 normalised activations, attention output,
 // SwiGLU output, appended K/V and the output), causal attention among the new
 // tokens and over the row's unmasked cache.  The projections are dense
-// contractions here and run on the tensor cores (gemm_tc.cu); the rest are
-// small per-token kernels, launched layer by layer on the caller's stream.
+// contractions here and run on the tensor cores (gemm_tc.cu), the attention on
+// mma.sync over blocks of tokens (prefill_flash_kernel); the rest are small
+// per-token kernels, launched layer by layer on the caller's stream.
 #include "common.cuh"
 
 namespace shard {
