@@ -214,6 +214,49 @@ cudaError_t reset_work_buffers(shard_s* sh) {
   return e;
 }
 
+// Frees everything a shard holds -- its kv states, device buffers and pinned
+// staging -- and the shard itself, on the current device after its work has
+// finished.  Buffers never allocated are null and skipped, so this also
+// undoes a shard_create that failed part-way.
+void release_shard(shard_s* sh) {
+  cudaDeviceSynchronize();
+  for (auto* st : sh->states) free_state(st);
+  cudaFree(sh->weight_pool);
+  cudaFree(sh->norms);
+  cudaFree(sh->embedding);
+  cudaFree(sh->rope);
+  cudaFree(sh->pf_x);
+  cudaFree(sh->pf_act);
+  cudaFree(sh->pf_attn);
+  cudaFree(sh->pf_h);
+  cudaFree(sh->pf_y);
+  cudaFree(sh->pf_q);
+  cudaFree(sh->X);
+  cudaFree(sh->acc_qkv);
+  cudaFree(sh->acc_gu);
+  cudaFree(sh->acc_store);
+  cudaFree(sh->cnt_kv);
+  cudaFree(sh->cnt_gu);
+  cudaFree(sh->cnt_store);
+  cudaFree(sh->attn_cnt);
+  cudaFree(sh->act_h);
+  cudaFree(sh->act_attn);
+  cudaFree(sh->act_f);
+  cudaFree(sh->status);
+  cudaFree(sh->exit_count);
+  cudaFree(sh->dstage);
+  if (sh->pin) cudaFreeHost(sh->pin);
+  if (sh->status_host) cudaFreeHost(sh->status_host);
+  cudaFree(sh->ops_dev);
+  cudaFree(sh->barrier);
+  cudaFree(sh->phase_clock);
+  delete sh;
+}
+
+struct ShardRelease {
+  void operator()(shard_s* sh) const { release_shard(sh); }
+};
+
 int check_pending_status(shard_s* sh) {
   const int bits = *reinterpret_cast<volatile int*>(sh->status_host);
   if (bits) {
@@ -249,7 +292,8 @@ int shard_create(const shard_config* cfg, const shard_weights_host* w, shard_t* 
   if (c.n_heads / c.n_kv_heads * kMaxTokens > 256) return fail(SHARD_EUNSUPPORTED, "n_heads / n_kv_heads must be <= 16");
   if (c.vocab > 0 && !w->embedding) return fail(SHARD_EINVAL, "vocab > 0 needs an embedding");
 
-  auto sh = std::unique_ptr<shard_s>(new shard_s());
+  // a failure below returns through the deleter, which frees what was allocated so far
+  auto sh = std::unique_ptr<shard_s, ShardRelease>(new shard_s());
   CUDA_TRY(cudaGetDevice(&sh->device));
   CUDA_TRY(cudaDeviceGetAttribute(&sh->num_sms, cudaDevAttrMultiProcessorCount, sh->device));
   if (c.head_dim != 64 && c.head_dim != 128) return fail(SHARD_EUNSUPPORTED, "head_dim must be 64 or 128");
@@ -435,38 +479,7 @@ int shard_create(const shard_config* cfg, const shard_weights_host* w, shard_t* 
 int shard_destroy(shard_t sh) {
   if (!sh) return fail(SHARD_EINVAL, "shard_destroy: null shard");
   cudaSetDevice(sh->device);
-  cudaDeviceSynchronize();
-  for (auto* st : sh->states) free_state(st);
-  cudaFree(sh->weight_pool);
-  cudaFree(sh->norms);
-  cudaFree(sh->embedding);
-  cudaFree(sh->rope);
-  cudaFree(sh->pf_x);
-  cudaFree(sh->pf_act);
-  cudaFree(sh->pf_attn);
-  cudaFree(sh->pf_h);
-  cudaFree(sh->pf_y);
-  cudaFree(sh->pf_q);
-  cudaFree(sh->X);
-  cudaFree(sh->acc_qkv);
-  cudaFree(sh->acc_gu);
-  cudaFree(sh->acc_store);
-  cudaFree(sh->cnt_kv);
-  cudaFree(sh->cnt_gu);
-  cudaFree(sh->cnt_store);
-  cudaFree(sh->attn_cnt);
-  cudaFree(sh->act_h);
-  cudaFree(sh->act_attn);
-  cudaFree(sh->act_f);
-  cudaFree(sh->status);
-  cudaFree(sh->exit_count);
-  cudaFree(sh->dstage);
-  if (sh->pin) cudaFreeHost(sh->pin);
-  if (sh->status_host) cudaFreeHost(sh->status_host);
-  cudaFree(sh->ops_dev);
-  cudaFree(sh->barrier);
-  cudaFree(sh->phase_clock);
-  delete sh;
+  release_shard(sh);
   return SHARD_OK;
 }
 
