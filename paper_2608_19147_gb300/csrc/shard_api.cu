@@ -606,7 +606,8 @@ int kv_state_read(kvstate_t st, int row, int layer, int start, int len, uint16_t
   int cur = 0;
   int rc = kv_state_length(st, row, &cur);
   if (rc) return rc;
-  if (start + len > cur) return fail(SHARD_EINVAL, "kv_state_read: [%d, %d) beyond row length %d", start, start + len, cur);
+  if ((long long)start + len > cur)
+    return fail(SHARD_EINVAL, "kv_state_read: [%d, %d + %d) beyond row length %d", start, start, len, cur);
   if (len == 0) return SHARD_OK;
   DevBuf<uint16_t> tmp;
   CUDA_TRY(tmp.alloc((size_t)len * sh->Hkv * sh->d));
@@ -733,7 +734,8 @@ static int step_impl(shard_t sh, kvstate_t st, const uint16_t* hidden_in, const 
   if (mask_stride < 1) return fail(SHARD_EINVAL, "shard_step: mask_stride must be >= 1");
   int M = 0, maxn = 0;
   for (int b = 0; b < B; ++b) {
-    if (n_new[b] < 1) return fail(SHARD_EINVAL, "shard_step: n_new[%d] = %d < 1", b, n_new[b]);
+    if (n_new[b] < 1 || n_new[b] > SHARD_MAX_TOKENS)
+      return fail(SHARD_EINVAL, "shard_step: n_new[%d] = %d outside [1, %d]", b, n_new[b], SHARD_MAX_TOKENS);
     M += n_new[b];
     maxn = std::max(maxn, n_new[b]);
   }
@@ -855,22 +857,43 @@ int shard_prefill(shard_t sh, kvstate_t st, int row, const uint16_t* hidden_in, 
   if (rc) return rc;
   const int P = st->len_host[row];
   if (st->cursor[row] != P) return fail(SHARD_EINVAL, "shard_prefill: row %d is not contiguous", row);
-  if (P + S > st->cap) return fail(SHARD_ECAPACITY, "shard_prefill: %d + %d entries > capacity %d", P, S, st->cap);
+  if ((long long)P + S > st->cap)
+    return fail(SHARD_ECAPACITY, "shard_prefill: %d + %d entries > capacity %d", P, S, st->cap);
   if (mask_len < P + S) return fail(SHARD_EINVAL, "shard_prefill: mask_len %d < %d", mask_len, P + S);
   CUDA_TRY(cudaSetDevice(sh->device));
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
   const int C = kPrefillChunk;
   const int y_rows = std::max(std::max(sh->dq + 2 * sh->dkv, 2 * sh->F), sh->H);
   if (!sh->pf_x) {
-    CUDA_TRY(cudaMalloc(&sh->pf_x, sizeof(float) * C * sh->H));
-    CUDA_TRY(cudaMalloc(&sh->pf_act, sizeof(uint16_t) * C * sh->Kp_H));
-    CUDA_TRY(cudaMalloc(&sh->pf_attn, sizeof(uint16_t) * C * sh->Kp_dq));
-    CUDA_TRY(cudaMalloc(&sh->pf_h, sizeof(uint16_t) * C * sh->Kp_F));
-    CUDA_TRY(cudaMalloc(&sh->pf_y, sizeof(float) * C * y_rows));
-    CUDA_TRY(cudaMalloc(&sh->pf_q, sizeof(float) * C * sh->dq));
-    CUDA_TRY(cudaMemset(sh->pf_act, 0, sizeof(uint16_t) * C * sh->Kp_H));
-    CUDA_TRY(cudaMemset(sh->pf_attn, 0, sizeof(uint16_t) * C * sh->Kp_dq));
-    CUDA_TRY(cudaMemset(sh->pf_h, 0, sizeof(uint16_t) * C * sh->Kp_F));
+    // all or none: a call that fails here leaves no partial set behind for
+    // the next call to mistake for a complete one
+    float *x = nullptr, *y = nullptr, *q = nullptr;
+    uint16_t *act = nullptr, *attn = nullptr, *hh = nullptr;
+    cudaError_t e = cudaMalloc(&x, sizeof(float) * C * sh->H);
+    if (e == cudaSuccess) e = cudaMalloc(&act, sizeof(uint16_t) * C * sh->Kp_H);
+    if (e == cudaSuccess) e = cudaMalloc(&attn, sizeof(uint16_t) * C * sh->Kp_dq);
+    if (e == cudaSuccess) e = cudaMalloc(&hh, sizeof(uint16_t) * C * sh->Kp_F);
+    if (e == cudaSuccess) e = cudaMalloc(&y, sizeof(float) * C * y_rows);
+    if (e == cudaSuccess) e = cudaMalloc(&q, sizeof(float) * C * sh->dq);
+    if (e == cudaSuccess) e = cudaMemset(act, 0, sizeof(uint16_t) * C * sh->Kp_H);
+    if (e == cudaSuccess) e = cudaMemset(attn, 0, sizeof(uint16_t) * C * sh->Kp_dq);
+    if (e == cudaSuccess) e = cudaMemset(hh, 0, sizeof(uint16_t) * C * sh->Kp_F);
+    if (e != cudaSuccess) {
+      cudaFree(x);
+      cudaFree(act);
+      cudaFree(attn);
+      cudaFree(hh);
+      cudaFree(y);
+      cudaFree(q);
+      return fail(e == cudaErrorMemoryAllocation ? SHARD_ENOMEM : SHARD_ECUDA, "shard_prefill: work buffers: %s",
+                  cudaGetErrorString(e));
+    }
+    sh->pf_x = x;
+    sh->pf_act = act;
+    sh->pf_attn = attn;
+    sh->pf_h = hh;
+    sh->pf_y = y;
+    sh->pf_q = q;
   }
   CUDA_TRY(launch_prefill_check(token_ids, sh->cfg.vocab, position_ids, sh->cfg.max_position, attention_mask, P, S,
                                 sh->status, s));
@@ -946,8 +969,12 @@ int shard_step_host(shard_t sh, kvstate_t st, const uint16_t* hidden_in, const i
     return fail(SHARD_EINVAL, "shard_step_host: null argument");
   if (B < 1 || B > SHARD_MAX_REQUESTS || mask_stride < 1) return fail(SHARD_EINVAL, "shard_step_host: bad B or mask_stride");
   int M = 0;
-  for (int b = 0; b < B; ++b) M += n_new[b] > 0 ? n_new[b] : 0;
-  if (M < 1 || M > SHARD_MAX_TOKENS) return fail(SHARD_EINVAL, "shard_step_host: bad token count");
+  for (int b = 0; b < B; ++b) {
+    if (n_new[b] < 1 || n_new[b] > SHARD_MAX_TOKENS)
+      return fail(SHARD_EINVAL, "shard_step_host: n_new[%d] = %d outside [1, %d]", b, n_new[b], SHARD_MAX_TOKENS);
+    M += n_new[b];
+  }
+  if (M > SHARD_MAX_TOKENS) return fail(SHARD_EINVAL, "shard_step_host: %d new tokens > %d", M, SHARD_MAX_TOKENS);
   CUDA_TRY(cudaSetDevice(sh->device));
   const size_t b_hid = hidden_in ? sizeof(uint16_t) * M * sh->H : 0;
   const size_t b_tok = token_ids ? sizeof(int32_t) * M : 0;
@@ -961,12 +988,14 @@ int shard_step_host(shard_t sh, kvstate_t st, const uint16_t* hidden_in, const i
   if (sh->pin_bytes < need) {
     if (sh->pin) cudaFreeHost(sh->pin);
     sh->pin = nullptr;
+    sh->pin_bytes = 0;  // a failed allocation leaves no stale size behind
     CUDA_TRY(cudaHostAlloc(&sh->pin, need, cudaHostAllocDefault));
     sh->pin_bytes = need;
   }
   if (sh->dstage_bytes < need) {
     cudaFree(sh->dstage);
     sh->dstage = nullptr;
+    sh->dstage_bytes = 0;
     CUDA_TRY(cudaMalloc(&sh->dstage, need));
     sh->dstage_bytes = need;
   }
