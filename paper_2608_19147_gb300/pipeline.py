@@ -140,13 +140,23 @@ def _recv_from_peer(src: int, hidden: int) -> Optional[_Msg]:
 def run_stage_rank(stage: StageFn, hidden: int) -> int:
     """Loop of a non-coordinating rank r > 0: receive from r - 1, run the
     stage, send to r + 1 (the last rank sends back to rank 0), until the
-    coordinator's stop message comes through.  Returns the number of steps run."""
+    coordinator's stop message comes through.  Returns the number of steps run.
+    If the upstream peer is lost, the results already computed are still
+    delivered downstream (as far as that peer is alive) before PeerLost
+    propagates, so the coordinator keeps every step that completed."""
     rank, world = dist.get_rank(), dist.get_world_size()
     src, dst = rank - 1, (rank + 1) % world
     sends = _Sends()
     n = 0
     while True:
-        msg = _recv_from_peer(src, hidden)
+        try:
+            msg = _recv_from_peer(src, hidden)
+        except PeerLost:
+            try:
+                sends.finish()
+            except RuntimeError:
+                pass
+            raise
         if msg is None:
             if dst != 0:
                 _send_stop(dst, sends)
