@@ -17,6 +17,12 @@ far larger than L2, so no L2 flush is needed between steps.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl gb300|reference]
                   [--config 8b-decode|8b-verify|8b-microbatch|70b-decode|70b-verify|tiny|8b-head|8b-head-verify|8b-prefill]
+                  [--no-cpu-baseline] [--no-other-workloads] [--layers N]
+
+At one GPU the default (8b-decode) line also carries `other_workloads`: the
+8B verify and micro-batch and the 70B decode and verify workloads, each run
+afterwards as `bench.py --config <name>` in a child process of its own, with
+its value, step time and roofline fraction.
 
 Under torchrun each rank runs an independent replica on its own GPU
 (replicas only: the path has no exchange step) and rank 0 prints one JSON
@@ -514,11 +520,62 @@ def run_gpu(args, rank: int, world: int):
         "gpu_launches": K * launches_per_step,
         "clocks": clocks,
     }
+    if want_other_workloads(args, world):
+        log("measuring the other step workloads in child processes")
+        result["other_workloads"] = other_workloads()
     if world == 1 and not args.no_cpu_baseline:
         result["cpu_baseline"] = cpu_baseline(args.config, weights, budget_s=args.cpu_budget)
     print(json.dumps(result), flush=True)
     if dist:
         dist.destroy_process_group()
+
+
+# The other step workloads, measured by this script in child processes after
+# the main line's timed region, so that one default run reports every shard
+# workload; each child is `bench.py --config <name>` with its own timing.
+OTHER_WORKLOADS = (("70b-decode", 64), ("8b-verify", 128), ("8b-microbatch", 64), ("70b-verify", 64))
+LAUNCHER_ENV = ("RANK", "WORLD_SIZE", "LOCAL_RANK", "LOCAL_WORLD_SIZE", "GROUP_RANK", "ROLE_RANK", "ROLE_WORLD_SIZE",
+                "GROUP_WORLD_SIZE", "MASTER_ADDR", "MASTER_PORT")
+
+
+def want_other_workloads(args, world: int) -> bool:
+    return (world == 1 and args.config == "8b-decode" and args.layers == 0 and not args.no_cpu_baseline
+            and not args.no_other_workloads)
+
+
+def _child_cmd(cfg: str, steps: int):
+    return [sys.executable, os.path.abspath(__file__), "--config", cfg, "--steps", str(steps), "--warmup", "3",
+            "--no-cpu-baseline"]
+
+
+def _child_env():
+    return {k: v for k, v in os.environ.items() if k not in LAUNCHER_ENV and not k.startswith("TORCHELASTIC_")}
+
+
+def other_workloads(timeout_s: float = 300.0) -> dict:
+    """Runs each of OTHER_WORKLOADS in a child process of its own and returns
+    its headline figures (or the reason it gave none): a child that fails
+    cannot disturb the main line, which is complete before they start."""
+    out = {}
+    for cfg, steps in OTHER_WORKLOADS:
+        t0 = time.time()
+        try:
+            r = subprocess.run(_child_cmd(cfg, steps), capture_output=True, text=True, timeout=timeout_s,
+                               env=_child_env())
+            lines = [ln for ln in r.stdout.splitlines() if ln.startswith("{")]
+            if r.returncode != 0 or not lines:
+                tail = (r.stderr.strip().splitlines() or ["no output"])[-1]
+                out[cfg] = {"error": "exit %d: %s" % (r.returncode, tail[:300])}
+                continue
+            d = json.loads(lines[-1])
+            rf = d["roofline"]
+            out[cfg] = {"workload": d["config"]["workload"], "value": d["value"], "unit": d["unit"],
+                        "ms_per_step": d["ms_per_step"], "steps": d["steps"], "achieved_gbs": rf["achieved"],
+                        "frac": rf["frac"], "peak": rf["peak"], "e2e": d["e2e"]["value"], "clocks": d["clocks"],
+                        "gpu_launches": d["gpu_launches"], "wall_s": round(time.time() - t0, 1)}
+        except Exception as e:  # timeout, unparsable output
+            out[cfg] = {"error": "%s: %s" % (type(e).__name__, str(e)[:300])}
+    return out
 
 
 # ---------------------------------------------------------------------------
@@ -985,7 +1042,10 @@ def main():
     ap.add_argument("--warmup", type=int, default=16)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--config", default="8b-decode", choices=list(CONFIGS))
-    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true",
+                    help="the workload's own line only: no CPU oracle leg and no other workloads")
+    ap.add_argument("--no-other-workloads", action="store_true",
+                    help="8b-decode at 1 GPU: skip measuring the other step workloads after the main line")
     ap.add_argument("--cpu-budget", type=float, default=20.0)
     ap.add_argument("--layers", type=int, default=0,
                     help="run only the stage's first N layers (profiling captures); default: the whole stage")
