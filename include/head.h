@@ -68,8 +68,10 @@ int head_destroy(head_t head);
  *   p_max   dev fp32 [M]: its softmax probability, or NULL
  * Does not synchronise.  Errors: EINVAL (M out of range, null hidden or
  * token), ECUDA.  A bounded device wait of the projection that gave up
- * (never expected) makes every row's token -1 and p_max NaN;
- * head_top1_host turns that into ECUDA. */
+ * (never expected) makes every row's token -1 and p_max NaN, and leaves the
+ * head's internal partial sums dirty: head_top1_host turns that into ECUDA
+ * and clears them; a head_top1 caller that reads a -1 token should destroy
+ * the head and create it again. */
 int head_top1(head_t head, const uint16_t* hidden, int M, int32_t* token, float* p_max, void* cuda_stream);
 
 /* head_top1 with host buffers: copies hidden (host fp16 [M][hidden]) to the

@@ -464,7 +464,11 @@ int head_top1_host(head_t h, const uint16_t* hidden, int M, int32_t* token, floa
   HEAD_CUDA_TRY(cudaStreamSynchronize(s));
   for (int m = 0; m < M; ++m)
     if (token[m] < 0) {
+      // a projection that gave up leaves partial sums and row-block counts
+      // behind: clear them with the status so the next call starts clean
       cudaMemsetAsync(h->status, 0, sizeof(int), s);
+      cudaMemsetAsync(h->acc, 0, sizeof(long long) * kMaxTokens * h->op.n_rb * kRowsPerBlock, s);
+      cudaMemsetAsync(h->cnt, 0, sizeof(int) * h->op.n_rb, s);
       cudaStreamSynchronize(s);
       return fail(SHARD_ECUDA, "head_top1_host: a device wait of the projection timed out");
     }
