@@ -418,12 +418,12 @@ int shard_create(const shard_config* cfg, const shard_weights_host* w, shard_t* 
   }
   {
     // cos/sin of pos * theta^(-2i/d), computed in double, stored as fp32.
-    const int half = sh->d / 2;
-    std::vector<float2> tab((size_t)c.max_position * half);
+    const int pairs = sh->d / 2;
+    std::vector<float2> tab((size_t)c.max_position * pairs);
     for (int p = 0; p < c.max_position; ++p)
-      for (int i = 0; i < half; ++i) {
+      for (int i = 0; i < pairs; ++i) {
         const double ang = (double)p * std::pow(c.rope_theta, -2.0 * i / sh->d);
-        tab[(size_t)p * half + i] = make_float2((float)std::cos(ang), (float)std::sin(ang));
+        tab[(size_t)p * pairs + i] = make_float2((float)std::cos(ang), (float)std::sin(ang));
       }
     CUDA_TRY(cudaMalloc(&sh->rope, sizeof(float2) * tab.size()));
     CUDA_TRY(cudaMemcpy(sh->rope, tab.data(), sizeof(float2) * tab.size(), cudaMemcpyHostToDevice));
