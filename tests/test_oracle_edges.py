@@ -11,6 +11,9 @@
   beam_idx gather among them) and as one request of 16 tokens, equals the
   same requests run one at a time, bit for bit (Section 8.6's
   batch-composition invariance at the size limit).
+- Arbitrary hole patterns (Section 5.2): holes anywhere in the cache and any
+  subset of each step's new entries rejected give the same bits as a cache
+  with exactly those entries deleted.
 """
 import dataclasses
 
@@ -107,3 +110,36 @@ def test_one_request_of_sixteen_tokens_equals_sixteen_single_steps(weights):
         ka, va = block.read(0, layer, 0, P + n)
         kb, vb = one.read(0, layer, 0, P + n)
         assert np.array_equal(ka, kb) and np.array_equal(va, vb)
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_arbitrary_holes_equal_physical_trim(weights, seed):
+    # holes anywhere in the cache -- not only rejected-draft suffixes -- and
+    # any subset of each step's new entries rejected afterwards: the masked
+    # run equals a run whose cache had exactly those entries deleted, bit for
+    # bit in fp64 and in fp16 (Section 5.2's exactness, for every hole pattern)
+    rng = np.random.default_rng(seed)
+    P = int(rng.integers(8, 40))
+    keep = rng.random(P) >= 0.3
+    keep[rng.integers(P)] = False  # at least one hole
+    masked = OracleEngine(TINY, weights, 1, 96)
+    trimmed = OracleEngine(TINY, weights, 1, 96)
+    prefill(masked, TINY, SEED + seed, 0, P)
+    prefill(trimmed, TINY, SEED + seed, 0, P)
+    trimmed.trim(0, keep.astype(np.uint8))
+    valid = keep.astype(np.uint8).tolist()
+    pos = P
+    for step in range(4):
+        n = int(rng.integers(1, 5))
+        h = synth.hidden_in(TINY, SEED + seed, step, n)
+        positions = np.arange(pos, pos + n, dtype=np.int32)
+        om = masked.step([n], positions, np.array(valid + [1] * n, np.uint8), hidden_in=h)
+        ot = trimmed.step([n], positions, np.ones(sum(valid) + n, np.uint8), hidden_in=h)
+        assert np.array_equal(om, ot), step
+        assert np.array_equal(masked.last_f64, trimmed.last_f64), step
+        new_keep = (rng.random(n) >= 0.4).astype(np.uint8)
+        valid += new_keep.tolist()
+        trimmed.trim(0, np.concatenate([np.ones(trimmed.length(0) - n, np.uint8), new_keep]))
+        pos += n
+    assert masked.length(0) == len(valid) and trimmed.length(0) == sum(valid)
+    assert sum(valid) < len(valid)
