@@ -141,12 +141,16 @@ class Plan:
                     step["tokens"] = synth.token_ids(s, seed, t, self.M)
                 else:
                     step["hidden"] = synth.hidden_in(s, seed, t, self.M)
-                kv_read = 0
+                kv_read = kv_phys = 0
                 for b in range(self.B):
                     # K and V of the entries attention must read: the live
                     # cache entries and the new ones, in every layer
                     kv_read += (sum(valid[b]) + self.n) * s.kv_bytes_per_token() * s.n_layers
+                    # and of every physical entry, masked holes included
+                    kv_phys += (lens[b] + self.n) * s.kv_bytes_per_token() * s.n_layers
                 step["kv_bytes"] = kv_read
+                step["kv_phys_bytes"] = kv_phys
+                step["entries"] = (sum(lens) + self.B * self.n, sum(sum(v) for v in valid) + self.B * self.n)
                 self.steps.append(step)
                 acc = self.n
                 if self.n > 1:
@@ -168,6 +172,17 @@ class Plan:
         io = self.M * s.hidden * 2 * 2
         norms = s.n_layers * 2 * s.hidden * 2
         return self.weight_bytes() + self.steps[t]["kv_bytes"] + io + norms
+
+    def kv_summary(self, K: int) -> dict:
+        """KV read per step counted twice (valid entries, as in the
+        algorithmic bytes, and physical entries including masked holes), and
+        the cache bloat: the step's physical entries over its valid ones
+        (cache plus new entries), mean over the steps and at the last step."""
+        st = self.steps[:K]
+        ratios = [phys / val for phys, val in (x["entries"] for x in st)]
+        return {"valid_bytes_per_step": sum(x["kv_bytes"] for x in st) / K,
+                "physical_bytes_per_step": sum(x["kv_phys_bytes"] for x in st) / K,
+                "cache_bloat_mean": sum(ratios) / K, "cache_bloat_last": ratios[-1]}
 
     def kind_bytes(self, kind: str) -> int:
         """Algorithmic bytes of one launch of a projection kind."""
@@ -502,6 +517,7 @@ def run_gpu(args, rank: int, world: int):
             "seed": SEED,
         },
         "step_alg_bytes": step_bytes,
+        "kv": plan.kv_summary(K),
         "roofline": {
             "kernel": "step_kernel (the whole decode step: %d layers in one launch)" % shape.n_layers,
             "bound": "hbm",
@@ -572,7 +588,7 @@ def other_workloads(timeout_s: float = 300.0) -> dict:
             out[cfg] = {"workload": d["config"]["workload"], "value": d["value"], "unit": d["unit"],
                         "ms_per_step": d["ms_per_step"], "steps": d["steps"], "achieved_gbs": rf["achieved"],
                         "frac": rf["frac"], "peak": rf["peak"], "e2e": d["e2e"]["value"], "clocks": d["clocks"],
-                        "gpu_launches": d["gpu_launches"], "wall_s": round(time.time() - t0, 1)}
+                        "gpu_launches": d["gpu_launches"], "kv": d.get("kv"), "wall_s": round(time.time() - t0, 1)}
         except Exception as e:  # timeout, unparsable output
             out[cfg] = {"error": "%s: %s" % (type(e).__name__, str(e)[:300])}
     return out

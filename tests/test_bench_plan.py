@@ -18,7 +18,9 @@ divides by (no GPU).
   gather-lineage semantics (Section 4: row b continues the sequence that row
   beam_idx[b] held).
 - The KV term of the algorithmic bytes counts the entries attention must
-  read (valid cache entries plus the new ones), never masked holes.
+  read (valid cache entries plus the new ones), never masked holes; the line
+  also reports the physical count, holes included, and the cache bloat
+  (physical over valid entries) that mask-based rewind costs.
 """
 import numpy as np
 import pytest
@@ -141,3 +143,23 @@ def test_tiny_and_70b_plans():
     p70 = bench.Plan("70b-verify", 3, bench.SEED)
     assert p70.M == 5 and p70.steps[0]["hidden"].shape == (5, 8192)
     assert p70.steps[0]["kv_bytes"] == (4096 + 5) * KV_ENTRY_BYTES * 20
+
+
+def test_kv_counted_valid_and_physical_with_cache_bloat():
+    # decode and micro-batch have no holes: both counts agree, no bloat
+    for cfg, K in (("8b-decode", 256), ("8b-microbatch", 64)):
+        k = bench.Plan(cfg, K, bench.SEED).kv_summary(K)
+        assert k["valid_bytes_per_step"] == k["physical_bytes_per_step"]
+        assert k["cache_bloat_mean"] == k["cache_bloat_last"] == 1.0
+    # verify: every step appends 5 physical entries and 1 + a valid ones
+    K = 128
+    p = bench.Plan("8b-verify", K, bench.SEED)
+    k = p.kv_summary(K)
+    valid = 512 + sum(1 + synth.accepted_drafts(bench.SEED, t, 4) for t in range(K - 1))
+    phys = 512 + 5 * (K - 1)
+    assert k["cache_bloat_last"] == pytest.approx((phys + 5) / (valid + 5))
+    assert k["physical_bytes_per_step"] > k["valid_bytes_per_step"]
+    assert k["physical_bytes_per_step"] == pytest.approx(
+        np.mean([512 + 5 * t + 5 for t in range(K)]) * KV_ENTRY_BYTES * 16)
+    # the algorithmic bytes count valid entries only
+    assert p.steps[3]["kv_bytes"] < p.steps[3]["kv_phys_bytes"]
