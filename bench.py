@@ -155,6 +155,7 @@ class Plan:
                 acc = self.n
                 if self.n > 1:
                     acc = 1 + synth.accepted_drafts(seed, t, self.n - 1)
+                step["emitted"] = acc * self.B  # tokens the step emits: the accepted drafts and the correction
                 for b in range(self.B):
                     valid[b] += [1] * acc + [0] * (self.n - acc)
                     lens[b] += self.n
@@ -518,6 +519,8 @@ def run_gpu(args, rank: int, world: int):
         },
         "step_alg_bytes": step_bytes,
         "kv": plan.kv_summary(K),
+        # a verify step processes 1 + 4 rows but emits 1 + accepted tokens
+        "emitted_tokens_per_s": replica_throughput(world, sum(plan.steps[t]["emitted"] for t in range(K)), ms / 1e3),
         "roofline": {
             "kernel": "step_kernel (the whole decode step: %d layers in one launch)" % shape.n_layers,
             "bound": "hbm",
@@ -588,7 +591,8 @@ def other_workloads(timeout_s: float = 300.0) -> dict:
             out[cfg] = {"workload": d["config"]["workload"], "value": d["value"], "unit": d["unit"],
                         "ms_per_step": d["ms_per_step"], "steps": d["steps"], "achieved_gbs": rf["achieved"],
                         "frac": rf["frac"], "peak": rf["peak"], "e2e": d["e2e"]["value"], "clocks": d["clocks"],
-                        "gpu_launches": d["gpu_launches"], "kv": d.get("kv"), "wall_s": round(time.time() - t0, 1)}
+                        "gpu_launches": d["gpu_launches"], "kv": d.get("kv"),
+                        "emitted_tokens_per_s": d.get("emitted_tokens_per_s"), "wall_s": round(time.time() - t0, 1)}
         except Exception as e:  # timeout, unparsable output
             out[cfg] = {"error": "%s: %s" % (type(e).__name__, str(e)[:300])}
     return out

@@ -163,3 +163,13 @@ def test_kv_counted_valid_and_physical_with_cache_bloat():
         np.mean([512 + 5 * t + 5 for t in range(K)]) * KV_ENTRY_BYTES * 16)
     # the algorithmic bytes count valid entries only
     assert p.steps[3]["kv_bytes"] < p.steps[3]["kv_phys_bytes"]
+
+
+def test_emitted_tokens_per_step():
+    p = bench.Plan("8b-decode", 8, bench.SEED)
+    assert all(st["emitted"] == 1 for st in p.steps)
+    p = bench.Plan("8b-microbatch", 8, bench.SEED)
+    assert all(st["emitted"] == 8 for st in p.steps)
+    K = 128
+    p = bench.Plan("8b-verify", K, bench.SEED)
+    assert [st["emitted"] for st in p.steps] == [1 + synth.accepted_drafts(bench.SEED, t, 4) for t in range(K)]
