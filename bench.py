@@ -571,15 +571,22 @@ def _child_env():
     return {k: v for k, v in os.environ.items() if k not in LAUNCHER_ENV and not k.startswith("TORCHELASTIC_")}
 
 
-def other_workloads(timeout_s: float = 300.0) -> dict:
+def other_workloads(timeout_s: float = 150.0, total_s: float = 400.0) -> dict:
     """Runs each of OTHER_WORKLOADS in a child process of its own and returns
     its headline figures (or the reason it gave none): a child that fails
-    cannot disturb the main line, which is complete before they start."""
+    cannot disturb the main line, which is complete before they start.  Each
+    child gets timeout_s, all of them together total_s (each took under 30 s
+    on a GB300); children that would start past that are skipped."""
     out = {}
+    start = time.time()
     for cfg, steps in OTHER_WORKLOADS:
         t0 = time.time()
+        left = total_s - (t0 - start)
+        if left < 10.0:
+            out[cfg] = {"error": "skipped: the other workloads' %.0f s were spent" % total_s}
+            continue
         try:
-            r = subprocess.run(_child_cmd(cfg, steps), capture_output=True, text=True, timeout=timeout_s,
+            r = subprocess.run(_child_cmd(cfg, steps), capture_output=True, text=True, timeout=min(timeout_s, left),
                                env=_child_env())
             lines = [ln for ln in r.stdout.splitlines() if ln.startswith("{")]
             if r.returncode != 0 or not lines:

@@ -67,3 +67,10 @@ def test_children_do_not_inherit_launcher_ranks(monkeypatch):
     assert not any(k in env for k in ("RANK", "WORLD_SIZE", "LOCAL_RANK", "MASTER_PORT", "TORCHELASTIC_RUN_ID"))
     cmd = bench._child_cmd("8b-verify", 128)
     assert cmd[-7:] == ["--config", "8b-verify", "--steps", "128", "--warmup", "3", "--no-cpu-baseline"]
+
+
+def test_children_share_one_overall_deadline(monkeypatch):
+    monkeypatch.setattr(bench, "_child_cmd", lambda c, s: [sys.executable, "-c", "import time; time.sleep(30)"])
+    out = bench.other_workloads(timeout_s=2, total_s=13)
+    errs = [out[c]["error"] for c, _ in bench.OTHER_WORKLOADS]
+    assert errs[0].startswith("TimeoutExpired") and any(e.startswith("skipped") for e in errs)
